@@ -1,0 +1,525 @@
+"""Pins of the CPU oracle against facts that do not come from the oracle itself.
+
+Every function raises AssertionError when the oracle disagrees with:
+* the hand-worked examples in tests/golden/worked_examples.json;
+* brute force on tiny inputs (exhaustive pair search, subset enumeration);
+* library routines (torch float64 layer_norm / linear / softmax, numpy stable argsort,
+  numpy cumsum, torch's float32 -> bfloat16 conversion);
+* invariants and special cases that follow from the definitions (conservation of
+  size-weighted mass, r = 0 identity, cosine scale invariance, W = 0 -> max-prob 1/C, ...).
+
+They are plain functions so that tests/test_oracle_mutants.py can run the whole set
+against oracle builds with a planted mistake and check that some pin fails.
+"""
+from __future__ import annotations
+
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import torch
+
+import oracle
+from workloads import Head, bf16_bits_to_f32, f32_to_bf16_bits
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "worked_examples.json")
+
+
+def _golden():
+    with open(GOLDEN) as f:
+        return json.load(f)
+
+
+def _num(v):
+    if isinstance(v, str):
+        if v == "inf":
+            return math.inf
+        return float(eval(v, {"sqrt": math.sqrt, "__builtins__": {}}))  # noqa: S307
+    return float(v)
+
+
+def _one(x):
+    """Offsets of a single-sample batch."""
+    return np.array([0, len(x)], np.int32)
+
+
+# ---------------------------------------------------------------------------
+# brute-force references (tiny inputs only)
+# ---------------------------------------------------------------------------
+def brute_merge(keys, x, sizes, scores, r):
+    """Exhaustive merge of one sample: cosine via numpy norms, argmax by scanning every B
+    candidate, top-r by enumerating all r-subsets of A (largest exact sum, then the
+    lexicographically smallest index set), outputs via a dense assignment matrix."""
+    keys = np.asarray(keys, np.float64)
+    x = np.asarray(x, np.float64)
+    N = len(x)
+    A = [p for p in range(2, N, 2)]
+    Bp = [p for p in range(1, N, 2)]
+    kn = keys / np.maximum(np.linalg.norm(keys, axis=1, keepdims=True), 1e-12)
+    S = kn[A] @ kn[Bp].T if A and Bp else np.zeros((len(A), len(Bp)))
+    match, sbest = [], []
+    for m in range(len(A)):
+        cand = sorted(range(len(Bp)), key=lambda n: (-S[m, n], n))
+        match.append(cand[0])
+        sbest.append(S[m, cand[0]])
+    r_eff = min(max(int(r), 0), len(A))
+    best_set = None
+    for comb in itertools.combinations(range(len(A)), r_eff):
+        key = (math.fsum(sbest[m] for m in comb), tuple(-m for m in comb))
+        if best_set is None or key > best_set[0]:
+            best_set = (key, comb)
+    chosen = set(best_set[1]) if best_set else set()
+    kept = [p for p in range(N) if not (p in A and A.index(p) in chosen)]
+    dest = {}
+    for p in range(N):
+        if p in A and A.index(p) in chosen:
+            dest[p] = kept.index(Bp[match[A.index(p)]])
+        else:
+            dest[p] = kept.index(p)
+    M = np.zeros((len(kept), N))
+    for p in range(N):
+        M[dest[p], p] = sizes[p]
+    Ind = (M > 0).astype(np.float64)
+    x_out = (M @ x) / M.sum(axis=1, keepdims=True)
+    return dict(x=x_out, sizes=M.sum(axis=1), scores=Ind @ np.asarray(scores, np.float64),
+                keep_idx=np.array(kept), dst_map=np.array([dest[p] for p in range(N)]),
+                a_match=np.array([Bp[match[A.index(p)]] if p in A else -1 for p in range(N)]),
+                sbest=np.array(sbest), chosen=sorted(chosen))
+
+
+def brute_prune_keep(scores, rho):
+    """Positions kept by pruning one sample: all k-subsets of the patches, largest exact
+    score sum, then the lexicographically smallest set; CLS always kept."""
+    P = len(scores) - 1
+    k = math.ceil(float(np.float32(rho)) * P)
+    k = min(max(k, 0), P)
+    best = None
+    for comb in itertools.combinations(range(1, P + 1), k):
+        key = (math.fsum(float(scores[p]) for p in comb), tuple(-p for p in comb))
+        if best is None or key > best[0]:
+            best = (key, comb)
+    return [0] + sorted(best[1])
+
+
+# ---------------------------------------------------------------------------
+# conversions
+# ---------------------------------------------------------------------------
+def pin_bf16_rounding_table():
+    """Round-to-nearest-even at the bf16 grid: exact midpoints go to the even neighbour."""
+    cases = {
+        1.0: 0x3F80, -1.0: 0xBF80, 0.0: 0x0000,
+        1.0 + 2 ** -8: 0x3F80,            # midpoint 1 | 1+2^-7 -> even (1.0)
+        1.0 + 3 * 2 ** -8: 0x3F82,        # midpoint 1+2^-7 | 1+2^-6 -> even (1+2^-6)
+        1.0 + 2 ** -8 + 2 ** -30: 0x3F81,  # just above a midpoint -> up
+        1.0 + 2 ** -7: 0x3F81,
+        2.0 ** 128: 0x7F80,               # overflow -> +inf
+        -(2.0 ** 128): 0xFF80,
+        2.0 ** -133: 0x0001,              # smallest bf16 subnormal
+        2.0 ** -134: 0x0000,              # half of it: tie -> even (0)
+        3 * 2.0 ** -135: 0x0001,          # 0.75 of the smallest subnormal -> up
+        2.0 ** -133 + 2.0 ** -134: 0x0002,  # 1.5 subnormal steps: tie -> even (2 steps)
+        5 * 2.0 ** -135: 0x0001,          # 1.25 steps -> 1
+        7 * 2.0 ** -135: 0x0002,          # 1.75 steps -> 2
+    }
+    for v, bits in cases.items():
+        got = oracle.double_to_bf16(v)
+        assert got == bits, f"bf16({v!r}) = {got:#06x}, expected {bits:#06x}"
+    assert oracle.double_to_bf16(-0.0) == 0x8000
+    for bits in (0x3F80, 0x0001, 0x7F7F, 0xC2F7):
+        v = oracle.bf16_to_double(bits)
+        assert oracle.double_to_bf16(v) == bits
+
+
+def pin_bf16_rounding_vs_torch():
+    """On float32 inputs the oracle's rounding equals torch's float32 -> bfloat16 cast."""
+    rng = np.random.default_rng(11)
+    v = np.concatenate([rng.standard_normal(4000).astype(np.float32),
+                        (rng.standard_normal(2000) * 1e-30).astype(np.float32),
+                        (rng.standard_normal(2000) * 1e30).astype(np.float32),
+                        (rng.standard_normal(2000) * 1e-39).astype(np.float32)])
+    # exact midpoints between neighbouring bf16 values
+    b = rng.integers(0x0080, 0x7F00, 1000).astype(np.uint32)
+    mids = ((b << 16) | 0x8000).view(np.float32)
+    v = np.concatenate([v, mids, -mids])
+    ref = torch.from_numpy(v).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    got = np.array([oracle.double_to_bf16(float(t)) for t in v], np.uint16)
+    bad = np.nonzero(got != ref)[0]
+    assert len(bad) == 0, f"{len(bad)} mismatches, first {v[bad[0]]!r}: {got[bad[0]]:#06x} vs {ref[bad[0]]:#06x}"
+
+
+# ---------------------------------------------------------------------------
+# merge
+# ---------------------------------------------------------------------------
+def pin_merge_worked_examples():
+    for ex in _golden()["merge"]:
+        keys = np.array(ex["keys"], np.float32)
+        x = np.array(ex["x"], np.float32)
+        sizes = np.array(ex["sizes"], np.float32)
+        scores = np.linspace(0.01, 0.07, len(x)).astype(np.float32)
+        for case in ex["cases"]:
+            m = oracle.merge("f32", _one(x), x, keys, sizes, scores, np.array([case["r"]], np.int32))
+            exp_x = np.array([[_num(v) for v in row] for row in case["x_out"]], np.float32)
+            assert m["x"].shape == exp_x.shape, (ex["name"], case["r"], m["x"].shape)
+            np.testing.assert_array_equal(m["x"], exp_x, err_msg=f"{ex['name']} r={case['r']}")
+            np.testing.assert_array_equal(m["sizes"], np.array(case["sizes_out"], np.float32))
+            np.testing.assert_array_equal(m["keep_idx"], case["keep_idx"])
+            np.testing.assert_array_equal(m["dst_map"], case["dst_map"])
+            np.testing.assert_array_equal(m["a_match"], ex["a_match"])
+            g = _num(case["topr_gap"])
+            if math.isinf(g):
+                assert math.isinf(m["topr_gap"][0])
+            else:
+                assert abs(m["topr_gap"][0] - g) < 1e-6, (ex["name"], m["topr_gap"][0], g)
+        for pos, expr in ex.get("argmax_gap", {}).items():
+            m = oracle.merge("f32", _one(x), x, keys, sizes, scores, np.array([0], np.int32))
+            assert abs(m["argmax_gap"][int(pos)] - _num(expr)) < 1e-12
+
+
+def _tiny_case(rng, N, dk, d, dtype="f32", dup=False):
+    keys = rng.standard_normal((N, dk)).astype(np.float32)
+    if dup and N > 4:
+        keys[3] = keys[1]          # exact duplicate B tokens -> exact ties
+        keys[4] = keys[1] * 2.0    # same direction, other scale
+    x = rng.standard_normal((N, d)).astype(np.float32)
+    sizes = rng.integers(1, 5, N).astype(np.float32)
+    sizes[0] = 1
+    scores = rng.random(N).astype(np.float32)
+    return keys, x, sizes, scores
+
+
+def pin_merge_brute_force():
+    """Exhaustive search on every N in 1..17 and several r."""
+    rng = np.random.default_rng(5)
+    for N in range(1, 18):
+        for trial in range(3):
+            keys, x, sizes, scores = _tiny_case(rng, N, 5, 3, dup=(trial == 2))
+            nA = (N - 1) // 2
+            for r in sorted({0, 1, nA // 2, nA, nA + 3}):
+                m = oracle.merge("f32", _one(x), x, keys, sizes, scores, np.array([r], np.int32))
+                bf = brute_merge(keys, x, sizes, scores, r)
+                np.testing.assert_array_equal(m["a_match"], bf["a_match"], err_msg=f"N={N} r={r}")
+                np.testing.assert_array_equal(m["keep_idx"], bf["keep_idx"], err_msg=f"N={N} r={r}")
+                np.testing.assert_array_equal(m["dst_map"], bf["dst_map"], err_msg=f"N={N} r={r}")
+                np.testing.assert_allclose(m["x"], bf["x"], rtol=1e-6, atol=1e-6)
+                np.testing.assert_array_equal(m["sizes"], bf["sizes"].astype(np.float32))
+                np.testing.assert_allclose(m["scores"], bf["scores"], rtol=1e-6)
+                # argmax gap: best minus runner-up over B
+                for p in range(2, N, 2):
+                    Bp = list(range(1, N, 2))
+                    kk = keys.astype(np.float64)
+                    kn = kk / np.linalg.norm(kk, axis=1, keepdims=True)
+                    s = np.sort(kn[Bp] @ kn[p])[::-1]
+                    gap = s[0] - s[1] if len(s) > 1 else math.inf
+                    assert (math.isinf(gap) and math.isinf(m["argmax_gap"][p])) or \
+                        abs(m["argmax_gap"][p] - gap) < 1e-12
+
+
+def pin_merge_invariants():
+    """Conservation: per sample, sum(size*x) and sum(size) are unchanged by merging; CLS is
+    untouched; the sample loses exactly r_eff tokens; every input row has a destination."""
+    rng = np.random.default_rng(7)
+    counts = np.array([1, 2, 3, 17, 64, 197, 33])
+    offsets = np.concatenate([[0], np.cumsum(counts)]).astype(np.int32)
+    T = int(offsets[-1])
+    x = rng.standard_normal((T, 24)).astype(np.float32)
+    keys = rng.standard_normal((T, 16)).astype(np.float32)
+    sizes = rng.integers(1, 5, T).astype(np.float32)
+    scores = rng.random(T).astype(np.float32)
+    r = np.array([3, 0, 1, 5, 40, 24, 100], np.int32)
+    m = oracle.merge("f32", offsets, x, keys, sizes, scores, r)
+    for i in range(len(counts)):
+        a, b = offsets[i], offsets[i + 1]
+        oa, ob = m["offsets"][i], m["offsets"][i + 1]
+        r_eff = min(max(int(r[i]), 0), (counts[i] - 1) // 2)
+        assert ob - oa == counts[i] - r_eff
+        mass_in = (sizes[a:b, None].astype(np.float64) * x[a:b]).sum(0)
+        mass_out = (m["sizes"][oa:ob, None].astype(np.float64) * m["x"][oa:ob]).sum(0)
+        scale = np.abs(sizes[a:b, None] * x[a:b]).sum(0).max()
+        assert np.max(np.abs(mass_out - mass_in)) <= 1e-5 * scale
+        assert m["sizes"][oa:ob].sum() == sizes[a:b].sum()
+        s_in = scores[a:b].astype(np.float64).sum()
+        assert abs(m["scores"][oa:ob].astype(np.float64).sum() - s_in) <= 1e-6 * s_in + 1e-12
+        np.testing.assert_array_equal(m["x"][oa], x[a])          # CLS untouched
+        assert m["keep_idx"][oa] == a
+        assert np.all((m["dst_map"][a:b] >= oa) & (m["dst_map"][a:b] < ob))
+        assert np.all(np.diff(m["keep_idx"][oa:ob]) > 0)          # ascending positions
+
+
+def pin_merge_identity_and_equal_keys():
+    """r = 0 is the identity; with all keys equal every A token picks the first B token and
+    the r lowest A positions merge into it (closed-form mean)."""
+    rng = np.random.default_rng(3)
+    N, d = 15, 6
+    x = rng.standard_normal((N, d)).astype(np.float32)
+    sizes = np.ones(N, np.float32)
+    scores = rng.random(N).astype(np.float32)
+    keys = rng.standard_normal((N, 4)).astype(np.float32)
+    m = oracle.merge("f32", _one(x), x, keys, sizes, scores, np.array([0], np.int32))
+    np.testing.assert_array_equal(m["x"], x)
+    np.testing.assert_array_equal(m["dst_map"], np.arange(N))
+    same = np.tile(np.array([[0.5, -1.0, 2.0, 0.25]], np.float32), (N, 1))
+    for r in (1, 3, 7):
+        m = oracle.merge("f32", _one(x), x, same, sizes, scores, np.array([r], np.int32))
+        merged_pos = [2 + 2 * q for q in range(r)]
+        for p in range(2, N, 2):
+            assert m["a_match"][p] == 1
+        expect = (x[1].astype(np.float64) + x[merged_pos].astype(np.float64).sum(0)) / (1 + r)
+        np.testing.assert_allclose(m["x"][1], expect, rtol=1e-6)
+        assert m["sizes"][1] == 1 + r
+        assert list(m["keep_idx"]) == [p for p in range(N) if p not in merged_pos]
+
+
+def pin_merge_scale_invariance():
+    """Cosine similarity ignores each key's length: rescaling keys by positive factors must not
+    change any decision (a path that skips the normalisation fails this)."""
+    rng = np.random.default_rng(9)
+    N = 41
+    keys, x, sizes, scores = _tiny_case(rng, N, 8, 4)
+    factors = np.exp2(rng.integers(-6, 7, N)).astype(np.float32)   # exact power-of-two scales
+    r = np.array([9], np.int32)
+    a = oracle.merge("f32", _one(x), x, keys, sizes, scores, r)
+    b = oracle.merge("f32", _one(x), x, keys * factors[:, None], sizes, scores, r)
+    np.testing.assert_array_equal(a["a_match"], b["a_match"])
+    np.testing.assert_array_equal(a["dst_map"], b["dst_map"])
+    np.testing.assert_array_equal(a["x"], b["x"])
+
+
+def pin_merge_orthogonal_pairs():
+    """Hand-built one-hot keys give a known matching: A token m points at B token pi(m)."""
+    nA = 6
+    perm = [4, 0, 5, 2, 1, 3]
+    N = 1 + 2 * nA
+    keys = np.zeros((N, nA + 1), np.float32)
+    keys[0, nA] = 1.0
+    for n in range(nA):
+        keys[1 + 2 * n, n] = 1.0
+    for m in range(nA):
+        keys[2 + 2 * m, perm[m]] = 1.0 + 0.1 * m
+        keys[2 + 2 * m, nA] = 0.05 * (m + 1)    # unequal best similarities
+    x = np.arange(N * 2, dtype=np.float32).reshape(N, 2)
+    m = oracle.merge("f32", _one(x), x, keys, np.ones(N, np.float32), np.zeros(N, np.float32),
+                     np.array([2], np.int32))
+    for q in range(nA):
+        assert m["a_match"][2 + 2 * q] == 1 + 2 * perm[q]
+    # the two A tokens with the smallest side component have the largest cosines: m = 0, 1
+    assert list(m["keep_idx"]) == [p for p in range(N) if p not in (2, 4)]
+
+
+def pin_merge_bf16_rounding_point():
+    """bf16: the weighted mean is rounded to bf16 once, from the exact mean; keys enter the
+    dot products as stored."""
+    x32 = np.array([[0, 0], [1.0, 3.0], [1.0 + 2 ** -6, 3.0 + 2 ** -6]], np.float32)
+    xb = f32_to_bf16_bits(x32)
+    keys = f32_to_bf16_bits(np.array([[1, 1], [1, 0], [1, 0]], np.float32))
+    m = oracle.merge("bf16", _one(xb), xb, keys, np.ones(3, np.float32), np.zeros(3, np.float32),
+                     np.array([1], np.int32))
+    # mean of 1 and 1+2^-6 is 1+2^-7 (exact, representable); mean of 3 and 3+2^-6 = 3+2^-7 lies
+    # halfway between the bf16 neighbours 3 and 3+2^-6 -> ties to even -> 3.0
+    got = bf16_bits_to_f32(m["x"][1])
+    np.testing.assert_array_equal(got, np.array([1.0 + 2 ** -7, 3.0], np.float32))
+
+
+# ---------------------------------------------------------------------------
+# exit check
+# ---------------------------------------------------------------------------
+def _torch_exit(x_cls64, gamma, beta, eps, W, b, dtype):
+    u = torch.nn.functional.layer_norm(torch.from_numpy(x_cls64), (x_cls64.shape[1],),
+                                       torch.from_numpy(gamma), torch.from_numpy(beta), eps)
+    if dtype == "bf16":
+        u = u.float().bfloat16().double()
+    lg = torch.nn.functional.linear(u, torch.from_numpy(W), torch.from_numpy(b))
+    p = torch.softmax(lg, dim=1)
+    return u.numpy(), lg.numpy(), p.max(dim=1).values.numpy()
+
+
+def pin_exit_vs_torch():
+    """LayerNorm(CLS) -> Linear -> softmax max against torch float64 library routines."""
+    rng = np.random.default_rng(21)
+    for dtype in ("f32", "bf16"):
+        B, N, d, C = 9, 5, 48, 37
+        x32 = (rng.standard_normal((B * N, d)) * 2 + 0.5).astype(np.float32)
+        W32 = (rng.standard_normal((C, d)) * 0.3).astype(np.float32)
+        g32 = (1 + 0.1 * rng.standard_normal(d)).astype(np.float32)
+        b32 = (0.1 * rng.standard_normal(d)).astype(np.float32)
+        bias = (0.2 * rng.standard_normal(C)).astype(np.float32)
+        if dtype == "bf16":
+            xs, Ws, gs, bs = (f32_to_bf16_bits(a) for a in (x32, W32, g32, b32))
+            xf, Wf, gf, bf = (bf16_bits_to_f32(a) for a in (xs, Ws, gs, bs))
+        else:
+            xs, Ws, gs, bs = x32, W32, g32, b32
+            xf, Wf, gf, bf = x32, W32, g32, b32
+        offsets = np.arange(0, B * N + 1, N, dtype=np.int32)
+        head = Head(gs, bs, 1e-6, Ws, bias, 0.5)
+        e = oracle.exit_check(dtype, offsets, xs, head)
+        u, lg, c = _torch_exit(xf[offsets[:-1]].astype(np.float64), gf.astype(np.float64),
+                               bf.astype(np.float64), 1e-6, Wf.astype(np.float64),
+                               bias.astype(np.float64), dtype)
+        if dtype == "bf16":
+            # the bf16 rounding of the LayerNorm output is the (separately pinned) oracle rounding
+            # applied to torch's float64 LayerNorm
+            u_ref = np.array([[oracle.bf16_to_double(oracle.double_to_bf16(v)) for v in row] for row in u])
+            np.testing.assert_array_equal(e["u"], u_ref)
+            lg = torch.nn.functional.linear(torch.from_numpy(u_ref), torch.from_numpy(Wf.astype(np.float64)),
+                                            torch.from_numpy(bias.astype(np.float64))).numpy()
+            c = torch.softmax(torch.from_numpy(lg), dim=1).max(dim=1).values.numpy()
+        else:
+            np.testing.assert_allclose(e["u"], u, rtol=1e-12, atol=1e-12)
+        np.testing.assert_allclose(e["logits"], lg, rtol=1e-6, atol=1e-6)
+        np.testing.assert_allclose(e["max_prob"], c, rtol=1e-6)
+        clear = np.abs(c - 0.5) > 1e-9
+        np.testing.assert_array_equal(e["exit_mask"][clear], (c[clear] >= 0.5).astype(np.uint8))
+        np.testing.assert_allclose(e["exit_gap"], np.abs(c - 0.5), atol=1e-9)
+
+
+def pin_exit_special_cases():
+    """W = 0, b = 0 -> max-prob exactly 1/C; the rule is c >= tau (equality exits);
+    tau <= 1/C -> all exit; tau > 1 -> none; one dominant logit -> c ~ 1;
+    constant CLS (zero variance) -> u = beta."""
+    rng = np.random.default_rng(2)
+    B, d, C = 6, 16, 4
+    x = rng.standard_normal((B, d)).astype(np.float32)
+    offsets = np.arange(B + 1, dtype=np.int32)
+    ones, zeros = np.ones(d, np.float32), np.zeros(d, np.float32)
+    W0 = np.zeros((C, d), np.float32)
+    e = oracle.exit_check("f32", offsets, x, Head(ones, zeros, 1e-6, W0, np.zeros(C, np.float32), 0.25))
+    np.testing.assert_array_equal(e["max_prob"], np.full(B, 0.25, np.float32))
+    assert e["exit_mask"].all()                       # c == tau exits
+    e = oracle.exit_check("f32", offsets, x, Head(ones, zeros, 1e-6, W0, np.zeros(C, np.float32),
+                                                 float(np.nextafter(np.float32(0.25), np.float32(1)))))
+    assert not e["exit_mask"].any()
+    W = (rng.standard_normal((C, d)) * 0.1).astype(np.float32)
+    e = oracle.exit_check("f32", offsets, x, Head(ones, zeros, 1e-6, W, np.zeros(C, np.float32), 0.2))
+    assert e["exit_mask"].all()                       # max-prob >= 1/C always
+    e = oracle.exit_check("f32", offsets, x, Head(ones, zeros, 1e-6, W, np.zeros(C, np.float32), 1.0001))
+    assert not e["exit_mask"].any()
+    bias = np.array([0, 60, 0, 0], np.float32)
+    e = oracle.exit_check("f32", offsets, x, Head(ones, zeros, 1e-6, W, bias, 0.999))
+    assert e["exit_mask"].all() and np.all(e["max_prob"] > 0.999)
+    xc = np.full((B, d), 3.5, np.float32)
+    beta = rng.standard_normal(d).astype(np.float32)
+    e = oracle.exit_check("f32", offsets, xc, Head(ones, beta, 1e-6, W, np.zeros(C, np.float32), 0.5))
+    np.testing.assert_allclose(e["u"], np.tile(beta, (B, 1)), rtol=0, atol=0)
+
+
+# ---------------------------------------------------------------------------
+# prune
+# ---------------------------------------------------------------------------
+def pin_prune_worked_examples():
+    for ex in _golden()["prune"]:
+        s = np.array(ex["scores"], np.float32)
+        N = len(s)
+        x = np.arange(N * 3, dtype=np.float32).reshape(N, 3)
+        sizes = np.arange(1, N + 1, dtype=np.float32)
+        p = oracle.prune("f32", _one(x), x, sizes, s, np.array([ex["rho"]], np.float32))
+        assert list(p["keep_idx"]) == ex["keep_idx"], (ex["name"], p["keep_idx"])
+        np.testing.assert_array_equal(p["x"], x[ex["keep_idx"]])
+        np.testing.assert_array_equal(p["sizes"], sizes[ex["keep_idx"]])
+        if "rho_one_keep_idx" in ex:
+            p = oracle.prune("f32", _one(x), x, sizes, s, np.array([1.0], np.float32))
+            assert list(p["keep_idx"]) == ex["rho_one_keep_idx"]
+
+
+def pin_prune_brute_force_and_argsort():
+    """Subset enumeration (P <= 16) and numpy's stable argsort agree with the oracle's keep set
+    and count k = ceil(rho * P)."""
+    rng = np.random.default_rng(13)
+    for P in range(0, 17):
+        for trial in range(4):
+            N = P + 1
+            s = rng.random(N).astype(np.float32)
+            if trial == 1:
+                s = np.round(s * 4).astype(np.float32) / 4     # many exact ties
+            rho = np.float32(rng.random()) if trial < 3 else np.float32(1.0)
+            x = rng.standard_normal((N, 2)).astype(np.float32)
+            p = oracle.prune("f32", _one(x), x, np.ones(N, np.float32), s, np.array([rho], np.float32))
+            expect = brute_prune_keep(s, rho)
+            assert list(p["keep_idx"]) == expect, (P, trial, p["keep_idx"], expect)
+            k = min(max(math.ceil(float(rho) * P), 0), P)
+            order = np.argsort(-s[1:].astype(np.float64), kind="stable")[:k] + 1
+            assert list(p["keep_idx"]) == [0] + sorted(order.tolist())
+
+
+# ---------------------------------------------------------------------------
+# compact and the composed stage
+# ---------------------------------------------------------------------------
+def pin_compact_examples():
+    for ex in _golden()["compact"]:
+        off = np.array(ex["offsets"], np.int32)
+        T = int(off[-1])
+        x = np.arange(T * 2, dtype=np.float32).reshape(T, 2)
+        c = oracle.compact("f32", off, x, np.ones(T, np.float32), np.zeros(T, np.float32),
+                           np.array(ex["exit_mask"], np.uint8))
+        assert list(c["offsets"]) == ex["offsets_out"]
+        assert list(c["ids"]) == ex["ids_out"]
+        assert list(c["keep_idx"]) == ex["keep_idx"]
+        np.testing.assert_array_equal(c["x"], x[ex["keep_idx"]])
+    rng = np.random.default_rng(4)
+    counts = rng.integers(1, 9, 50)
+    off = np.concatenate([[0], np.cumsum(counts)]).astype(np.int32)
+    T = int(off[-1])
+    x = rng.standard_normal((T, 3)).astype(np.float32)
+    for mask in (np.zeros(50, np.uint8), np.ones(50, np.uint8), (rng.random(50) < 0.4).astype(np.uint8)):
+        ids = rng.permutation(1000)[:50].astype(np.int32)
+        c = oracle.compact("f32", off, x, np.ones(T, np.float32), None, mask, ids)
+        surv = np.nonzero(mask == 0)[0]
+        np.testing.assert_array_equal(c["offsets"], np.concatenate([[0], np.cumsum(counts[surv])]))
+        np.testing.assert_array_equal(c["ids"], ids[surv])
+        assert c["n_out"] == len(surv)
+
+
+def pin_stage_exit_sees_merged_cls():
+    """Merging never moves CLS, so the exit check on merged tokens equals the exit check on
+    the stage input bit for bit (the CUDA path relies on this identity)."""
+    from workloads import make_workload
+    w = make_workload("ragged_b8192_n65_chain4_bf16", batch=64)
+    b, spec = w.batch, w.stages[0]
+    m = oracle.merge("bf16", b.offsets, b.x, b.keys, b.sizes, b.scores, spec.r)
+    e1 = oracle.exit_check("bf16", m["offsets"], m["x"], spec.head)
+    e0 = oracle.exit_check("bf16", b.offsets, b.x, spec.head)
+    for k in ("exit_mask", "logits", "max_prob"):
+        np.testing.assert_array_equal(e0[k], e1[k])
+    assert 0 < e0["exit_mask"].sum() < 64
+
+
+def pin_stage_composition():
+    """The stage equals merge -> exit -> (drop exited) -> prune, and every output row that no
+    merge touched is a verbatim copy of its input row."""
+    from workloads import make_workload
+    w = make_workload("ragged_b8192_n65_chain4_f32", batch=40)
+    b, spec = w.batch, w.stages[0]
+    res = oracle.stage(b, spec)
+    m = oracle.merge("f32", b.offsets, b.x, b.keys, b.sizes, b.scores, spec.r)
+    surv = np.nonzero(res["exit_mask"] == 0)[0]
+    assert res["n_out"] == len(surv)
+    np.testing.assert_array_equal(res["ids"], surv)
+    k = 0
+    for j, i in enumerate(surv):
+        n_merged = m["offsets"][i + 1] - m["offsets"][i]
+        kk = min(max(math.ceil(float(spec.rho[i]) * (n_merged - 1)), 0), n_merged - 1)
+        assert res["offsets"][j + 1] - res["offsets"][j] == 1 + kk
+        k += 1 + kk
+    assert res["offsets"][-1] == k
+    untouched = res["sizes"] == b.sizes[res["keep_idx"]]
+    np.testing.assert_array_equal(res["x"][untouched], b.x[res["keep_idx"][untouched]])
+
+
+ALL_PINS = [
+    pin_bf16_rounding_table,
+    pin_bf16_rounding_vs_torch,
+    pin_merge_worked_examples,
+    pin_merge_brute_force,
+    pin_merge_invariants,
+    pin_merge_identity_and_equal_keys,
+    pin_merge_scale_invariance,
+    pin_merge_orthogonal_pairs,
+    pin_merge_bf16_rounding_point,
+    pin_exit_vs_torch,
+    pin_exit_special_cases,
+    pin_prune_worked_examples,
+    pin_prune_brute_force_and_argsort,
+    pin_compact_examples,
+    pin_stage_exit_sees_merged_cls,
+    pin_stage_composition,
+]

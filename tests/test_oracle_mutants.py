@@ -1,0 +1,70 @@
+"""Each planted mistake in the oracle must trip at least one pin.
+
+The mutants are built from a copy of oracle/fusion_oracle.c with one textual change
+each (a dropped term, a wrong sign or index, a flipped comparison, a wrong tie rule),
+compiled with gcc into a temporary directory, and run on the CPU only.
+"""
+import ctypes
+import os
+import subprocess
+import sys
+
+import pytest
+
+sys.path.insert(0, os.path.dirname(os.path.abspath(__file__)))
+
+import oracle  # noqa: E402
+from oracle_pins import ALL_PINS  # noqa: E402
+
+MUTANTS = {
+    "bf16_round_half_up": ("frac > 0.5 || (frac == 0.5 && fmod(whole, 2.0) == 1.0)", "frac >= 0.5"),
+    "bf16_subnormal_spacing": ("lead = -126;", "lead = -127;"),
+    "argmax_ties_to_last": ("if (s > bv) {", "if (s >= bv) {"),
+    "b_index_off_by_one": ("khat[(int64_t)pb * dk + j]", "khat[(int64_t)(pb + 1 < N ? pb + 1 : pb) * dk + j]"),
+    "no_key_normalisation": ("double inv = 1.0 / (nrm > 1e-12 ? nrm : 1e-12);", "double inv = 1.0;"),
+    "sort_ties_to_last": ("(val[idx[j]] == val[cur] && idx[j] > cur)", "(val[idx[j]] == val[cur] && idx[j] < cur)"),
+    "unweighted_size_sum": ("wsum += sizes[ra];", "wsum += 1.0;"),
+    "unweighted_mean": ("num[j] += (double)sizes[ra] * load_elem", "num[j] += load_elem"),
+    "dropped_score_sum": ("ssum += scores[ra];", ";"),
+    "a_match_wrong_row": ("(int32_t)(base + 1 + 2 * match[(p - 2) / 2])", "(int32_t)(base + 2 * match[(p - 2) / 2])"),
+    "unbiased_variance": ("var /= d;", "var /= (d - 1);"),
+    "ln_without_eps": ("1.0 / sqrt(var + eps)", "1.0 / sqrt(var)"),
+    "ln_no_bf16_rounding": ("v = bf16_to_double(double_to_bf16(v));", "v = v;"),
+    "dropped_bias": ("l[k] = acc + (double)bias[k];", "l[k] = acc;"),
+    "softmax_no_shift": ("S += exp(l[k] - lmax);", "S += exp(l[k]);"),
+    "exit_strict_compare": ("(c >= tau) ? 1 : 0", "(c > tau) ? 1 : 0"),
+    "prune_floor": ("double kk = ceil((double)rho[i] * (double)P);", "double kk = floor((double)rho[i] * (double)P);"),
+    "prune_drops_cls": ("if (p > 0 && !kept[p - 1])", "if (p == 0 || !kept[p - 1])"),
+    "compact_keeps_exited": ("if (exit_mask[i])\n            continue;", "if (0)\n            continue;"),
+}
+
+
+def _build_mutant(tmp_path, name, old, new):
+    with open(os.path.join(os.path.dirname(oracle.__file__), "fusion_oracle.c")) as f:
+        src = f.read()
+    assert src.count(old) >= 1, f"mutation site for {name} not found"
+    src = src.replace(old, new)
+    c = tmp_path / f"{name}.c"
+    so = tmp_path / f"lib{name}.so"
+    c.write_text(src)
+    subprocess.check_call(["gcc", "-O1", "-std=c11", "-fPIC", "-shared", "-o", str(so), str(c), "-lm"])
+    return oracle.configure(ctypes.CDLL(str(so)))
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_is_caught(name, tmp_path):
+    old, new = MUTANTS[name]
+    lib = _build_mutant(tmp_path, name, old, new)
+    saved = oracle._load()
+    oracle._lib = lib
+    caught = None
+    try:
+        for pin in ALL_PINS:
+            try:
+                pin()
+            except (AssertionError, RuntimeError) as e:
+                caught = (pin.__name__, str(e)[:120])
+                break
+    finally:
+        oracle._lib = saved
+    assert caught is not None, f"no pin caught the planted mistake {name}"

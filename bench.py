@@ -1,0 +1,441 @@
+#!/usr/bin/env python
+"""Benchmark of the Fusion staged token-adaptation path on GB300.
+
+A step is one pass of the whole path over one synthetic batch: the DeiT-S
+12-block schedule (batch 256, N = 197, d = 384, bf16), merging at every block and
+exit-check -> compaction -> pruning at blocks 4, 6, 8 and 10; the survivors of
+stage s are the input of stage s+1.  There is no transformer block between
+stages, so the L2 cache is flushed (a 512 MB write, untimed) before every stage
+and every stage reads its input from HBM, as it would after a real block.
+
+value     images/s per stage: images entering each stage, summed over the step's
+          stages and over all ranks, divided by the (max over ranks) sum of the
+          stages' CUDA-event times.
+roofline  the per-sample kernel (merge + prune + gather), which moves almost all
+          bytes: algorithmic bytes / event-timed duration vs the measured HBM copy
+          bandwidth.
+e2e       the same metric through the public C ABI with host buffers: pinned
+          host -> device copy of the step's inputs, the chain, device -> host read
+          of the results, all inside the timed region.
+
+--impl reference times the CPU oracle (the only other implementation of the
+method here) on the host cores, on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "images/s per merge→exit→prune stage (DeiT-S, b256); % of HBM roofline"
+UNIT = "images/s"
+DEFAULT_WORKLOAD = "deit_s_chain12_bf16_b256"
+FLUSH_BYTES = 512 << 20
+KERNELS_PER_STAGE = 2      # plan or exit check, then the per-sample kernel
+
+
+def parse_args():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--e2e-steps", type=int, default=None)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--ref-sample", type=int, default=16, help="images per reference step")
+    return ap.parse_args()
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+def source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2607_02612_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(f.encode() + fh.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload: str):
+    """DRAM bytes per launch of the per-sample kernel from the committed ncu summary,
+    only if it was taken on the current kernel sources."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            t = json.load(f)
+    except (OSError, ValueError):
+        return None
+    e = t.get(workload)
+    if not e or e.get("source_hash") != source_hash():
+        return None
+    return e
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or not self.path:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(n)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------------------
+# algorithmic bytes (compulsory traffic) of one stage, from its inputs and outputs
+# ---------------------------------------------------------------------------
+def stage_bytes(spec, dtype, dim, in_off, in_ids, out_off, out_ids, classes):
+    eb = 2 if dtype == "bf16" else 4
+    B_in = len(in_off) - 1
+    B_out = len(out_off) - 1
+    counts_in = np.diff(in_off).astype(np.int64)
+    counts_out = np.diff(out_off).astype(np.int64)
+    surv = {int(t): j for j, t in enumerate(out_ids)}
+    first = 0
+    if spec.exit:
+        first += B_in * dim * eb + classes * dim * eb + classes * 4 + 2 * dim * eb   # CLS rows, W, b, gamma/beta
+        first += B_in * (classes * 4 + 1 + 4)                                        # logits, mask, max-prob
+    first += (B_in + 1) * 4 + B_in * 8 + B_out * 12 + 4                              # offsets, r/rho, plan outputs
+    image = 0
+    for i in range(B_in):
+        t = int(in_ids[i])
+        if t not in surv:
+            continue
+        n_in = int(counts_in[i])
+        n_out = int(counts_out[surv[t]])
+        r_eff = min(max(int(spec.r[t]), 0), (n_in - 1) // 2) if spec.merge else 0
+        rows_read = n_in if r_eff > 0 else n_out     # all keys (= tokens) are needed to decide a merge
+        image += rows_read * dim * eb + n_in * 8 + 16                                # tokens, sizes+scores, scalars
+        image += n_out * (dim * eb + 12)                                            # tokens, size, score, row id
+    return first, image
+
+
+# ---------------------------------------------------------------------------
+# reference arm: the CPU oracle
+# ---------------------------------------------------------------------------
+def run_reference(args, world, rank):
+    if rank != 0:
+        return 0
+    import oracle
+    from workloads import make_workload
+    w = make_workload(args.workload)
+    n = min(args.ref_sample, w.batch.batch)
+    sub = make_workload(args.workload, batch=n)
+    units = 0
+    t_total = 0.0
+    for k in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        res = oracle.chain(sub)
+        dt = time.perf_counter() - t0
+        if k >= args.warmup:
+            t_total += dt
+            units += n + sum(int(r["n_out"]) for r in res[:-1])
+    value = units / t_total if t_total > 0 else 0.0
+    sample = f"{n} of {w.batch.batch} images per step, full {len(w.stages)}-stage schedule, one thread"
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t_total / max(args.steps, 1),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f64", "data": "synthetic",
+            "config": {"workload": args.workload, "batch": w.batch.batch, "sample_batch": n},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def cpu_baseline(workload_name: str):
+    import oracle
+    from workloads import make_workload
+    w = make_workload(workload_name)
+    n = min(w.batch.batch, 256)
+    sub = make_workload(workload_name, batch=n) if n != w.batch.batch else w
+    t0 = time.perf_counter()
+    res = oracle.chain(sub)
+    dt = time.perf_counter() - t0
+    units = n + sum(int(r["n_out"]) for r in res[:-1])
+    return {"value": units / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{n} of {w.batch.batch} images, one full {len(w.stages)}-stage schedule "
+                      f"({dt:.1f} s, single thread)"}
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+def main():
+    args = parse_args()
+    world, rank, local = dist_env()
+    if args.impl == "reference":
+        return run_reference(args, world, rank)
+
+    import torch
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    import paper_2607_02612_gb300 as fz
+    from paper_2607_02612_gb300 import runner
+    from workloads import make_workload
+
+    fz.build()
+    lib = fz.load()
+    assert lib is not None
+
+    # cpu baseline first (before any GPU work forks nothing; single thread)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(args.workload)
+
+    w = make_workload(args.workload, seed_offset=rank)
+    b = w.batch
+    specs = w.stages
+    classes = max([s.head.classes for s in specs if s.head is not None] + [1])
+    fus = runner.Fusion(b.batch, classes, dev)
+    db = runner.device_batch(b.dtype, b.offsets, b.x, b.keys, b.sizes, b.scores, device=dev)
+    cst = []
+    for s in specs:
+        r = torch.from_numpy(s.r).to(dev) if s.r is not None else None
+        rho = torch.from_numpy(s.rho).to(dev) if s.rho is not None else None
+        head = runner.head_tensors(s.head, b.dtype, dev) if s.head is not None else None
+        flags = ((fz.FUSION_STAGE_MERGE if s.merge else 0) | (fz.FUSION_STAGE_EXIT if s.exit else 0) |
+                 (fz.FUSION_STAGE_PRUNE if s.prune else 0))
+        cst.append(runner.ChainStage(flags, r, rho, head))
+    chain = runner.Chain(fus, db, cst)
+    for o in chain.outs:           # row ids are not needed by the next block
+        o["keep_idx"] = None
+    S = len(cst)
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    def run_step(evs):
+        for s in range(S):
+            flush.fill_(s & 0xFF)
+            fz.fusion_profile_next(*evs[s])
+            chain.run_stage(s)
+
+    mk = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    warm_evs = [(mk(), mk(), mk()) for _ in range(S)]
+    for _ in range(args.warmup):
+        run_step(warm_evs)
+    torch.cuda.synchronize()
+    st = int(fus.status.item())
+    if st != 0:
+        raise SystemExit(f"device status {st} ({fz.fusion_status_string(st)})")
+
+    evs = [[(mk(), mk(), mk()) for _ in range(S)] for _ in range(args.steps)]
+    barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        t0 = time.perf_counter()
+        for k in range(args.steps):
+            run_step(evs[k])
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+    barrier()
+    stage_ms = np.array([[evs[k][s][0].elapsed_time(evs[k][s][2]) for s in range(S)] for k in range(args.steps)])
+    first_ms = np.array([[evs[k][s][0].elapsed_time(evs[k][s][1]) for s in range(S)] for k in range(args.steps)])
+    image_ms = np.array([[evs[k][s][1].elapsed_time(evs[k][s][2]) for s in range(S)] for k in range(args.steps)])
+    clocks = clk.summary()
+
+    # images entering each stage and algorithmic bytes, from the (deterministic) outputs
+    in_off, in_ids = b.offsets, np.arange(b.batch, dtype=np.int32)
+    units_step = 0
+    bytes_first = bytes_image = 0
+    per_stage = []
+    for s in range(S):
+        o = chain.outs[s]
+        nb = int(o["batch"].item())
+        out_off = o["offsets"][:nb + 1].cpu().numpy()
+        out_ids = o["ids"][:nb].cpu().numpy()
+        f1, im = stage_bytes(specs[s], b.dtype, b.dim, in_off, in_ids, out_off, out_ids,
+                             specs[s].head.classes if specs[s].head is not None else 0)
+        bytes_first += f1
+        bytes_image += im
+        units_step += len(in_off) - 1
+        per_stage.append({"stage": s + 1, "images_in": len(in_off) - 1, "tokens_in": int(in_off[-1]),
+                          "ms": float(np.median(stage_ms[:, s])), "image_kernel_ms": float(np.median(image_ms[:, s])),
+                          "image_kernel_bytes": im})
+        in_off, in_ids = out_off, out_ids
+
+    step_ms = stage_ms.sum(axis=1)
+    total_ms = float(step_ms.sum())
+    units = units_step * args.steps
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([total_ms], device=dev)
+        u = torch.tensor([float(units)], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        dist.all_reduce(u, op=dist.ReduceOp.SUM)
+        total_ms, units = float(t.item()), float(u.item())
+    value = units / (total_ms / 1e3)
+    peak, peak_src = peaks()
+    img_s = float(image_ms.sum()) / 1e3
+    achieved = bytes_image * args.steps / img_s / 1e9
+    step_achieved = (bytes_first + bytes_image) * args.steps / (float(stage_ms.sum()) / 1e3) / 1e9
+    tr = recorded_traffic(args.workload)
+
+    # ---- end to end through the C ABI with host buffers -------------------------------
+    e2e = run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world)
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": b.dtype, "data": "synthetic",
+        "config": {"workload": args.workload, "batch": b.batch, "tokens": int(np.diff(b.offsets).max()),
+                   "dim": b.dim, "stages": S, "exit_blocks": list(w.spec.exit_blocks),
+                   "l2": "flushed before every stage (512 MB write, untimed)",
+                   "timing": "CUDA events around each stage's kernels, summed"},
+        "roofline": {"bound": "hbm", "kernel": "k_image (merge + prune + gather)", "achieved": achieved,
+                     "peak": peak, "unit": "GB/s", "frac": achieved / peak, "peak_source": peak_src,
+                     "traffic": (tr["dram_bytes_per_launch"] if tr else None),
+                     "algorithmic_bytes_per_launch": bytes_image / S,
+                     "whole_step_frac": step_achieved / peak},
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": KERNELS_PER_STAGE * S * args.steps,
+        "clocks": clocks,
+        "stages": per_stage,
+        "kernel_ms_per_step": {"first (exit check or plan)": float(first_ms.sum(axis=1).mean()),
+                               "k_image": float(image_ms.sum(axis=1).mean())},
+        "wall_s_timed_region": wall,
+        "images_per_s_full_schedule": b.batch * world / (total_ms / args.steps / 1e3),
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world):
+    """Host inputs -> device -> chain -> host results, timed together."""
+    import torch
+    steps = args.e2e_steps or max(3, min(args.steps, 10))
+    db = chain.inp
+    host = {
+        "x": torch.from_numpy(np.ascontiguousarray(b.x).view(np.int16) if b.dtype == "bf16" else b.x).pin_memory(),
+        "sizes": torch.from_numpy(b.sizes).pin_memory(),
+        "scores": torch.from_numpy(b.scores).pin_memory(),
+        "offsets": torch.from_numpy(b.offsets).pin_memory(),
+    }
+    dst = {"x": db.x.view(torch.int16) if b.dtype == "bf16" else db.x, "sizes": db.sizes, "scores": db.scores,
+           "offsets": db.offsets}
+    h2d = sum(t.numel() * t.element_size() for t in host.values())
+    last = chain.outs[-1]
+    exit_outs = [o for o in chain.outs if o["exit_mask"] is not None]
+    d2h_bytes = []
+
+    def one():
+        for k in host:
+            dst[k].copy_(host[k], non_blocking=True)
+        chain.run()
+        nb = int(last["batch"].item())                       # the result's size, then the result
+        rows = int(last["offsets"][nb].item())
+        res = [last["offsets"][:nb + 1].cpu(), last["ids"][:nb].cpu(), last["sizes"][:rows].cpu(),
+               last["x"][:rows].cpu()]
+        for o in exit_outs:
+            res += [o["exit_mask"].cpu(), o["max_prob"].cpu()]
+        d2h_bytes.append(sum(t.numel() * t.element_size() for t in res))
+        return res
+
+    for _ in range(2):
+        one()
+    torch.cuda.synchronize()
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        one()
+    torch.cuda.synchronize()
+    dt = time.perf_counter() - t0
+    barrier()
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([dt], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        dt = float(t.item())
+    return {"value": units_step * steps * world / dt, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+            "d2h_bytes_per_step": int(d2h_bytes[-1]), "steps": steps,
+            "note": "pinned host inputs, C-ABI chain (no L2 flush), host reads the survivor count then the results"}
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,385 @@
+// C ABI of the Fusion library: argument checks, workspace carving and kernel
+// launches.  Every call validates on the host first and enqueues nothing when a
+// check fails.
+#include <stdint.h>
+
+#include "launch.h"
+
+using namespace fz;
+
+namespace {
+
+constexpr const char *kVersion = "fusion-gb300 0.1.0 (sm_103a)";
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int check_dtype(int dtype) {
+    return (dtype == FUSION_F32 || dtype == FUSION_BF16) ? FUSION_OK : FUSION_ERR_DTYPE;
+}
+
+int check_dim(int32_t d) {
+    return (d >= 16 && d <= FUSION_MAX_DIM && d % 16 == 0) ? FUSION_OK : FUSION_ERR_SHAPE;
+}
+
+int check_ragged(const fusion_ragged &in) {
+    if (!in.offsets) return FUSION_ERR_INVALID_ARG;
+    if (in.max_batch < 0 || in.max_tokens < 1 || in.max_tokens > FUSION_MAX_TOKENS) return FUSION_ERR_SHAPE;
+    if (in.max_rows < 0 || in.max_rows > INT32_MAX) return FUSION_ERR_SHAPE;
+    return FUSION_OK;
+}
+
+int check_workspace(const void *ws, size_t bytes, int32_t max_batch, int32_t classes) {
+    if (!ws || !aligned16(ws)) return FUSION_ERR_WORKSPACE;
+    return bytes >= ws_layout(max_batch, classes).total ? FUSION_OK : FUSION_ERR_WORKSPACE;
+}
+
+int check_head(const fusion_exit_head &h) {
+    if (!h.ln_gamma || !h.ln_beta || !h.weight || !h.bias) return FUSION_ERR_INVALID_ARG;
+    if (!aligned16(h.ln_gamma) || !aligned16(h.ln_beta) || !aligned16(h.weight)) return FUSION_ERR_INVALID_ARG;
+    if (h.classes < 1) return FUSION_ERR_SHAPE;
+    return FUSION_OK;
+}
+
+Ragged dev(const fusion_ragged &in) {
+    return Ragged{in.max_batch, in.max_tokens, (long long)in.max_rows, in.offsets, in.batch, in.ids};
+}
+
+Head dev(const fusion_exit_head &h) {
+    return Head{h.ln_gamma, h.ln_beta, h.ln_eps, h.weight, h.bias, h.classes, h.tau};
+}
+
+struct Ws {
+    int *slot;
+    int *plan;
+    int *counters;
+    float2 *partials;
+};
+
+Ws carve(void *ws, int32_t max_batch, int32_t classes) {
+    const WsLayout L = ws_layout(max_batch, classes);
+    unsigned char *b = static_cast<unsigned char *>(ws);
+    return Ws{reinterpret_cast<int *>(b + L.slot), reinterpret_cast<int *>(b + L.plan),
+              reinterpret_cast<int *>(b + L.counters), reinterpret_cast<float2 *>(b + L.partials)};
+}
+
+int cuda_rc(cudaError_t e) { return e == cudaSuccess ? FUSION_OK : FUSION_ERR_CUDA; }
+
+// Events armed by fusion_profile_next() for the next call of this host thread.
+struct ProfileEvents {
+    cudaEvent_t start = nullptr, mid = nullptr, end = nullptr;
+};
+thread_local ProfileEvents g_profile;
+
+// Takes the armed events (if any) for the call that is starting.
+ProfileEvents take_profile() {
+    ProfileEvents e = g_profile;
+    g_profile = ProfileEvents{};
+    return e;
+}
+
+void record(cudaEvent_t e, cudaStream_t s) {
+    if (e) cudaEventRecord(e, s);
+}
+
+#define FZ_TRY(expr)                    \
+    do {                                \
+        const int rc_ = (expr);         \
+        if (rc_ != FUSION_OK) return rc_; \
+    } while (0)
+
+ImageParams image_params(const fusion_ragged &in, const void *x, int32_t dim, const void *keys,
+                         int32_t key_dim, const float *sizes, const float *scores, const int32_t *r,
+                         const float *rho, int do_merge, int do_prune, const Ws &w,
+                         const int32_t *offsets_out, void *x_out, float *sizes_out, float *scores_out,
+                         int32_t *keep_idx, int32_t *dst_map, int32_t *a_match, int32_t *status,
+                         const ImageGeometry &G) {
+    ImageParams p{};
+    p.in = dev(in);
+    p.x = x;
+    p.keys = keys ? keys : x;
+    p.dim = dim;
+    p.kdim = keys ? key_dim : dim;
+    p.keys_alias = (keys == nullptr || keys == x) && p.kdim == dim;
+    p.sizes = sizes;
+    p.scores = scores;
+    p.r = r;
+    p.rho = rho;
+    p.do_merge = do_merge;
+    p.do_prune = do_prune;
+    p.need_match = a_match != nullptr;
+    p.slot = w.slot;
+    p.plan = w.plan;
+    p.offsets_out = offsets_out;
+    p.x_out = x_out;
+    p.sizes_out = sizes_out;
+    p.scores_out = scores_out;
+    p.keep_idx = keep_idx;
+    p.dst_map = dst_map;
+    p.a_match = a_match;
+    p.status = status;
+    p.resident = G.resident;
+    p.kc = G.kc;
+    p.ra = G.ra;
+    p.rb = G.rb;
+    return p;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *fusion_version(void) { return kVersion; }
+
+int fusion_profile_next(void *start, void *mid, void *end) {
+    g_profile.start = static_cast<cudaEvent_t>(start);
+    g_profile.mid = static_cast<cudaEvent_t>(mid);
+    g_profile.end = static_cast<cudaEvent_t>(end);
+    return FUSION_OK;
+}
+
+const char *fusion_status_string(int code) {
+    switch (code) {
+        case FUSION_OK: return "ok";
+        case FUSION_ERR_INVALID_ARG: return "invalid argument (NULL, misaligned pointer or bad flags)";
+        case FUSION_ERR_SHAPE: return "shape out of range (dim, key_dim, max_tokens, classes, batch)";
+        case FUSION_ERR_DTYPE: return "unsupported dtype";
+        case FUSION_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+        case FUSION_ERR_CUDA: return "CUDA error";
+        case FUSION_DEV_BAD_OFFSETS: return "device: malformed offsets";
+        case FUSION_DEV_BAD_BATCH: return "device: batch count out of range";
+        case FUSION_DEV_NONFINITE: return "device: NaN or Inf in a decision input";
+        case FUSION_DEV_INTERNAL: return "device: internal consistency check failed";
+        case FUSION_DEV_BAD_IDS: return "device: sample id out of range";
+        default: return "unknown status";
+    }
+}
+
+size_t fusion_workspace_size(int32_t max_batch, int32_t classes) {
+    return ws_layout(max_batch < 0 ? 0 : max_batch, classes < 1 ? 1 : classes).total;
+}
+
+int fusion_merge(int dtype, fusion_ragged in, const void *x, int32_t dim, const void *keys,
+                 int32_t key_dim, const float *sizes, const float *scores, const int32_t *r,
+                 void *x_out, float *sizes_out, float *scores_out, int32_t *offsets_out,
+                 int32_t *keep_idx, int32_t *dst_map, int32_t *a_match, void *workspace,
+                 size_t workspace_bytes, int32_t *dev_status, void *stream) {
+    FZ_TRY(check_dtype(dtype));
+    FZ_TRY(check_ragged(in));
+    FZ_TRY(check_dim(dim));
+    if (!keys) return FUSION_ERR_INVALID_ARG;
+    FZ_TRY(check_dim(key_dim));
+    if (!x || !sizes || !r || !x_out || !sizes_out || !offsets_out) return FUSION_ERR_INVALID_ARG;
+    if ((scores == nullptr) != (scores_out == nullptr)) return FUSION_ERR_INVALID_ARG;
+    if (!aligned16(x) || !aligned16(keys) || !aligned16(x_out)) return FUSION_ERR_INVALID_ARG;
+    FZ_TRY(check_workspace(workspace, workspace_bytes, in.max_batch, 1));
+    const ImageGeometry G = image_geometry(dtype, in.max_tokens, key_dim, 1);
+    if (!G.ok) return FUSION_ERR_SHAPE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const Ws w = carve(workspace, in.max_batch, 1);
+    const ProfileEvents ev = take_profile();
+
+    PlanArgs pa{};
+    pa.in = dev(in);
+    pa.merge = 1;
+    pa.r = r;
+    pa.offsets_out = offsets_out;
+    pa.slot = w.slot;
+    pa.plan = w.plan;
+    pa.status = dev_status;
+    record(ev.start, s);
+    FZ_TRY(cuda_rc(launch_plan(pa, s)));
+    record(ev.mid, s);
+    const ImageParams p = image_params(in, x, dim, keys, key_dim, sizes, scores, r, nullptr, 1, 0, w,
+                                       offsets_out, x_out, sizes_out, scores_out, keep_idx, dst_map,
+                                       a_match, dev_status, G);
+    const int rc = cuda_rc(launch_image(dtype, p, G.smem, s));
+    record(ev.end, s);
+    return rc;
+}
+
+int fusion_exit_check(int dtype, fusion_ragged in, const void *x, int32_t dim,
+                      fusion_exit_head head, uint8_t *exit_mask, float *logits, float *max_prob,
+                      void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream) {
+    FZ_TRY(check_dtype(dtype));
+    FZ_TRY(check_ragged(in));
+    FZ_TRY(check_dim(dim));
+    FZ_TRY(check_head(head));
+    if (!x || !exit_mask || !aligned16(x)) return FUSION_ERR_INVALID_ARG;
+    FZ_TRY(check_workspace(workspace, workspace_bytes, in.max_batch, head.classes));
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const Ws w = carve(workspace, in.max_batch, head.classes);
+    ExitParams e{};
+    e.in = dev(in);
+    e.x = x;
+    e.dim = dim;
+    e.head = dev(head);
+    e.exit_mask = exit_mask;
+    e.logits = logits;
+    e.max_prob = max_prob;
+    e.counters = w.counters;
+    e.partials = w.partials;
+    e.n_ctile = ceil_div(head.classes, kExitCT);
+    e.n_btile = ceil_div(in.max_batch > 0 ? in.max_batch : 1, kExitBT);
+    e.do_plan = 0;
+    e.status = dev_status;
+    const ProfileEvents ev = take_profile();
+    record(ev.start, s);
+    const int rc = cuda_rc(launch_exit(dtype, e, s));
+    record(ev.mid, s);
+    record(ev.end, s);
+    return rc;
+}
+
+int fusion_prune(int dtype, fusion_ragged in, const void *x, int32_t dim, const float *sizes,
+                 const float *scores, const float *rho, void *x_out, float *sizes_out,
+                 float *scores_out, int32_t *offsets_out, int32_t *keep_idx, void *workspace,
+                 size_t workspace_bytes, int32_t *dev_status, void *stream) {
+    FZ_TRY(check_dtype(dtype));
+    FZ_TRY(check_ragged(in));
+    FZ_TRY(check_dim(dim));
+    if (!x || !sizes || !scores || !rho || !x_out || !sizes_out || !offsets_out) return FUSION_ERR_INVALID_ARG;
+    if (!aligned16(x) || !aligned16(x_out)) return FUSION_ERR_INVALID_ARG;
+    FZ_TRY(check_workspace(workspace, workspace_bytes, in.max_batch, 1));
+    const ImageGeometry G = image_geometry(dtype, in.max_tokens, dim, 0);
+    if (!G.ok) return FUSION_ERR_SHAPE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const Ws w = carve(workspace, in.max_batch, 1);
+    PlanArgs pa{};
+    pa.in = dev(in);
+    pa.prune = 1;
+    pa.rho = rho;
+    pa.offsets_out = offsets_out;
+    pa.slot = w.slot;
+    pa.plan = w.plan;
+    pa.status = dev_status;
+    const ProfileEvents ev = take_profile();
+    record(ev.start, s);
+    FZ_TRY(cuda_rc(launch_plan(pa, s)));
+    record(ev.mid, s);
+    const ImageParams p = image_params(in, x, dim, nullptr, dim, sizes, scores, nullptr, rho, 0, 1, w,
+                                       offsets_out, x_out, sizes_out, scores_out, keep_idx, nullptr,
+                                       nullptr, dev_status, G);
+    const int rc = cuda_rc(launch_image(dtype, p, G.smem, s));
+    record(ev.end, s);
+    return rc;
+}
+
+int fusion_compact(int dtype, fusion_ragged in, const void *x, int32_t dim, const float *sizes,
+                   const float *scores, const uint8_t *exit_mask, void *x_out, float *sizes_out,
+                   float *scores_out, int32_t *offsets_out, int32_t *ids_out, int32_t *batch_out,
+                   int32_t *keep_idx, void *workspace, size_t workspace_bytes,
+                   int32_t *dev_status, void *stream) {
+    FZ_TRY(check_dtype(dtype));
+    FZ_TRY(check_ragged(in));
+    FZ_TRY(check_dim(dim));
+    if (!x || !sizes || !exit_mask || !x_out || !sizes_out || !offsets_out || !ids_out || !batch_out)
+        return FUSION_ERR_INVALID_ARG;
+    if ((scores == nullptr) != (scores_out == nullptr)) return FUSION_ERR_INVALID_ARG;
+    if (!aligned16(x) || !aligned16(x_out)) return FUSION_ERR_INVALID_ARG;
+    FZ_TRY(check_workspace(workspace, workspace_bytes, in.max_batch, 1));
+    const ImageGeometry G = image_geometry(dtype, in.max_tokens, dim, 0);
+    if (!G.ok) return FUSION_ERR_SHAPE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const Ws w = carve(workspace, in.max_batch, 1);
+    PlanArgs pa{};
+    pa.in = dev(in);
+    pa.exit_mask = exit_mask;
+    pa.offsets_out = offsets_out;
+    pa.ids_out = ids_out;
+    pa.batch_out = batch_out;
+    pa.slot = w.slot;
+    pa.plan = w.plan;
+    pa.status = dev_status;
+    const ProfileEvents ev = take_profile();
+    record(ev.start, s);
+    FZ_TRY(cuda_rc(launch_plan(pa, s)));
+    record(ev.mid, s);
+    const ImageParams p = image_params(in, x, dim, nullptr, dim, sizes, scores, nullptr, nullptr, 0, 0, w,
+                                       offsets_out, x_out, sizes_out, scores_out, keep_idx, nullptr,
+                                       nullptr, dev_status, G);
+    const int rc = cuda_rc(launch_image(dtype, p, G.smem, s));
+    record(ev.end, s);
+    return rc;
+}
+
+int fusion_stage(int dtype, int flags, fusion_ragged in, const void *x, int32_t dim,
+                 const void *keys, int32_t key_dim, const float *sizes, const float *scores,
+                 const int32_t *r, const float *rho, fusion_exit_head head, uint8_t *exit_mask,
+                 float *logits, float *max_prob, void *x_out, float *sizes_out, float *scores_out,
+                 int32_t *offsets_out, int32_t *ids_out, int32_t *batch_out, int32_t *keep_idx,
+                 int32_t *a_match, void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                 void *stream) {
+    FZ_TRY(check_dtype(dtype));
+    if (flags < 0 || flags > (FUSION_STAGE_MERGE | FUSION_STAGE_EXIT | FUSION_STAGE_PRUNE))
+        return FUSION_ERR_INVALID_ARG;
+    const int do_merge = (flags & FUSION_STAGE_MERGE) != 0;
+    const int do_exit = (flags & FUSION_STAGE_EXIT) != 0;
+    const int do_prune = (flags & FUSION_STAGE_PRUNE) != 0;
+    FZ_TRY(check_ragged(in));
+    FZ_TRY(check_dim(dim));
+    if (!x || !sizes || !x_out || !sizes_out || !offsets_out || !ids_out || !batch_out)
+        return FUSION_ERR_INVALID_ARG;
+    if ((scores == nullptr) != (scores_out == nullptr)) return FUSION_ERR_INVALID_ARG;
+    if (!aligned16(x) || !aligned16(x_out)) return FUSION_ERR_INVALID_ARG;
+    if (do_merge) {
+        if (!keys || !r || !aligned16(keys)) return FUSION_ERR_INVALID_ARG;
+        FZ_TRY(check_dim(key_dim));
+    }
+    if (do_prune && (!rho || !scores)) return FUSION_ERR_INVALID_ARG;
+    if (!do_merge && a_match) return FUSION_ERR_INVALID_ARG;
+    const int classes = do_exit ? head.classes : 1;
+    if (do_exit) {
+        FZ_TRY(check_head(head));
+        if (!exit_mask) return FUSION_ERR_INVALID_ARG;
+    }
+    FZ_TRY(check_workspace(workspace, workspace_bytes, in.max_batch, classes));
+    const ImageGeometry G = image_geometry(dtype, in.max_tokens, do_merge ? key_dim : dim, do_merge);
+    if (!G.ok) return FUSION_ERR_SHAPE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const Ws w = carve(workspace, in.max_batch, classes);
+
+    const ProfileEvents ev = take_profile();
+    record(ev.start, s);
+    PlanArgs pa{};
+    pa.in = dev(in);
+    pa.merge = do_merge;
+    pa.prune = do_prune;
+    pa.r = r;
+    pa.rho = rho;
+    pa.exit_mask = do_exit ? exit_mask : nullptr;
+    pa.offsets_out = offsets_out;
+    pa.ids_out = ids_out;
+    pa.batch_out = batch_out;
+    pa.slot = w.slot;
+    pa.plan = w.plan;
+    pa.status = dev_status;
+    if (do_exit) {
+        ExitParams e{};
+        e.in = dev(in);
+        e.x = x;
+        e.dim = dim;
+        e.head = dev(head);
+        e.exit_mask = exit_mask;
+        e.logits = logits;
+        e.max_prob = max_prob;
+        e.counters = w.counters;
+        e.partials = w.partials;
+        e.n_ctile = ceil_div(head.classes, kExitCT);
+        e.n_btile = ceil_div(in.max_batch > 0 ? in.max_batch : 1, kExitBT);
+        e.do_plan = 1;
+        e.plan = pa;
+        e.status = dev_status;
+        FZ_TRY(cuda_rc(launch_exit(dtype, e, s)));
+    } else {
+        FZ_TRY(cuda_rc(launch_plan(pa, s)));
+    }
+    record(ev.mid, s);
+    const ImageParams p = image_params(in, x, dim, do_merge ? keys : nullptr, key_dim, sizes, scores, r,
+                                       rho, do_merge, do_prune, w, offsets_out, x_out, sizes_out,
+                                       scores_out, keep_idx, nullptr, a_match, dev_status, G);
+    const int rc = cuda_rc(launch_image(dtype, p, G.smem, s));
+    record(ev.end, s);
+    return rc;
+}
+
+}  // extern "C"

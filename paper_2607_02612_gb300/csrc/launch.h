@@ -1,0 +1,75 @@
+// Host-side launchers of the Fusion kernels (one translation unit each).
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+#include "plan.cuh"
+
+namespace fz {
+
+// ---- exit check (+ optional plan for the fused stage) ----------------------
+struct ExitParams {
+    Ragged in;
+    const void *x;
+    int dim;
+    Head head;
+    uint8_t *exit_mask;
+    float *logits;
+    float *max_prob;
+    int *counters;   // workspace: [n_btile + 1], zero on entry, zero on exit
+    float2 *partials;
+    int n_ctile;
+    int n_btile;
+    int do_plan;     // run the compaction plan in the last CTA
+    PlanArgs plan;
+    int *status;
+};
+cudaError_t launch_exit(int dtype, const ExitParams &p, cudaStream_t s);
+size_t exit_smem_bytes(int dtype, int dim);
+
+// ---- stand-alone plan ----------------------------------------------------------
+cudaError_t launch_plan(const PlanArgs &a, cudaStream_t s);
+
+// ---- per-sample merge / prune / gather -----------------------------------------
+struct ImageParams {
+    Ragged in;
+    const void *x;
+    const void *keys;
+    int dim;
+    int kdim;
+    int keys_alias;
+    const float *sizes;
+    const float *scores;
+    const int *r;
+    const float *rho;
+    int do_merge;
+    int do_prune;
+    int need_match;      // compute matches even when no token merges (a_match requested)
+    const int *slot;     // workspace: output sample of every input sample (-1: gone)
+    const int *plan;     // workspace: plan[0] = batch valid
+    const int *offsets_out;
+    void *x_out;
+    float *sizes_out;
+    float *scores_out;
+    int *keep_idx;
+    int *dst_map;
+    int *a_match;
+    int *status;
+    // staging geometry, fixed by the host from max_tokens and the key width
+    int resident;        // every key dim staged at once
+    int kc;              // key dims staged per chunk (multiple of 16)
+    int ra, rb;          // rows per chunk column of the A and B staging regions
+};
+
+struct ImageGeometry {
+    int ok;              // fits in shared memory
+    int resident;
+    int kc;
+    int ra, rb;
+    size_t smem;         // dynamic shared memory bytes
+};
+ImageGeometry image_geometry(int dtype, int max_tokens, int kdim, int do_merge);
+cudaError_t launch_image(int dtype, const ImageParams &p, size_t smem, cudaStream_t s);
+
+}  // namespace fz

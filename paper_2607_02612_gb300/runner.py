@@ -1,0 +1,227 @@
+"""Python-side plumbing around the C ABI: device buffers, output allocation,
+stage chains and CUDA-graph capture.  torch provides memory and streams only;
+every step of the computation runs in libfusion.so.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+from typing import Dict, List, Optional
+
+import numpy as np
+import torch
+
+from . import _binding as fb
+
+DTYPE_CODE = {"f32": fb.FUSION_F32, "bf16": fb.FUSION_BF16}
+TORCH_DTYPE = {"f32": torch.float32, "bf16": torch.bfloat16}
+
+
+def tokens_to_torch(a: np.ndarray, dtype: str, device) -> torch.Tensor:
+    """float32 array or bf16 bit patterns (uint16) -> device tensor of the storage dtype."""
+    a = np.ascontiguousarray(a)
+    if dtype == "bf16":
+        return torch.from_numpy(a.view(np.int16)).to(device).view(torch.bfloat16)
+    return torch.from_numpy(a.astype(np.float32, copy=False)).to(device)
+
+
+def tokens_to_numpy(t: torch.Tensor, dtype: str) -> np.ndarray:
+    """Device tensor -> float32 array or bf16 bit patterns (uint16)."""
+    if dtype == "bf16":
+        return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+    return t.float().cpu().numpy()
+
+
+@dataclass
+class DeviceBatch:
+    """A ragged token batch on the device plus the host-side bounds the C ABI needs."""
+    dtype: str
+    dim: int
+    max_batch: int
+    max_tokens: int
+    max_rows: int
+    x: torch.Tensor
+    keys: torch.Tensor
+    sizes: torch.Tensor
+    scores: Optional[torch.Tensor]
+    offsets: torch.Tensor
+    batch: Optional[torch.Tensor] = None
+    ids: Optional[torch.Tensor] = None
+
+    @property
+    def key_dim(self) -> int:
+        return int(self.keys.shape[1])
+
+    def ragged(self) -> fb.fusion_ragged:
+        return fb.ragged(self.max_batch, self.max_tokens, self.max_rows, self.offsets, self.batch, self.ids)
+
+
+def device_batch(dtype: str, offsets, x, keys, sizes, scores, ids=None, max_tokens=None,
+                 device="cuda") -> DeviceBatch:
+    offsets = np.asarray(offsets, np.int32)
+    B = len(offsets) - 1
+    xt = tokens_to_torch(x, dtype, device)
+    kt = xt if keys is x else tokens_to_torch(keys, dtype, device)
+    if max_tokens is None:
+        max_tokens = int(np.max(np.diff(offsets))) if B > 0 else 1
+    return DeviceBatch(
+        dtype=dtype, dim=int(xt.shape[1]), max_batch=B, max_tokens=int(max_tokens), max_rows=int(xt.shape[0]),
+        x=xt, keys=kt, sizes=torch.from_numpy(np.asarray(sizes, np.float32)).to(device),
+        scores=None if scores is None else torch.from_numpy(np.asarray(scores, np.float32)).to(device),
+        offsets=torch.from_numpy(offsets).to(device),
+        ids=None if ids is None else torch.from_numpy(np.asarray(ids, np.int32)).to(device))
+
+
+@dataclass
+class HeadTensors:
+    gamma: torch.Tensor
+    beta: torch.Tensor
+    eps: float
+    weight: torch.Tensor
+    bias: torch.Tensor
+    tau: float
+
+    @property
+    def classes(self) -> int:
+        return int(self.weight.shape[0])
+
+    def c_struct(self) -> fb.fusion_exit_head:
+        return fb.exit_head(self.gamma, self.beta, self.eps, self.weight, self.bias, self.classes, self.tau)
+
+
+def head_tensors(head, dtype: str, device="cuda") -> HeadTensors:
+    return HeadTensors(tokens_to_torch(head.gamma, dtype, device), tokens_to_torch(head.beta, dtype, device),
+                       float(head.eps), tokens_to_torch(head.weight, dtype, device),
+                       torch.from_numpy(np.asarray(head.bias, np.float32)).to(device), float(head.tau))
+
+
+class Fusion:
+    """Owns a zero-initialised workspace and a device status word; each method
+    allocates its outputs and enqueues one C-ABI call on the current stream."""
+
+    def __init__(self, max_batch: int, classes: int = 1, device="cuda"):
+        self.device = torch.device(device)
+        self.ws_bytes = fb.fusion_workspace_size(max_batch, classes)
+        self.workspace = torch.zeros(self.ws_bytes, dtype=torch.uint8, device=self.device)
+        self.status = torch.zeros(1, dtype=torch.int32, device=self.device)
+        self.max_batch = max_batch
+        self.classes = classes
+
+    def _outputs(self, b: DeviceBatch, with_scores: bool) -> Dict[str, torch.Tensor]:
+        dev = self.device
+        return dict(
+            x=torch.empty((b.max_rows, b.dim), dtype=TORCH_DTYPE[b.dtype], device=dev),
+            sizes=torch.empty(b.max_rows, dtype=torch.float32, device=dev),
+            scores=torch.empty(b.max_rows, dtype=torch.float32, device=dev) if with_scores else None,
+            offsets=torch.zeros(b.max_batch + 1, dtype=torch.int32, device=dev),
+            keep_idx=torch.full((b.max_rows,), -1, dtype=torch.int32, device=dev))
+
+    def merge(self, b: DeviceBatch, r: torch.Tensor, *, dst_map=True, a_match=True) -> Dict[str, torch.Tensor]:
+        o = self._outputs(b, b.scores is not None)
+        o["dst_map"] = torch.full((b.max_rows,), -1, dtype=torch.int32, device=self.device) if dst_map else None
+        o["a_match"] = torch.full((b.max_rows,), -1, dtype=torch.int32, device=self.device) if a_match else None
+        fb.check(fb.fusion_merge(DTYPE_CODE[b.dtype], b.ragged(), b.x, b.dim, b.keys, b.key_dim, b.sizes,
+                                 b.scores, r, o["x"], o["sizes"], o["scores"], o["offsets"], o["keep_idx"],
+                                 o["dst_map"], o["a_match"], self.workspace, self.ws_bytes, self.status))
+        return o
+
+    def exit_check(self, b: DeviceBatch, head: HeadTensors) -> Dict[str, torch.Tensor]:
+        dev = self.device
+        o = dict(exit_mask=torch.zeros(b.max_batch, dtype=torch.uint8, device=dev),
+                 logits=torch.zeros((b.max_batch, head.classes), dtype=torch.float32, device=dev),
+                 max_prob=torch.zeros(b.max_batch, dtype=torch.float32, device=dev))
+        fb.check(fb.fusion_exit_check(DTYPE_CODE[b.dtype], b.ragged(), b.x, b.dim, head.c_struct(),
+                                      o["exit_mask"], o["logits"], o["max_prob"], self.workspace, self.ws_bytes,
+                                      self.status))
+        return o
+
+    def prune(self, b: DeviceBatch, rho: torch.Tensor) -> Dict[str, torch.Tensor]:
+        o = self._outputs(b, True)
+        fb.check(fb.fusion_prune(DTYPE_CODE[b.dtype], b.ragged(), b.x, b.dim, b.sizes, b.scores, rho, o["x"],
+                                 o["sizes"], o["scores"], o["offsets"], o["keep_idx"], self.workspace,
+                                 self.ws_bytes, self.status))
+        return o
+
+    def compact(self, b: DeviceBatch, exit_mask: torch.Tensor) -> Dict[str, torch.Tensor]:
+        o = self._outputs(b, b.scores is not None)
+        o["ids"] = torch.zeros(b.max_batch, dtype=torch.int32, device=self.device)
+        o["batch"] = torch.zeros(1, dtype=torch.int32, device=self.device)
+        fb.check(fb.fusion_compact(DTYPE_CODE[b.dtype], b.ragged(), b.x, b.dim, b.sizes, b.scores, exit_mask,
+                                   o["x"], o["sizes"], o["scores"], o["offsets"], o["ids"], o["batch"],
+                                   o["keep_idx"], self.workspace, self.ws_bytes, self.status))
+        return o
+
+    def stage(self, b: DeviceBatch, flags: int, r=None, rho=None, head: Optional[HeadTensors] = None,
+              a_match: bool = False, out: Optional[Dict[str, torch.Tensor]] = None) -> Dict[str, torch.Tensor]:
+        o = out if out is not None else self.stage_outputs(b, flags, head, a_match)
+        fb.check(fb.fusion_stage(
+            DTYPE_CODE[b.dtype], flags, b.ragged(), b.x, b.dim, b.keys, b.key_dim, b.sizes, b.scores, r, rho,
+            head.c_struct() if head is not None else None, o["exit_mask"], o["logits"], o["max_prob"], o["x"],
+            o["sizes"], o["scores"], o["offsets"], o["ids"], o["batch"], o["keep_idx"], o.get("a_match"),
+            self.workspace, self.ws_bytes, self.status))
+        return o
+
+    def stage_outputs(self, b: DeviceBatch, flags: int, head: Optional[HeadTensors], a_match: bool = False):
+        dev = self.device
+        o = self._outputs(b, b.scores is not None)
+        o["ids"] = torch.zeros(b.max_batch, dtype=torch.int32, device=dev)
+        o["batch"] = torch.zeros(1, dtype=torch.int32, device=dev)
+        has_exit = bool(flags & fb.FUSION_STAGE_EXIT)
+        o["exit_mask"] = torch.zeros(b.max_batch, dtype=torch.uint8, device=dev) if has_exit else None
+        o["logits"] = (torch.zeros((b.max_batch, head.classes), dtype=torch.float32, device=dev)
+                       if has_exit else None)
+        o["max_prob"] = torch.zeros(b.max_batch, dtype=torch.float32, device=dev) if has_exit else None
+        o["a_match"] = torch.full((b.max_rows,), -1, dtype=torch.int32, device=dev) if a_match else None
+        return o
+
+
+def output_batch(b: DeviceBatch, o: Dict[str, torch.Tensor]) -> DeviceBatch:
+    """The batch a stage hands to the next block (keys alias the new tokens)."""
+    return DeviceBatch(dtype=b.dtype, dim=b.dim, max_batch=b.max_batch, max_tokens=b.max_tokens,
+                       max_rows=b.max_rows, x=o["x"], keys=o["x"], sizes=o["sizes"], scores=o["scores"],
+                       offsets=o["offsets"], batch=o["batch"], ids=o["ids"])
+
+
+@dataclass
+class ChainStage:
+    flags: int
+    r: Optional[torch.Tensor] = None
+    rho: Optional[torch.Tensor] = None
+    head: Optional[HeadTensors] = None
+
+
+@dataclass
+class Chain:
+    """A schedule of stages over pre-allocated buffers; stage s+1 reads what stage s wrote.
+    run() enqueues every stage on the current stream with no host synchronisation."""
+    fusion: Fusion
+    inp: DeviceBatch
+    stages: List[ChainStage]
+    outs: List[Dict[str, torch.Tensor]] = field(default_factory=list)
+    batches: List[DeviceBatch] = field(default_factory=list)
+
+    def __post_init__(self):
+        b = self.inp
+        for st in self.stages:
+            o = self.fusion.stage_outputs(b, st.flags, st.head)
+            self.outs.append(o)
+            self.batches.append(b)
+            b = output_batch(b, o)
+
+    def run_stage(self, s: int, stream=None):
+        st, b, o = self.stages[s], self.batches[s], self.outs[s]
+        fb.check(fb.fusion_stage(
+            DTYPE_CODE[b.dtype], st.flags, b.ragged(), b.x, b.dim, b.keys, b.key_dim, b.sizes, b.scores, st.r,
+            st.rho, st.head.c_struct() if st.head is not None else None, o["exit_mask"], o["logits"],
+            o["max_prob"], o["x"], o["sizes"], o["scores"], o["offsets"], o["ids"], o["batch"], o["keep_idx"],
+            None, self.fusion.workspace, self.fusion.ws_bytes, self.fusion.status, stream))
+
+    def run(self, stream=None):
+        for s in range(len(self.stages)):
+            self.run_stage(s, stream)
+
+    def capture(self) -> torch.cuda.CUDAGraph:
+        """Capture the whole chain as one CUDA graph (run() once before, eagerly)."""
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.run()
+        return g

@@ -1,0 +1,146 @@
+"""The C-ABI library on the host: it loads, exports every function include/fusion.h
+declares, and rejects bad arguments before enqueueing anything.  No GPU needed:
+every call here fails a host-side check, so no CUDA call is made."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2607_02612_gb300 as fz
+from paper_2607_02612_gb300 import _binding as fb
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "fusion.h")
+
+FAKE = 0x100000   # never dereferenced: every call below fails a host check first
+
+
+@pytest.fixture(scope="module")
+def lib():
+    fz.build()
+    return fb.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(fusion_[a-z_]+)\s*\(", text)))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = declared_functions()
+    assert set(names) == set(fb.EXPORTED), names
+    raw = ctypes.CDLL(fb.LIB_PATH)
+    for n in names:
+        assert hasattr(raw, n), n
+
+
+def test_status_strings_and_version(lib):
+    assert fz.fusion_status_string(0) == "ok"
+    for code in (-1, -2, -3, -4, -5, 1, 2, 4, 8, 16):
+        assert fz.fusion_status_string(code) != "unknown status"
+    assert "sm_103a" in fz.fusion_version()
+
+
+def test_workspace_size_grows_with_batch_and_classes(lib):
+    a = fz.fusion_workspace_size(256, 1000)
+    assert a > 0 and a % 256 == 0
+    assert fz.fusion_workspace_size(8192, 1000) > a
+    assert fz.fusion_workspace_size(256, 4000) > a
+    assert fz.fusion_workspace_size(0, 1) > 0
+
+
+def _r(max_batch=4, max_tokens=197, max_rows=800, offsets=FAKE):
+    return fz.ragged(max_batch, max_tokens, max_rows, offsets)
+
+
+def _merge(**kw):
+    args = dict(dtype=fz.FUSION_BF16, in_=_r(), x=FAKE, dim=384, keys=FAKE, key_dim=384, sizes=FAKE,
+                scores=FAKE, r=FAKE, x_out=FAKE, sizes_out=FAKE, scores_out=FAKE, offsets_out=FAKE,
+                keep_idx=None, dst_map=None, a_match=None, workspace=FAKE,
+                workspace_bytes=fz.fusion_workspace_size(4, 1), dev_status=FAKE, stream=0)
+    args.update(kw)
+    return fz.fusion_merge(*args.values())
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(dtype=7), fz.FUSION_ERR_DTYPE),
+    (dict(dim=17), fz.FUSION_ERR_SHAPE),
+    (dict(dim=0), fz.FUSION_ERR_SHAPE),
+    (dict(dim=2048), fz.FUSION_ERR_SHAPE),
+    (dict(key_dim=8), fz.FUSION_ERR_SHAPE),
+    (dict(x=None), fz.FUSION_ERR_INVALID_ARG),
+    (dict(keys=None), fz.FUSION_ERR_INVALID_ARG),
+    (dict(r=None), fz.FUSION_ERR_INVALID_ARG),
+    (dict(x=FAKE + 8), fz.FUSION_ERR_INVALID_ARG),
+    (dict(x_out=FAKE + 4), fz.FUSION_ERR_INVALID_ARG),
+    (dict(scores_out=None), fz.FUSION_ERR_INVALID_ARG),
+    (dict(in_=_r(max_tokens=0)), fz.FUSION_ERR_SHAPE),
+    (dict(in_=_r(max_tokens=5000)), fz.FUSION_ERR_SHAPE),
+    (dict(in_=_r(max_batch=-1)), fz.FUSION_ERR_SHAPE),
+    (dict(in_=_r(offsets=None)), fz.FUSION_ERR_INVALID_ARG),
+    (dict(workspace=None), fz.FUSION_ERR_WORKSPACE),
+    (dict(workspace_bytes=16), fz.FUSION_ERR_WORKSPACE),
+])
+def test_merge_rejects_bad_arguments(lib, kw, code):
+    assert _merge(**kw) == code
+
+
+def _head(**kw):
+    h = dict(gamma=FAKE, beta=FAKE, eps=1e-6, weight=FAKE, bias=FAKE, classes=1000, tau=0.9)
+    h.update(kw)
+    return fz.exit_head(*h.values())
+
+
+def _stage(**kw):
+    args = dict(dtype=fz.FUSION_BF16, flags=7, in_=_r(), x=FAKE, dim=384, keys=FAKE, key_dim=384, sizes=FAKE,
+                scores=FAKE, r=FAKE, rho=FAKE, head=_head(), exit_mask=FAKE, logits=FAKE, max_prob=FAKE,
+                x_out=FAKE, sizes_out=FAKE, scores_out=FAKE, offsets_out=FAKE, ids_out=FAKE, batch_out=FAKE,
+                keep_idx=None, a_match=None, workspace=FAKE, workspace_bytes=fz.fusion_workspace_size(4, 1000),
+                dev_status=FAKE, stream=0)
+    args.update(kw)
+    return fz.fusion_stage(*args.values())
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(flags=8), fz.FUSION_ERR_INVALID_ARG),
+    (dict(flags=-1), fz.FUSION_ERR_INVALID_ARG),
+    (dict(head=_head(classes=0)), fz.FUSION_ERR_SHAPE),
+    (dict(head=_head(weight=None)), fz.FUSION_ERR_INVALID_ARG),
+    (dict(head=_head(gamma=FAKE + 2)), fz.FUSION_ERR_INVALID_ARG),
+    (dict(exit_mask=None), fz.FUSION_ERR_INVALID_ARG),
+    (dict(rho=None), fz.FUSION_ERR_INVALID_ARG),
+    (dict(ids_out=None), fz.FUSION_ERR_INVALID_ARG),
+    (dict(batch_out=None), fz.FUSION_ERR_INVALID_ARG),
+    (dict(flags=6, a_match=FAKE), fz.FUSION_ERR_INVALID_ARG),
+    (dict(workspace_bytes=fz.fusion_workspace_size(4, 1)), fz.FUSION_ERR_WORKSPACE),
+    (dict(scores=None, scores_out=None), fz.FUSION_ERR_INVALID_ARG),   # prune needs scores
+])
+def test_stage_rejects_bad_arguments(lib, kw, code):
+    assert _stage(**kw) == code
+
+
+def test_other_calls_reject_bad_arguments(lib):
+    ws = fz.fusion_workspace_size(4, 1000)
+    assert fz.fusion_exit_check(fz.FUSION_F32, _r(), FAKE, 384, _head(classes=0), FAKE, None, None, FAKE, ws,
+                                FAKE, 0) == fz.FUSION_ERR_SHAPE
+    assert fz.fusion_exit_check(fz.FUSION_F32, _r(), FAKE, 384, _head(), None, None, None, FAKE, ws,
+                                FAKE, 0) == fz.FUSION_ERR_INVALID_ARG
+    assert fz.fusion_prune(fz.FUSION_F32, _r(), FAKE, 384, FAKE, None, FAKE, FAKE, FAKE, FAKE, FAKE, None,
+                           FAKE, ws, FAKE, 0) == fz.FUSION_ERR_INVALID_ARG
+    assert fz.fusion_compact(fz.FUSION_F32, _r(), FAKE, 384, FAKE, None, None, FAKE, FAKE, None, FAKE, FAKE,
+                             FAKE, None, FAKE, ws, FAKE, 0) == fz.FUSION_ERR_INVALID_ARG
+    assert fz.fusion_compact(2, _r(), FAKE, 384, FAKE, None, FAKE, FAKE, FAKE, None, FAKE, FAKE,
+                             FAKE, None, FAKE, ws, FAKE, 0) == fz.FUSION_ERR_DTYPE
+
+
+def test_binding_refuses_host_tensors(lib):
+    import torch
+    with pytest.raises(fz.FusionError):
+        fb._ptr(torch.zeros(4))
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    with pytest.raises(fz.FusionError):
+        fb.load(str(tmp_path / "libfusion.so"))

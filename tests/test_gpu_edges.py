@@ -1,0 +1,204 @@
+"""Edge cases and device-side error reporting of the CUDA path (GPU only).
+
+Degenerate samples (P = 0, 1, 2), clamped merge counts, keep ratios 0 and 1, all or
+no samples exiting, exact ties (identical keys), zero-norm keys, signed-zero
+scores, keys separate from or aliased to the tokens, an empty batch, a device batch
+count below the host bound, the largest supported sample, and malformed inputs
+that must raise status bits without touching memory out of bounds.
+"""
+import os
+import sys
+
+import numpy as np
+import pytest
+import torch
+
+sys.path.insert(0, os.path.dirname(os.path.abspath(__file__)))
+
+import oracle  # noqa: E402
+import parity as P  # noqa: E402
+import paper_2607_02612_gb300 as fz  # noqa: E402
+from paper_2607_02612_gb300 import runner  # noqa: E402
+from workloads import Batch, Head, StageSpec, f32_to_bf16_bits  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+
+def make_batch(counts, dim, dtype, seed=0, keys="alias", kdim=None, same_keys=False, zero_key=False,
+               signed_zero_scores=False, sizes="ones"):
+    rng = np.random.default_rng(seed)
+    counts = np.asarray(counts)
+    offs = np.concatenate([[0], np.cumsum(counts)]).astype(np.int32)
+    T = int(offs[-1])
+    x32 = rng.standard_normal((T, dim)).astype(np.float32)
+    if same_keys:
+        x32[:] = rng.standard_normal(dim).astype(np.float32)
+    if zero_key and T > 3:
+        x32[3] = 0.0
+    sz = np.ones(T, np.float32) if sizes == "ones" else rng.integers(1, 5, T).astype(np.float32)
+    sc = rng.random(T).astype(np.float32)
+    if signed_zero_scores:
+        sc[::2] = -0.0
+        sc[1::2] = 0.0
+    x = f32_to_bf16_bits(x32) if dtype == "bf16" else x32
+    if keys == "alias":
+        k = x
+    else:
+        k32 = rng.standard_normal((T, kdim or dim)).astype(np.float32)
+        k = f32_to_bf16_bits(k32) if dtype == "bf16" else k32
+    return Batch(dtype, offs, x, k, sz, sc)
+
+
+def make_head(dim, C, dtype, tau, seed=1, scale=1.0):
+    rng = np.random.default_rng(seed)
+    W = (rng.standard_normal((C, dim)) * scale).astype(np.float32)
+    rd = (lambda a: f32_to_bf16_bits(a)) if dtype == "bf16" else (lambda a: a)
+    return Head(rd(np.ones(dim, np.float32)), rd(np.zeros(dim, np.float32)), 1e-6, rd(W),
+                np.zeros(C, np.float32), tau)
+
+
+def run_stage_and_compare(b, spec, label):
+    classes = spec.head.classes if spec.head is not None else 1
+    f = runner.Fusion(b.batch, classes)
+    r, rho, head = P.stage_tensors(spec, b.dtype)
+    g = P.to_host(f.stage(P.device_batch(b), P.flags_of(spec), r, rho, head, a_match=spec.merge), b.dtype)
+    assert int(f.status.item()) == 0, label
+    o = oracle.stage(b, spec)
+    rep = P.Report()
+    ids = np.arange(b.batch)
+    if spec.exit:
+        P.compare_exit(rep, b.dtype, ids, g["exit_mask"], g["logits"], g["max_prob"], o)
+    nb = int(g["batch"][0])
+    assert nb == o["n_out"], label
+    P.compare_tokens(rep, b.dtype, b.offsets, ids, b.offsets, ids, g, o, g["ids"][:nb], o["ids"],
+                     a_match_gpu=g.get("a_match"))
+    print(f"[{label}] {rep.summary()}")
+    rep.check()
+    return g, o
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("keys", ["alias", "separate"])
+def test_degenerate_and_ragged_samples(dtype, keys):
+    counts = [1, 2, 3, 4, 5, 6, 17, 64, 65, 1, 33, 2]
+    b = make_batch(counts, 48, dtype, keys=keys, kdim=32, sizes="u1to4")
+    B = len(counts)
+    r = np.array([0, 3, 1, 1, 2, 99, 8, -4, 40, 5, 16, 0], np.int32)
+    rho = np.array([0.0, 1.0, 0.5, 0.3, 1.0, 0.0, 0.61, 0.9, 0.25, 1.0, 0.99, 0.5], np.float32)
+    for flags in [(True, False, False), (False, False, True), (True, False, True), (True, True, True)]:
+        m, e, p = flags
+        head = make_head(48, 10, dtype, 0.45, scale=0.15) if e else None
+        spec = StageSpec(m, e, p, r=r, rho=rho, head=head)
+        run_stage_and_compare(b, spec, f"{dtype}/{keys}/{flags}")
+    assert B == len(r)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_identical_keys_zero_norm_and_signed_zero(dtype):
+    b = make_batch([33, 20, 9], 32, dtype, same_keys=True, signed_zero_scores=True)
+    spec = StageSpec(True, False, True, r=np.array([5, 9, 4], np.int32), rho=np.array([0.5, 0.7, 0.34], np.float32))
+    g, o = run_stage_and_compare(b, spec, f"ties {dtype}")
+    b2 = make_batch([17, 17], 32, dtype, zero_key=True, seed=4)
+    spec2 = StageSpec(True, False, False, r=np.array([8, 8], np.int32))
+    run_stage_and_compare(b2, spec2, f"zero-key {dtype}")
+
+
+@pytest.mark.parametrize("tau", [0.0, 2.0])
+def test_all_or_no_samples_exit(tau):
+    b = make_batch([10] * 37, 64, "bf16", seed=3)
+    spec = StageSpec(True, True, True, r=np.full(37, 3, np.int32), rho=np.full(37, 0.5, np.float32),
+                     head=make_head(64, 130, "bf16", tau))
+    g, o = run_stage_and_compare(b, spec, f"tau={tau}")
+    assert int(g["batch"][0]) == (0 if tau == 0.0 else 37)
+    assert g["offsets"][0] == 0
+
+
+def test_empty_batch_and_device_count():
+    b = make_batch([5, 7, 9, 11], 32, "f32", seed=8)
+    db = P.device_batch(b)
+    f = runner.Fusion(4, 3)
+    spec = StageSpec(True, True, True, r=np.full(4, 2, np.int32), rho=np.full(4, 0.5, np.float32),
+                     head=make_head(32, 3, "f32", 2.0))
+    r, rho, head = P.stage_tensors(spec, "f32")
+    # device count 0: nothing survives, nothing is written
+    db.batch = torch.zeros(1, dtype=torch.int32, device="cuda")
+    g = P.to_host(f.stage(db, 7, r, rho, head), "f32")
+    assert int(f.status.item()) == 0
+    assert int(g["batch"][0]) == 0 and g["offsets"][0] == 0
+    assert np.all(g["keep_idx"] == -1)
+    # device count 2 of a bound of 4: only the first two samples are processed
+    db.batch = torch.full((1,), 2, dtype=torch.int32, device="cuda")
+    g = P.to_host(f.stage(db, 7, r, rho, head), "f32")
+    sub = Batch("f32", b.offsets[:3], b.x, b.keys, b.sizes, b.scores)
+    o = oracle.stage(sub, StageSpec(True, True, True, r=spec.r, rho=spec.rho, head=spec.head))
+    assert int(g["batch"][0]) == o["n_out"] == 2
+    np.testing.assert_array_equal(g["offsets"][:3], o["offsets"])
+    np.testing.assert_array_equal(g["keep_idx"][:o["offsets"][-1]], o["keep_idx"])
+
+
+def test_ids_index_router_outputs():
+    """With ids, r and rho are read at the original image number."""
+    b = make_batch([9, 11, 13], 32, "f32", seed=5)
+    b.ids = np.array([2, 0, 1], np.int32)
+    spec = StageSpec(True, False, True, r=np.array([3, 1, 2], np.int32), rho=np.array([0.2, 0.6, 0.9], np.float32))
+    g, o = run_stage_and_compare(b, spec, "ids")
+    np.testing.assert_array_equal(g["ids"][:3], b.ids)
+
+
+def test_largest_sample():
+    b = make_batch([fz.FUSION_MAX_TOKENS, 3], 16, "bf16", seed=6)
+    spec = StageSpec(True, False, True, r=np.array([300, 1], np.int32), rho=np.array([0.37, 1.0], np.float32))
+    run_stage_and_compare(b, spec, "max tokens")
+
+
+# ---------------------------------------------------------------------------
+# malformed inputs: status bits, no out-of-bounds access, no token writes
+# ---------------------------------------------------------------------------
+def _stage_raw(b, db, offsets=None, batch=None, ids=None, keys=None):
+    f = runner.Fusion(db.max_batch, 1)
+    o = f.stage_outputs(db, 5, None)
+    o["x"].fill_(7)
+    o["keep_idx"].fill_(-5)
+    rr = torch.full((db.max_batch,), 2, dtype=torch.int32, device="cuda")
+    rho = torch.full((db.max_batch,), 0.5, dtype=torch.float32, device="cuda")
+    rg = fz.ragged(db.max_batch, db.max_tokens, db.max_rows, offsets if offsets is not None else db.offsets,
+                   batch, ids)
+    fz.check(fz.fusion_stage(fz.FUSION_F32, 5, rg, db.x, db.dim, keys if keys is not None else db.keys,
+                             db.key_dim, db.sizes, db.scores, rr, rho, None, None, None, None, o["x"],
+                             o["sizes"], o["scores"], o["offsets"], o["ids"], o["batch"], o["keep_idx"], None,
+                             f.workspace, f.ws_bytes, f.status))
+    torch.cuda.synchronize()
+    return int(f.status.item()), o
+
+
+def test_bad_offsets_raise_status_and_write_nothing():
+    b = make_batch([8, 8, 8], 16, "f32", seed=7)
+    db = P.device_batch(b)
+    for bad in ([0, 8, 4, 24], [0, 8, 16, 99], [-3, 8, 16, 24], [0, 0, 16, 24], [0, 8, 16, 24 + 0]):
+        offs = torch.tensor(bad, dtype=torch.int32, device="cuda")
+        st, o = _stage_raw(b, db, offsets=offs)
+        if bad == [0, 8, 16, 24]:
+            assert st == 0
+            continue
+        assert st & fz.FUSION_DEV_BAD_OFFSETS, bad
+        assert torch.all(o["keep_idx"] == -5) and torch.all(o["x"] == 7), bad
+
+
+def test_bad_batch_and_ids_raise_status():
+    b = make_batch([8, 8], 16, "f32", seed=9)
+    db = P.device_batch(b)
+    st, o = _stage_raw(b, db, batch=torch.full((1,), 3, dtype=torch.int32, device="cuda"))
+    assert st & fz.FUSION_DEV_BAD_BATCH
+    assert torch.all(o["keep_idx"] == -5)
+    st, o = _stage_raw(b, db, ids=torch.tensor([0, 7], dtype=torch.int32, device="cuda"))
+    assert st & fz.FUSION_DEV_BAD_IDS
+    assert torch.all(o["keep_idx"] == -5)
+
+
+def test_nonfinite_keys_raise_status():
+    b = make_batch([9, 9], 16, "f32", seed=10, keys="separate")
+    db = P.device_batch(b)
+    k = db.keys.clone()
+    k[2, 3] = float("nan")
+    st, _ = _stage_raw(b, db, keys=k)
+    assert st & fz.FUSION_DEV_NONFINITE

@@ -1,0 +1,211 @@
+"""CUDA path vs the CPU oracle on the seeded workloads (GPU only).
+
+Reduced batches span many CTAs and ragged tails and finish in seconds on the
+oracle; the full-size checks run the GPU at the benchmark's sizes and compare a
+seeded sample of images against the oracle run on those images alone (images
+are independent apart from compaction order, which is compared through ids).
+"""
+import os
+import sys
+
+import numpy as np
+import pytest
+import torch
+
+sys.path.insert(0, os.path.dirname(os.path.abspath(__file__)))
+
+import oracle  # noqa: E402
+import parity as P  # noqa: E402
+from paper_2607_02612_gb300 import runner  # noqa: E402
+from workloads import Batch, make_workload  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+CASES = [
+    ("deit_s_stage_f32_b8", None),
+    ("deit_s_chain12_bf16_b256", None),
+    ("deit_b_stage_bf16_b512", 96),
+    ("vit_l16_384_stage_bf16_b128", 12),
+    ("ragged_b8192_n65_chain4_f32", 512),
+    ("ragged_b8192_n65_chain4_bf16", 512),
+]
+IDS = [c[0] for c in CASES]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2607_02612_gb300 import build
+    build()
+    assert torch.cuda.is_available()
+
+
+def _first(w, attr):
+    for s in w.stages:
+        if getattr(s, attr):
+            return s
+    raise AssertionError(attr)
+
+
+def _report(rep, label):
+    print(f"[{label}] {rep.summary()}")
+    rep.check()
+
+
+@pytest.mark.parametrize("name,B", CASES, ids=IDS)
+def test_merge_parity(name, B):
+    w = make_workload(name, batch=B)
+    b, spec = w.batch, w.stages[0]
+    fz = runner.Fusion(b.batch)
+    db = P.device_batch(b)
+    g = P.to_host(fz.merge(db, torch.from_numpy(spec.r).cuda()), b.dtype)
+    assert int(fz.status.item()) == 0
+    o = oracle.merge(b.dtype, b.offsets, b.x, b.keys, b.sizes, b.scores, spec.r)
+    np.testing.assert_array_equal(g["offsets"], o["offsets"])
+    rep = P.Report()
+    P.count_decision_near_ties(rep, o)
+    ids = np.arange(b.batch)
+    P.compare_tokens(rep, b.dtype, b.offsets, ids, b.offsets, ids, g, o, ids, ids, a_match_gpu=g["a_match"])
+    for i in range(b.batch):
+        if i in rep.excluded:
+            continue
+        a0, a1 = b.offsets[i], b.offsets[i + 1]
+        assert np.array_equal(g["dst_map"][a0:a1], o["dst_map"][a0:a1]), f"dst_map of sample {i}"
+    _report(rep, f"merge {name}")
+
+
+@pytest.mark.parametrize("name,B", CASES, ids=IDS)
+def test_exit_parity(name, B):
+    w = make_workload(name, batch=B)
+    b, spec = w.batch, _first(w, "exit")
+    fz = runner.Fusion(b.batch, spec.head.classes)
+    g = P.to_host(fz.exit_check(P.device_batch(b), runner.head_tensors(spec.head, b.dtype)), b.dtype)
+    assert int(fz.status.item()) == 0
+    o = oracle.exit_check(b.dtype, b.offsets, b.x, spec.head)
+    rep = P.Report()
+    P.compare_exit(rep, b.dtype, np.arange(b.batch), g["exit_mask"], g["logits"], g["max_prob"], o)
+    _report(rep, f"exit {name}")
+
+
+@pytest.mark.parametrize("name,B", CASES, ids=IDS)
+def test_prune_parity(name, B):
+    w = make_workload(name, batch=B)
+    b, spec = w.batch, _first(w, "prune")
+    fz = runner.Fusion(b.batch)
+    g = P.to_host(fz.prune(P.device_batch(b), torch.from_numpy(spec.rho).cuda()), b.dtype)
+    assert int(fz.status.item()) == 0
+    o = oracle.prune(b.dtype, b.offsets, b.x, b.sizes, b.scores, spec.rho)
+    np.testing.assert_array_equal(g["offsets"], o["offsets"])
+    t = int(o["offsets"][-1])
+    np.testing.assert_array_equal(g["keep_idx"][:t], o["keep_idx"])
+    np.testing.assert_array_equal(g["x"][:t], o["x"])
+    np.testing.assert_array_equal(g["sizes"][:t], o["sizes"])
+    np.testing.assert_array_equal(g["scores"][:t], o["scores"])
+
+
+@pytest.mark.parametrize("name,B", CASES[:2] + CASES[4:], ids=IDS[:2] + IDS[4:])
+def test_compact_parity(name, B):
+    w = make_workload(name, batch=B)
+    b = w.batch
+    mask = (np.random.default_rng(17).random(b.batch) < 0.45).astype(np.uint8)
+    fz = runner.Fusion(b.batch)
+    g = P.to_host(fz.compact(P.device_batch(b), torch.from_numpy(mask).cuda()), b.dtype)
+    assert int(fz.status.item()) == 0
+    o = oracle.compact(b.dtype, b.offsets, b.x, b.sizes, b.scores, mask)
+    nb = int(g["batch"][0])
+    assert nb == o["n_out"]
+    np.testing.assert_array_equal(g["offsets"][:nb + 1], o["offsets"])
+    np.testing.assert_array_equal(g["ids"][:nb], o["ids"])
+    t = int(o["offsets"][-1])
+    np.testing.assert_array_equal(g["keep_idx"][:t], o["keep_idx"])
+    np.testing.assert_array_equal(g["x"][:t], o["x"])
+
+
+@pytest.mark.parametrize("name,B", CASES, ids=IDS)
+def test_fused_stage_parity(name, B):
+    """merge -> exit -> prune -> compact in one call equals the oracle's composition."""
+    w = make_workload(name, batch=B)
+    b, spec = w.batch, _first(w, "exit")
+    fz = runner.Fusion(b.batch, spec.head.classes)
+    r, rho, head = P.stage_tensors(spec, b.dtype)
+    g = P.to_host(fz.stage(P.device_batch(b), P.flags_of(spec), r, rho, head, a_match=True), b.dtype)
+    assert int(fz.status.item()) == 0
+    o = oracle.stage(b, spec)
+    rep = P.Report()
+    P.count_decision_near_ties(rep, o)
+    ids = np.arange(b.batch)
+    P.compare_exit(rep, b.dtype, ids, g["exit_mask"], g["logits"], g["max_prob"], o)
+    nb = int(g["batch"][0])
+    P.compare_tokens(rep, b.dtype, b.offsets, ids, b.offsets, ids, g, o, g["ids"][:nb], o["ids"],
+                     a_match_gpu=g["a_match"])
+    _report(rep, f"stage {name}")
+
+
+@pytest.mark.parametrize("name,B,graph", [
+    ("deit_s_chain12_bf16_b256", None, True),
+    ("ragged_b8192_n65_chain4_bf16", 1024, False),
+    ("ragged_b8192_n65_chain4_f32", 1024, True),
+])
+def test_chain_parity(name, B, graph):
+    """Every stage of a chained schedule (compaction between blocks, no host sync)."""
+    w = make_workload(name, batch=B)
+    g_outs, status = P.chain_on_gpu(w, graph=graph)
+    assert status == 0
+    o_outs = oracle.chain(w)
+    rep = P.Report()
+    P.compare_chain(rep, w, g_outs, o_outs)
+    assert rep.compared_samples > 0
+    _report(rep, f"chain {name}")
+
+
+def _subset(batch: Batch, idx: np.ndarray) -> Batch:
+    """The images idx of a batch, repacked (ids keep the original image numbers)."""
+    counts = np.diff(batch.offsets)[idx]
+    offs = np.concatenate([[0], np.cumsum(counts)]).astype(np.int32)
+    rows = np.concatenate([np.arange(batch.offsets[i], batch.offsets[i + 1]) for i in idx])
+    x = batch.x[rows]
+    keys = x if batch.keys_alias else batch.keys[rows]
+    return Batch(batch.dtype, offs, x, keys, batch.sizes[rows], batch.scores[rows], ids=idx.astype(np.int32))
+
+
+@pytest.mark.parametrize("name", ["deit_b_stage_bf16_b512", "vit_l16_384_stage_bf16_b128",
+                                  "ragged_b8192_n65_chain4_bf16", "ragged_b8192_n65_chain4_f32",
+                                  "deit_s_chain12_bf16_b256"])
+def test_full_size_sampled(name):
+    """Full batch on the GPU in the benchmark's configuration (CUDA graph); the oracle
+    recomputes a seeded sample of images one by one and every stage of theirs must match."""
+    w = make_workload(name)
+    g_outs, status = P.chain_on_gpu(w, graph=True)
+    assert status == 0
+    n = 48 if w.batch.batch > 48 else w.batch.batch
+    idx = np.sort(np.random.default_rng(99).choice(w.batch.batch, n, replace=False))
+    w_sub = type(w)(w.spec, _subset(w.batch, idx), w.stages)
+    o_outs = oracle.chain(w_sub)
+    rep = P.Report()
+    # per stage, compare the sampled ids only
+    o_ids_in = idx.astype(np.int32)
+    o_off_in = w_sub.batch.offsets
+    g_ids_in = np.arange(w.batch.batch, dtype=np.int32)
+    g_off_in = w.batch.offsets
+    for s, (g, o) in enumerate(zip(g_outs, o_outs)):
+        spec = w.stages[s]
+        P.count_decision_near_ties(rep, o)
+        g_nb = int(g["batch"][0])
+        if spec.exit:
+            gpos = {int(t): i for i, t in enumerate(g_ids_in)}
+            for i, t in enumerate(o_ids_in):
+                t = int(t)
+                if t in rep.excluded:
+                    continue
+                ig = gpos[t]
+                if g["exit_mask"][ig] != o["exit_mask"][i]:
+                    if o["exit_gap"][i] < P.NEAR_TIE:
+                        rep.near_tie_mismatch["exit"] += 1
+                        rep.excluded.add(t)
+                    else:
+                        rep.fail(f"stage {s}: exit differs for image {t}")
+        P.compare_tokens(rep, w.batch.dtype, o_off_in, o_ids_in, g_off_in, g_ids_in, g, o, g["ids"][:g_nb],
+                         o["ids"])
+        o_ids_in, o_off_in = o["ids"], o["offsets"]
+        g_ids_in, g_off_in = g["ids"][:g_nb], g["offsets"][:g_nb + 1]
+    assert rep.compared_samples > 0
+    _report(rep, f"full {name}")

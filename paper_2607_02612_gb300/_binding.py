@@ -145,6 +145,8 @@ def _event(e) -> Optional[int]:
     if e is None:
         return None
     if isinstance(e, torch.cuda.Event):
+        if not e.cuda_event:   # torch creates the CUDA event lazily, at its first record()
+            e.record()
         return e.cuda_event
     return int(e)
 

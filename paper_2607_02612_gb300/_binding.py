@@ -65,6 +65,10 @@ def load(path: Optional[str] = None):
     if _lib is not None and path is None:
         return _lib
     p = path or LIB_PATH
+    if path is None:
+        from .build import build as _build, _stale
+        if _stale():
+            _build()   # sources changed since the last build: rebuild (needs nvcc)
     if not os.path.exists(p):
         raise FusionError(f"{p} is missing: build the CUDA library first "
                           "(python -m paper_2607_02612_gb300.build)")

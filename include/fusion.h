@@ -181,6 +181,28 @@ int fusion_exit_check(int dtype, fusion_ragged in, const void *x, int32_t dim,
                       void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream);
 
 /*
+ * fusion_exit_check_noalloc: fusion_exit_check for callers that cannot allocate
+ * device memory.  The paper has no counterpart; this is a deployment aid.
+ *
+ * Some callers have no way to call cudaMalloc (a plugin host that passes only
+ * input and output buffers, a C program without a device allocator, a loop where
+ * an allocation would stall).  This call takes the same inputs and outputs as
+ * fusion_exit_check but no workspace: its scratch lives in a 1 MiB device array
+ * inside the library, present on every GPU that loads the library until the
+ * process exits.  A batch bound and class count whose scratch exceeds 1 MiB (see
+ * fusion_workspace_size) is rejected with FUSION_ERR_WORKSPACE before anything is
+ * enqueued.  The first call on a device looks up the array's device address, so
+ * make that first call before any stream capture.  Calls allocate nothing
+ * (no cudaMalloc / cudaFree); each one clears the counters it needs with an
+ * asynchronous memset on `stream`.  All calls on a device share the one array:
+ * calls that may run concurrently on the GPU (unordered streams) race and must
+ * not be issued.
+ */
+int fusion_exit_check_noalloc(int dtype, fusion_ragged in, const void *x, int32_t dim,
+                              fusion_exit_head head, uint8_t *exit_mask, float *logits,
+                              float *max_prob, int32_t *dev_status, void *stream);
+
+/*
  * fusion_prune: keep CLS and the k_i = ceil(rho * P_i) patch tokens with the
  * largest scores (Sec. III-E, Eq. 8, with the keep count taken per sample), in
  * ascending position.  rho is read as its exact float32 value; k is clamped to

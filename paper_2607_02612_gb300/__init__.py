@@ -30,6 +30,7 @@ from ._binding import (  # noqa: F401
     exit_head,
     fusion_compact,
     fusion_exit_check,
+    fusion_exit_check_noalloc,
     fusion_merge,
     fusion_profile_next,
     fusion_prune,

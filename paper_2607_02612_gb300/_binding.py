@@ -37,7 +37,8 @@ FUSION_MAX_TOKENS = 1024
 FUSION_MAX_DIM = 1024
 
 EXPORTED = ("fusion_status_string", "fusion_version", "fusion_profile_next", "fusion_workspace_size",
-            "fusion_merge", "fusion_exit_check", "fusion_prune", "fusion_compact", "fusion_stage")
+            "fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune", "fusion_compact",
+            "fusion_stage")
 
 
 class FusionError(RuntimeError):
@@ -86,11 +87,13 @@ def load(path: Optional[str] = None):
     lib.fusion_workspace_size.restype = SZ
     lib.fusion_merge.argtypes = [ctypes.c_int, R, V, I32, V, I32, V, V, V, V, V, V, V, V, V, V, V, SZ, V, V]
     lib.fusion_exit_check.argtypes = [ctypes.c_int, R, V, I32, H, V, V, V, V, SZ, V, V]
+    lib.fusion_exit_check_noalloc.argtypes = [ctypes.c_int, R, V, I32, H, V, V, V, V, V]
     lib.fusion_prune.argtypes = [ctypes.c_int, R, V, I32, V, V, V, V, V, V, V, V, V, SZ, V, V]
     lib.fusion_compact.argtypes = [ctypes.c_int, R, V, I32, V, V, V, V, V, V, V, V, V, V, V, SZ, V, V]
     lib.fusion_stage.argtypes = [ctypes.c_int, ctypes.c_int, R, V, I32, V, I32, V, V, V, V, H, V, V, V,
                                  V, V, V, V, V, V, V, V, V, SZ, V, V]
-    for name in ("fusion_merge", "fusion_exit_check", "fusion_prune", "fusion_compact", "fusion_stage"):
+    for name in ("fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune",
+                 "fusion_compact", "fusion_stage"):
         getattr(lib, name).restype = ctypes.c_int
     del I64, F
     if path is None:
@@ -178,6 +181,13 @@ def fusion_exit_check(dtype, in_, x, dim, head, exit_mask, logits, max_prob, wor
     return load().fusion_exit_check(int(dtype), in_, _ptr(x), int(dim), head, _ptr(exit_mask), _ptr(logits),
                                     _ptr(max_prob), _ptr(workspace), int(workspace_bytes), _ptr(dev_status),
                                     _stream(stream))
+
+
+def fusion_exit_check_noalloc(dtype, in_, x, dim, head, exit_mask, logits, max_prob, dev_status,
+                              stream=None) -> int:
+    """fusion_exit_check with the library's built-in scratch (for callers that cannot allocate)."""
+    return load().fusion_exit_check_noalloc(int(dtype), in_, _ptr(x), int(dim), head, _ptr(exit_mask),
+                                            _ptr(logits), _ptr(max_prob), _ptr(dev_status), _stream(stream))
 
 
 def fusion_prune(dtype, in_, x, dim, sizes, scores, rho, x_out, sizes_out, scores_out, offsets_out,

@@ -1,0 +1,68 @@
+"""fusion_exit_check_noalloc against fusion_exit_check (GPU only).
+
+The no-allocation variant serves callers that cannot call cudaMalloc (plugin hosts
+that pass only inputs and outputs, programs without a device allocator).  It must
+give the same exit decisions, logits and max-probabilities as the workspace-based
+call, on two calls in a row (the built-in scratch keeps the previous call's
+contents, so the second call checks that the per-call reset works), and it must
+refuse a batch whose scratch would not fit.  This file is collected last.
+"""
+import ctypes
+import os
+import sys
+
+import numpy as np
+import pytest
+import torch
+
+sys.path.insert(0, os.path.dirname(os.path.abspath(__file__)))
+
+import parity as P  # noqa: E402
+import paper_2607_02612_gb300 as fz  # noqa: E402
+from paper_2607_02612_gb300 import _binding as fb  # noqa: E402
+from paper_2607_02612_gb300 import runner  # noqa: E402
+from workloads import make_workload  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("name,B", [("deit_s_chain12_bf16_b256", None), ("ragged_b8192_n65_chain4_f32", 2048)])
+def test_noalloc_matches_workspace_call_twice(name, B):
+    fz.build()
+    lib = fb.load()
+    w = make_workload(name, batch=B)
+    b = w.batch
+    spec = next(s for s in w.stages if s.exit)
+    db = P.device_batch(b)
+    head = runner.head_tensors(spec.head, b.dtype)
+    dt = runner.DTYPE_CODE[b.dtype]
+    f = runner.Fusion(b.batch, head.classes)
+    ref = f.exit_check(db, head)
+    torch.cuda.synchronize()
+    assert int(f.status.item()) == 0
+    for call in range(2):
+        mask = torch.full((b.batch,), 7, dtype=torch.uint8, device="cuda")
+        logits = torch.full((b.batch, head.classes), float("nan"), dtype=torch.float32, device="cuda")
+        maxp = torch.full((b.batch,), -1.0, dtype=torch.float32, device="cuda")
+        status = torch.zeros(1, dtype=torch.int32, device="cuda")
+        rc = lib.fusion_exit_check_noalloc(dt, db.ragged(), db.x.data_ptr(), db.dim, head.c_struct(),
+                                           mask.data_ptr(), logits.data_ptr(), maxp.data_ptr(),
+                                           status.data_ptr(), torch.cuda.current_stream().cuda_stream)
+        assert rc == fz.FUSION_OK, fz.fusion_status_string(rc)
+        torch.cuda.synchronize()
+        assert int(status.item()) == 0
+        assert torch.equal(mask, ref["exit_mask"]), f"call {call}: exit masks differ"
+        tol = P.TOL[b.dtype]
+        e = P.rel_err_rows(logits.cpu().numpy(), ref["logits"].cpu().numpy())
+        assert e.max() <= tol, f"call {call}: logits off by {e.max()}"
+        ep = np.abs(maxp.cpu().numpy() - ref["max_prob"].cpu().numpy()) / ref["max_prob"].cpu().numpy()
+        assert ep.max() <= tol, f"call {call}: max_prob off by {ep.max()}"
+
+
+def test_noalloc_rejects_batches_beyond_its_scratch():
+    lib = fb.load()
+    big = fz.ragged(1 << 20, 197, 1 << 28, 0x100000)
+    head = fz.exit_head(0x100000, 0x100000, 1e-6, 0x100000, 0x100000, 1000, 0.9)
+    rc = lib.fusion_exit_check_noalloc(fz.FUSION_BF16, big, 0x100000, 384, head, 0x100000, None, None, None, None)
+    assert rc == fz.FUSION_ERR_WORKSPACE
+    assert fz.fusion_workspace_size(1 << 20, 1000) > (1 << 20)

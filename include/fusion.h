@@ -77,6 +77,7 @@ extern "C" {
 #define FUSION_DEV_NONFINITE 4   /* NaN/Inf in keys, scores, rho or a CLS row */
 #define FUSION_DEV_INTERNAL 8    /* an internal consistency check failed (a library bug) */
 #define FUSION_DEV_BAD_IDS 16    /* a sample id outside [0, max_batch) */
+#define FUSION_DEV_TIMEOUT 32    /* a bounded wait inside a kernel gave up (outputs of that sample skipped) */
 
 /* ---- storage types and stage flags --------------------------------------- */
 #define FUSION_F32 0

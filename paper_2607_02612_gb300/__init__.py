@@ -13,6 +13,7 @@ from ._binding import (  # noqa: F401
     FUSION_DEV_BAD_OFFSETS,
     FUSION_DEV_INTERNAL,
     FUSION_DEV_NONFINITE,
+    FUSION_DEV_TIMEOUT,
     FUSION_ERR_CUDA,
     FUSION_ERR_DTYPE,
     FUSION_ERR_INVALID_ARG,

@@ -28,6 +28,7 @@ FUSION_DEV_BAD_BATCH = 2
 FUSION_DEV_NONFINITE = 4
 FUSION_DEV_INTERNAL = 8
 FUSION_DEV_BAD_IDS = 16
+FUSION_DEV_TIMEOUT = 32
 FUSION_F32 = 0
 FUSION_BF16 = 1
 FUSION_STAGE_MERGE = 1

@@ -32,9 +32,8 @@ struct Head {
 };
 
 // Geometry shared by the exit kernel, its workspace and the host.
-constexpr int kExitBT = 32;     // samples per exit CTA
+constexpr int kExitBT = 8;      // samples per exit CTA (one LayerNorm per warp)
 constexpr int kExitCT = 128;    // classes per exit CTA
-constexpr int kExitKC = 64;     // head K chunk staged in shared memory
 constexpr int kExitThreads = 256;
 
 constexpr int kPlanThreads = 1024;
@@ -217,6 +216,15 @@ __device__ __forceinline__ F2 f2_div(F2 a, F2 b) {
     const float q2 = __fdiv_rn(r.hi, b.hi);
     return quick_two_sum(q1, q2);
 }
+// 1 / sqrt(v) for a positive float-float v: one Newton step in float-float on the
+// float32 estimate, about 44 correct bits.
+__device__ __forceinline__ F2 f2_rsqrt(F2 v) {
+    const float y = rsqrtf(v.hi);
+    const F2 vy2 = f2_mul(v, two_prod(y, y));                    // v * y^2 ~ 1
+    const F2 e = f2_add({1.0f, 0.0f}, {-vy2.hi, -vy2.lo});       // 1 - v y^2, tiny
+    const float corr = __fmul_rn(__fmul_rn(0.5f, y), e.hi);      // y e / 2
+    return quick_two_sum(y, corr);
+}
 __device__ __forceinline__ F2 f2_shfl_xor(F2 v, int m) {
     return {__shfl_xor_sync(0xFFFFFFFFu, v.hi, m), __shfl_xor_sync(0xFFFFFFFFu, v.lo, m)};
 }
@@ -242,44 +250,6 @@ __device__ __forceinline__ uint16_t f2_to_bf16_bits(F2 v) {
         if (away || (!toward && (up & 1u))) up += 1;
     }
     return (uint16_t)up;
-}
-
-// Round a double to the nearest bfloat16, ties to even, in a single step.
-__device__ __forceinline__ uint16_t double_to_bf16_bits(double d) {
-    const unsigned long long b = (unsigned long long)__double_as_longlong(d);
-    const uint32_t sign = (uint32_t)(b >> 63) << 15;
-    const int e = (int)((b >> 52) & 0x7FF);
-    unsigned long long m = b & 0x000FFFFFFFFFFFFFull;
-    if (e == 0x7FF) return (uint16_t)(sign | 0x7F80u | (m ? 0x40u : 0u));
-    if (e == 0) return (uint16_t)sign;                       // double subnormals round to 0
-    int ex = e - 1023;                                        // value = 1.m * 2^ex
-    m |= 0x0010000000000000ull;                               // 53-bit significand
-    int shift;                                                // bits to drop
-    int bexp;                                                 // biased bf16 exponent
-    if (ex >= -126) {
-        shift = 52 - 7;
-        bexp = ex + 127;
-    } else {                                                  // bf16 subnormal: spacing 2^-133
-        shift = 52 - 7 + (-126 - ex);
-        bexp = 0;
-        if (shift > 60) return (uint16_t)sign;
-    }
-    unsigned long long q = m >> shift;
-    const unsigned long long rem = m & ((1ull << shift) - 1);
-    const unsigned long long half = 1ull << (shift - 1);
-    if (rem > half || (rem == half && (q & 1ull))) q += 1;
-    uint32_t out;
-    if (bexp > 0) {
-        if (q == 0x100ull) {   // significand overflow: next binade
-            q = 0x80ull;
-            bexp += 1;
-        }
-        if (bexp >= 255) return (uint16_t)(sign | 0x7F80u);
-        out = ((uint32_t)bexp << 7) | (uint32_t)(q & 0x7Full);
-    } else {
-        out = (uint32_t)q;   // q == 0x80 becomes the smallest normal, which is the right bits
-    }
-    return (uint16_t)(sign | out);
 }
 
 // ---------------------------------------------------------------------------
@@ -321,16 +291,24 @@ __device__ __forceinline__ int block_scan_excl(int *v, int n, int *tmp) {
     return total;
 }
 
-// ceil(rho * P) with rho taken exactly (the product of a float and an integer below
-// 2^24 is exact in double), clamped to [0, P].  NaN keeps nothing; NaN and +-inf set
-// `nonfinite`.
+// ceil(rho * P) with rho taken exactly, clamped to [0, P]; NaN keeps nothing; NaN and
+// +-inf set `nonfinite`.  P < 2^24 and rho has 24 significant bits, so the product is
+// exactly p + e with p = fl(rho * P) and e = fma(rho, P, -p).  No integer lies strictly
+// between p and the exact product (integers up to 2^24 are floats and p is the nearest
+// float), so the ceiling is ceil(p), except when p is itself an integer: then it is
+// p + 1 if e > 0.
 __device__ __forceinline__ int keep_count(float rho, int P, bool &nonfinite) {
     if (isnan(rho) || isinf(rho)) nonfinite = true;
     if (P <= 0 || isnan(rho)) return 0;
-    const double v = (double)rho * (double)P;
-    if (!(v > 0.0)) return 0;
-    if (v >= (double)P) return P;
-    return (int)ceil(v);
+    const float fP = (float)P;
+    const float prod = __fmul_rn(rho, fP);
+    const float err = __fmaf_rn(rho, fP, -prod);
+    if (!(prod > 0.0f || (prod == 0.0f && err > 0.0f))) return 0;
+    if (prod >= fP) return P;
+    float c = ceilf(prod);
+    if (c == prod && err > 0.0f) c += 1.0f;
+    const int k = (int)c;
+    return k > P ? P : k;
 }
 
 __device__ __forceinline__ int merge_count(int r, int P) {

@@ -124,6 +124,15 @@ ImageParams image_params(const fusion_ragged &in, const void *x, int32_t dim, co
     return p;
 }
 
+// The per-sample kernel: TMA + tcgen05 when the shape allows it, else the general one.
+cudaError_t launch_sample_kernel(int dtype, const ImageParams &p, const ImageGeometry &G, cudaStream_t s) {
+    if (p.do_merge) {
+        const TcGeometry T = image_tc_geometry(dtype, p.in.max_tokens, p.kdim, p.in.max_rows, 1, 227);
+        if (T.ok) return launch_image_tc(p, T, s);
+    }
+    return launch_image(dtype, p, G.smem, s);
+}
+
 }  // namespace
 
 extern "C" {
@@ -150,6 +159,7 @@ const char *fusion_status_string(int code) {
         case FUSION_DEV_NONFINITE: return "device: NaN or Inf in a decision input";
         case FUSION_DEV_INTERNAL: return "device: internal consistency check failed";
         case FUSION_DEV_BAD_IDS: return "device: sample id out of range";
+        case FUSION_DEV_TIMEOUT: return "device: a bounded wait timed out";
         default: return "unknown status";
     }
 }
@@ -192,7 +202,7 @@ int fusion_merge(int dtype, fusion_ragged in, const void *x, int32_t dim, const 
     const ImageParams p = image_params(in, x, dim, keys, key_dim, sizes, scores, r, nullptr, 1, 0, w,
                                        offsets_out, x_out, sizes_out, scores_out, keep_idx, dst_map,
                                        a_match, dev_status, G);
-    const int rc = cuda_rc(launch_image(dtype, p, G.smem, s));
+    const int rc = cuda_rc(launch_sample_kernel(dtype, p, G, s));
     record(ev.end, s);
     return rc;
 }
@@ -259,7 +269,7 @@ int fusion_prune(int dtype, fusion_ragged in, const void *x, int32_t dim, const 
     const ImageParams p = image_params(in, x, dim, nullptr, dim, sizes, scores, nullptr, rho, 0, 1, w,
                                        offsets_out, x_out, sizes_out, scores_out, keep_idx, nullptr,
                                        nullptr, dev_status, G);
-    const int rc = cuda_rc(launch_image(dtype, p, G.smem, s));
+    const int rc = cuda_rc(launch_sample_kernel(dtype, p, G, s));
     record(ev.end, s);
     return rc;
 }
@@ -297,7 +307,7 @@ int fusion_compact(int dtype, fusion_ragged in, const void *x, int32_t dim, cons
     const ImageParams p = image_params(in, x, dim, nullptr, dim, sizes, scores, nullptr, nullptr, 0, 0, w,
                                        offsets_out, x_out, sizes_out, scores_out, keep_idx, nullptr,
                                        nullptr, dev_status, G);
-    const int rc = cuda_rc(launch_image(dtype, p, G.smem, s));
+    const int rc = cuda_rc(launch_sample_kernel(dtype, p, G, s));
     record(ev.end, s);
     return rc;
 }
@@ -377,7 +387,7 @@ int fusion_stage(int dtype, int flags, fusion_ragged in, const void *x, int32_t 
     const ImageParams p = image_params(in, x, dim, do_merge ? keys : nullptr, key_dim, sizes, scores, r,
                                        rho, do_merge, do_prune, w, offsets_out, x_out, sizes_out,
                                        scores_out, keep_idx, nullptr, a_match, dev_status, G);
-    const int rc = cuda_rc(launch_image(dtype, p, G.smem, s));
+    const int rc = cuda_rc(launch_sample_kernel(dtype, p, G, s));
     record(ev.end, s);
     return rc;
 }

@@ -23,57 +23,30 @@
 // that received merged A tokens, the size-weighted mean of its sources computed
 // in float-float arithmetic and rounded once (bf16: ties to even, from a value
 // with about 44 correct bits, so the rounding matches the exact mean).
-#include "launch.h"
+#include "sample.cuh"
 
 namespace fz {
 namespace {
 
 constexpr int kSPW = 2;   // output strips per warp per pass (accumulators live in registers)
 
-struct ImgLayout {
-    size_t stage_a, stage_b;
-    size_t best, ss_a, ss_b, match, sel, mflag, kflag, opos, srcpos, scnt, slist, msize, mscore, tmp;
-    size_t total;
-};
-
-__host__ __device__ inline ImgLayout img_layout(int nmax, int ra, int rb, int stage_chunks, int stage) {
-    const int nA = (nmax - 1) / 2 > 0 ? (nmax - 1) / 2 : 1;
-    const int nB = nmax / 2 > 0 ? nmax / 2 : 1;
-    ImgLayout L;
-    size_t off = 0;
-    L.stage_a = off;
-    if (stage) off += (size_t)stage_chunks * ra * 16;
-    L.stage_b = off;
-    if (stage) off += (size_t)stage_chunks * rb * 16 + 512;   // tail: padded strip rows read past the end
-    off = (off + 15) / 16 * 16;
-    L.best = off;   off += sizeof(unsigned long long) * nA;
-    L.ss_a = off;   off += sizeof(float) * nA;
-    L.ss_b = off;   off += sizeof(float) * nB;
-    L.match = off;  off += sizeof(int) * nA;
-    L.sel = off;    off += sizeof(int) * nA;
-    L.mflag = off;  off += sizeof(int) * nmax;
-    L.kflag = off;  off += sizeof(int) * nmax;
-    L.opos = off;   off += sizeof(int) * (nmax + 1);
-    L.srcpos = off; off += sizeof(int) * nmax;
-    L.scnt = off;   off += sizeof(int) * (nB + 1);
-    L.slist = off;  off += sizeof(int) * nA;
-    L.msize = off;  off += sizeof(float) * nmax;
-    L.mscore = off; off += sizeof(float) * nmax;
-    L.tmp = off;    off += sizeof(int) * 40;
-    L.total = (off + 15) / 16 * 16;
-    return L;
-}
-
 __host__ __device__ inline int rows_odd8(int n) {   // smallest R >= n with R % 8 == 1
     if (n < 1) n = 1;
     return n + ((9 - n % 8) % 8);
+}
+
+// Staging area: A region (stage_chunks x ra rows) then B region (stage_chunks x rb rows)
+// of 16-byte chunks, plus a tail for padded strip rows read past the end.
+__host__ __device__ inline size_t stage_a_bytes(int stage_chunks, int ra) { return (size_t)stage_chunks * ra * 16; }
+__host__ __device__ inline size_t stage_total(int stage_chunks, int ra, int rb) {
+    return (size_t)stage_chunks * (ra + rb) * 16 + 512;
 }
 
 // ---------------------------------------------------------------------------
 // similarity + row argmax over one sample
 // ---------------------------------------------------------------------------
 template <typename T>
-__device__ void sim_argmax(const ImageParams &p, unsigned char *sm, const ImgLayout &L, int start,
+__device__ void sim_argmax(const ImageParams &p, unsigned char *sm, size_t stage_b, MetaPtrs &m, int start,
                            int nA, int nB) {
     constexpr int CH = Elem<T>::kPerChunk;
     constexpr bool kBf16 = (Elem<T>::kBytes == 2);
@@ -81,11 +54,11 @@ __device__ void sim_argmax(const ImageParams &p, unsigned char *sm, const ImgLay
     const int g = lane >> 2, t4 = lane & 3;
     const T *keys = reinterpret_cast<const T *>(p.keys);
     const int kdim = p.kdim;
-    unsigned char *regA = sm + L.stage_a;
-    unsigned char *regB = sm + L.stage_b;
-    float *ssA = reinterpret_cast<float *>(sm + L.ss_a);
-    float *ssB = reinterpret_cast<float *>(sm + L.ss_b);
-    unsigned long long *best = reinterpret_cast<unsigned long long *>(sm + L.best);
+    unsigned char *regA = sm;
+    unsigned char *regB = sm + stage_b;
+    float *ssA = m.inv_a;   // squared norms, then inverse norms
+    float *ssB = m.inv_b;
+    unsigned long long *best = m.best;
     const int ra = p.ra, rb = p.rb;
 
     const int MT = (nA + 15) / 16, NG = (nB + 31) / 32;
@@ -277,224 +250,46 @@ __device__ void sim_argmax(const ImageParams &p, unsigned char *sm, const ImgLay
 // ---------------------------------------------------------------------------
 // the per-sample kernel
 // ---------------------------------------------------------------------------
+// Chunk c of input token pos from the chunk-major staging area (CLS from global).
 template <typename T>
-__device__ __forceinline__ uint4 load_src_chunk(const ImageParams &p, const unsigned char *sm,
-                                                const ImgLayout &L, bool from_smem, int start, int pos,
-                                                int c) {
-    constexpr int CH = Elem<T>::kPerChunk;
-    if (from_smem && pos > 0) {
-        if (pos & 1) return *reinterpret_cast<const uint4 *>(sm + L.stage_b + ((size_t)c * p.rb + (pos - 1) / 2) * 16);
-        return *reinterpret_cast<const uint4 *>(sm + L.stage_a + ((size_t)c * p.ra + (pos - 2) / 2) * 16);
+struct ChunkMajorLoader {
+    const unsigned char *regA, *regB;
+    int ra, rb;
+    GlobalLoader<T> g;
+    __device__ __forceinline__ uint4 operator()(int pos, int c) const {
+        if (pos == 0) return g(0, c);
+        if (pos & 1) return *reinterpret_cast<const uint4 *>(regB + ((size_t)c * rb + (pos - 1) / 2) * 16);
+        return *reinterpret_cast<const uint4 *>(regA + ((size_t)c * ra + (pos - 2) / 2) * 16);
     }
-    return ldg16(reinterpret_cast<const T *>(p.x) + ((long long)start + pos) * p.dim + c * CH);
-}
-
-__device__ __forceinline__ uint4 pack_chunk(const F2 (&q)[4]) {
-    return make_uint4(__float_as_uint(q[0].hi), __float_as_uint(q[1].hi), __float_as_uint(q[2].hi),
-                      __float_as_uint(q[3].hi));
-}
-__device__ __forceinline__ uint4 pack_chunk(const F2 (&q)[8]) {
-    uint32_t w[4];
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-        w[k] = (uint32_t)f2_to_bf16_bits(q[2 * k]) | ((uint32_t)f2_to_bf16_bits(q[2 * k + 1]) << 16);
-    return make_uint4(w[0], w[1], w[2], w[3]);
-}
+};
 
 template <typename T>
 __global__ void __launch_bounds__(kImageThreads, 1) k_image(ImageParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
     constexpr int CH = Elem<T>::kPerChunk;
+    SampleInfo s;
+    if (!sample_info(p, blockIdx.x, s)) return;
     const int tid = threadIdx.x;
-    const int i = blockIdx.x;
-    const int B = device_batch(p.in);
-    if (B < 0 || i >= B) return;
-    if (p.plan[0] == 0) return;
-    const int j = p.slot[i];
-    if (j < 0) return;
-
-    const int start = p.in.offsets[i];
-    const int N = p.in.offsets[i + 1] - start;
-    const int out_start = p.offsets_out[j];
-    const int out_n = p.offsets_out[j + 1] - out_start;
-    const int id = p.in.ids ? p.in.ids[i] : i;
-    const int P = N - 1, nA = P / 2, nB = (P + 1) / 2;
-    const int r_eff = p.do_merge ? merge_count(p.r[id], P) : 0;
-    const bool decide = p.do_merge && nA > 0 && (r_eff > 0 || p.need_match);
-
     const int stage_chunks = p.resident ? p.kdim / CH : p.kc / CH;
-    const ImgLayout L = img_layout(p.in.max_tokens, p.ra, p.rb, stage_chunks, p.do_merge);
-    unsigned long long *best = reinterpret_cast<unsigned long long *>(sm + L.best);
-    float *ssA = reinterpret_cast<float *>(sm + L.ss_a);
-    float *ssB = reinterpret_cast<float *>(sm + L.ss_b);
-    int *match = reinterpret_cast<int *>(sm + L.match);
-    int *sel = reinterpret_cast<int *>(sm + L.sel);
-    int *mflag = reinterpret_cast<int *>(sm + L.mflag);
-    int *kflag = reinterpret_cast<int *>(sm + L.kflag);
-    int *opos = reinterpret_cast<int *>(sm + L.opos);
-    int *srcpos = reinterpret_cast<int *>(sm + L.srcpos);
-    int *scnt = reinterpret_cast<int *>(sm + L.scnt);
-    int *slist = reinterpret_cast<int *>(sm + L.slist);
-    float *msize = reinterpret_cast<float *>(sm + L.msize);
-    float *mscore = reinterpret_cast<float *>(sm + L.mscore);
-    int *tmp = reinterpret_cast<int *>(sm + L.tmp);
-
-    for (int m = tid; m < nA; m += kImageThreads) {
-        best[m] = 0ull;
-        ssA[m] = 0.0f;
-        sel[m] = 0;
-        match[m] = 0;
-    }
-    for (int n = tid; n <= nB; n += kImageThreads) {
-        if (n < nB) ssB[n] = 0.0f;
-        scnt[n] = 0;
-    }
+    const size_t stage_b = p.do_merge ? stage_a_bytes(stage_chunks, p.ra) : 0;
+    const size_t stage = p.do_merge ? stage_total(stage_chunks, p.ra, p.rb) : 0;
+    MetaPtrs m(sm, meta_layout(p.in.max_tokens, stage));
+    meta_init<kImageThreads>(p, s, m);
+    for (int a = tid; a < s.nA; a += kImageThreads) m.inv_a[a] = 0.0f;
+    for (int n = tid; n < s.nB; n += kImageThreads) m.inv_b[n] = 0.0f;
     __syncthreads();
 
-    // ---- merge decisions: pair every A token with its best B token, keep the r best
-    if (decide) {
-        sim_argmax<T>(p, sm, L, start, nA, nB);
-        for (int m = tid; m < nA; m += kImageThreads)
-            match[m] = (int)(0xFFFFFFFFu - (uint32_t)(best[m] & 0xFFFFFFFFull));
-        if (r_eff > 0) {
-            for (int m = tid; m < nA; m += kImageThreads) {
-                const unsigned long long km = (best[m] & 0xFFFFFFFF00000000ull) | (0xFFFFFFFFull - (unsigned)m);
-                int rank = 0;
-                for (int q = 0; q < nA; ++q) {
-                    const unsigned long long kq = (best[q] & 0xFFFFFFFF00000000ull) | (0xFFFFFFFFull - (unsigned)q);
-                    rank += (kq > km) ? 1 : 0;
-                }
-                sel[m] = rank < r_eff ? 1 : 0;
-            }
-        }
-        __syncthreads();
+    // merge decisions: pair every A token with its best B token, keep the r best
+    if (s.decide) {
+        sim_argmax<T>(p, sm, stage_b, m, s.start, s.nA, s.nB);
+        select_top_r<kImageThreads>(s, m);
     }
-
-    // ---- merged token set: survivors keep ascending position ------------------------
-    for (int pos = tid; pos < N; pos += kImageThreads)
-        mflag[pos] = (pos >= 2 && !(pos & 1) && sel[(pos - 2) / 2]) ? 0 : 1;
-    if (r_eff > 0)
-        for (int m = tid; m < nA; m += kImageThreads)
-            if (sel[m]) atomicAdd(&scnt[match[m]], 1);
-    __syncthreads();
-    block_scan_excl(scnt, nB + 1, tmp);   // scnt[n] = first slot of B token n's sources
-    if (r_eff > 0) {
-        for (int m = tid; m < nA; m += kImageThreads) {
-            if (!sel[m]) continue;
-            const int n = match[m];
-            int before = 0;
-            for (int q = 0; q < m; ++q) before += (sel[q] && match[q] == n) ? 1 : 0;
-            slist[scnt[n] + before] = m;   // sources of every B token in ascending A order
-        }
-    }
-    __syncthreads();
-
-    // merged sizes and scores (sums over the sources, exact in double)
-    for (int pos = tid; pos < N; pos += kImageThreads) {
-        if (!mflag[pos]) continue;
-        double sz = p.sizes[start + pos];
-        double sc = p.scores ? (double)p.scores[start + pos] : 0.0;
-        if (pos & 1) {
-            const int n = (pos - 1) / 2;
-            for (int q = scnt[n]; q < scnt[n + 1]; ++q) {
-                const int a = start + 2 + 2 * slist[q];
-                sz += p.sizes[a];
-                if (p.scores) sc += (double)p.scores[a];
-            }
-        }
-        msize[pos] = (float)sz;
-        mscore[pos] = (float)sc;
-        if (p.scores && !isfinite(mscore[pos]) && pos > 0) raise_status(p.status, FUSION_DEV_NONFINITE);
-    }
-    __syncthreads();
-
-    // ---- prune: CLS + the k highest merged scores, lowest position on ties -----------
-    if (p.do_prune) {
-        bool nf = false;
-        const int k = keep_count(p.rho[id], N - r_eff - 1, nf);
-        for (int pos = tid; pos < N; pos += kImageThreads) {
-            int keep = 0;
-            if (pos == 0) {
-                keep = 1;
-            } else if (mflag[pos]) {
-                const unsigned long long kp = rank_key(mscore[pos], pos);
-                int rank = 0;
-                for (int q = 1; q < N; ++q)
-                    rank += (mflag[q] && rank_key(mscore[q], q) > kp) ? 1 : 0;
-                keep = rank < k ? 1 : 0;
-            }
-            kflag[pos] = keep;
-            opos[pos] = keep;
-        }
+    const GlobalLoader<T> gl{reinterpret_cast<const T *>(p.x), (long long)s.start, p.dim};
+    if (s.decide && p.resident && p.keys_alias) {
+        const ChunkMajorLoader<T> ld{sm, sm + stage_b, p.ra, p.rb, gl};
+        finish_sample<T, kImageThreads>(p, s, m, ld);
     } else {
-        for (int pos = tid; pos < N; pos += kImageThreads) {
-            kflag[pos] = mflag[pos];
-            opos[pos] = mflag[pos];
-        }
-    }
-    __syncthreads();
-    const int total = block_scan_excl(opos, N, tmp);
-    if (total != out_n) {   // the plan and the decisions disagree: a library bug
-        if (tid == 0) raise_status(p.status, FUSION_DEV_INTERNAL);
-        return;
-    }
-    for (int pos = tid; pos < N; pos += kImageThreads)
-        if (kflag[pos]) srcpos[opos[pos]] = pos;
-    __syncthreads();
-
-    // ---- index outputs ----------------------------------------------------------------
-    for (int o = tid; o < out_n; o += kImageThreads) {
-        const int pos = srcpos[o];
-        const long long orow = (long long)out_start + o;
-        p.sizes_out[orow] = msize[pos];
-        if (p.scores_out) p.scores_out[orow] = mscore[pos];
-        if (p.keep_idx) p.keep_idx[orow] = start + pos;
-    }
-    if (p.a_match)
-        for (int pos = tid; pos < N; pos += kImageThreads)
-            p.a_match[start + pos] = (pos >= 2 && !(pos & 1)) ? start + 1 + 2 * match[(pos - 2) / 2] : -1;
-    if (p.dst_map && !p.do_prune)
-        for (int pos = tid; pos < N; pos += kImageThreads) {
-            const bool gone = pos >= 2 && !(pos & 1) && sel[(pos - 2) / 2];
-            const int dest = gone ? 1 + 2 * match[(pos - 2) / 2] : pos;
-            p.dst_map[start + pos] = out_start + opos[dest];
-        }
-
-    // ---- token rows: copies and size-weighted means, 16 bytes per thread --------------
-    const int ncx = p.dim / CH;
-    const bool from_smem = decide && p.resident && p.keys_alias;
-    T *xo = reinterpret_cast<T *>(p.x_out);
-    for (int it = tid; it < out_n * ncx; it += kImageThreads) {
-        const int o = it / ncx, c = it - o * ncx;
-        const int pos = srcpos[o];
-        const uint4 self = load_src_chunk<T>(p, sm, L, from_smem, start, pos, c);
-        uint4 outv = self;
-        if (pos & 1) {
-            const int n = (pos - 1) / 2;
-            const int q0 = scnt[n], q1 = scnt[n + 1];
-            if (q1 > q0) {
-                float f[CH];
-                chunk_to_f(self, f);
-                const float sb = p.sizes[start + pos];
-                F2 den = {sb, 0.0f};
-                F2 num[CH];
-#pragma unroll
-                for (int e = 0; e < CH; ++e) num[e] = two_prod(sb, f[e]);
-                for (int q = q0; q < q1; ++q) {
-                    const int apos = 2 + 2 * slist[q];
-                    const float sa = p.sizes[start + apos];
-                    den = f2_add_f(den, sa);
-                    chunk_to_f(load_src_chunk<T>(p, sm, L, from_smem, start, apos, c), f);
-#pragma unroll
-                    for (int e = 0; e < CH; ++e) num[e] = f2_add(num[e], two_prod(sa, f[e]));
-                }
-                F2 qv[CH];
-#pragma unroll
-                for (int e = 0; e < CH; ++e) qv[e] = f2_div(num[e], den);
-                outv = pack_chunk(qv);
-            }
-        }
-        *reinterpret_cast<uint4 *>(xo + ((long long)out_start + o) * p.dim + c * CH) = outv;
+        finish_sample<T, kImageThreads>(p, s, m, gl);
     }
 }
 
@@ -508,14 +303,13 @@ ImageGeometry image_geometry(int dtype, int max_tokens, int kdim, int do_merge) 
     G.ra = rows_odd8(nA);
     G.rb = rows_odd8(nB);
     constexpr size_t kBudget = 227 * 1024 - 2048;   // leave room for static shared memory
-    const size_t meta = img_layout(max_tokens, G.ra, G.rb, 0, 0).total;
+    const size_t meta = meta_layout(max_tokens, 0).total;
     if (!do_merge) {
         G.ok = meta <= kBudget;
         G.smem = meta;
         return G;
     }
-    const size_t per_dim = (size_t)(G.ra + G.rb) * eb;   // staged bytes per key dim
-    const size_t full = img_layout(max_tokens, G.ra, G.rb, kdim / CH, 1).total;
+    const size_t full = meta_layout(max_tokens, stage_total(kdim / CH, G.ra, G.rb)).total;
     if (full <= kBudget) {
         G.ok = 1;
         G.resident = 1;
@@ -523,6 +317,7 @@ ImageGeometry image_geometry(int dtype, int max_tokens, int kdim, int do_merge) 
         G.smem = full;
         return G;
     }
+    const size_t per_dim = (size_t)(G.ra + G.rb) * eb;   // staged bytes per key dim
     if (meta + 1024 >= kBudget) return G;
     int kc = (int)((kBudget - meta - 1024) / per_dim) / 16 * 16;
     if (kc > kdim) kc = kdim;
@@ -530,7 +325,7 @@ ImageGeometry image_geometry(int dtype, int max_tokens, int kdim, int do_merge) 
     G.ok = 1;
     G.resident = 0;
     G.kc = kc;
-    G.smem = img_layout(max_tokens, G.ra, G.rb, kc / CH, 1).total;
+    G.smem = meta_layout(max_tokens, stage_total(kc / CH, G.ra, G.rb)).total;
     return G;
 }
 

@@ -1,0 +1,376 @@
+// Per-sample merge -> prune -> gather for bf16 tokens on the 5th-generation tensor
+// cores (tcgen05) with TMA, for samples of at most 257 tokens (|A|, |B| <= 128).
+//
+// One CTA of 256 threads per input sample.  The keys of half A (even positions) and
+// half B (odd positions) arrive by TMA tensor loads in K-blocks of 64 dims, 128-byte
+// swizzled: K-block kb of a half is a [rows][128 B] tile, 16-byte chunk j of row t
+// stored at chunk position j ^ (t % 8).  Two tensor maps per parity of the global row
+// index (every other row of the token matrix) cover boxes of 32 and 8 rows, so any
+// half of any sample loads in whole 8-row groups.  The K-blocks stream through a ring
+// of stages (the whole sample stays resident when it fits).
+//
+// Thread 0 produces (TMA), thread 32 issues tcgen05.mma (M = 128 A rows, N = |B|
+// rounded up to 16, K = 16 per instruction, f32 accumulation in tensor memory), and
+// every thread accumulates the squared norm of one A or B row from the same stages.
+// A stage is released when the MMAs that read it completed (tcgen05.commit) and all
+// warps are done with it.  The epilogue reads S from tensor memory, one A row per
+// thread (two warpgroups split the columns), forms cos = dot * inv|a| * inv|b| and
+// keeps the largest value with the lowest B index.  Everything after the decisions
+// (top-r, merged set, sums, pruning, gather) is the shared finish phase.
+//
+// Every wait on an mbarrier is bounded; on a timeout the CTA raises
+// FUSION_DEV_TIMEOUT, skips its outputs and frees its tensor memory.
+#include <cuda.h>
+
+#include "sample.cuh"
+
+namespace fz {
+namespace {
+
+constexpr int kTcThreads = 256;
+constexpr int kMaxStages = 16;
+constexpr uint32_t kWaitSpins = 1u << 22;
+
+struct TcMaps {
+    CUtensorMap e32, o32, e8, o8;   // even / odd rows, boxes of 32 / 8 rows x 64 dims
+};
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+// Bounded wait for the completion of the phase with the given parity.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+    for (uint32_t it = 0; it < kWaitSpins; ++it) {
+        uint32_t done;
+        asm volatile(
+            "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+            : "=r"(done)
+            : "r"(bar), "r"(parity)
+            : "memory");
+        if (done) return true;
+    }
+    return false;
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+            dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups 1024 B apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t addr) {
+    return (uint64_t)((addr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) | (1ull << 46) |
+           (2ull << 61);
+}
+__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate) {
+    asm volatile(
+        "{ .reg .pred p; setp.ne.b32 p, %4, 0; tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p; }" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+          "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Chunk c of input token pos from the resident swizzled stages (CLS from global).
+struct SwizzledLoader {
+    const unsigned char *regA, *regB;
+    uint32_t kbA, kbB;   // bytes of one K-block of each half
+    GlobalLoader<__nv_bfloat16> g;
+    __device__ __forceinline__ uint4 operator()(int pos, int c) const {
+        if (pos == 0) return g(0, c);
+        const bool isB = pos & 1;
+        const int r = isB ? (pos - 1) >> 1 : (pos - 2) >> 1;
+        const unsigned char *base = (isB ? regB : regA) + (size_t)(c >> 3) * (isB ? kbB : kbA);
+        return *reinterpret_cast<const uint4 *>(base + r * 128 + (((c & 7) ^ (r & 7)) << 4));
+    }
+};
+
+__global__ void __launch_bounds__(kTcThreads, 1)
+    k_image_tc(const __grid_constant__ TcMaps maps, ImageParams p, TcGeometry g) {
+    extern __shared__ unsigned char sm_raw[];
+    unsigned char *sm = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~uintptr_t(1023));
+    __shared__ __align__(8) unsigned long long bar_full[kMaxStages], bar_empty[kMaxStages], bar_done;
+    __shared__ uint32_t tmem_base;
+    __shared__ int s_fail;
+    __shared__ unsigned long long half_best[kTcThreads / 2];
+
+    SampleInfo s;
+    if (!sample_info(p, blockIdx.x, s)) return;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    MetaPtrs m(sm, meta_layout(p.in.max_tokens, g.meta_base));
+    meta_init<kTcThreads>(p, s, m);
+    const bool dec = s.decide;
+    const int S = g.stages, nkb = g.n_kb;
+    unsigned char *regA = sm + g.stage_a;   // stage st, half A: regA + st * kbA
+    unsigned char *regB = sm + g.stage_b;
+
+    if (tid == 0) {
+        s_fail = 0;
+        if (dec) {
+            for (int st = 0; st < S; ++st) {
+                mbar_init(smem_addr(&bar_full[st]), 1);
+                mbar_init(smem_addr(&bar_empty[st]), 1 + kTcThreads / 32);
+            }
+            mbar_init(smem_addr(&bar_done), 1);
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        }
+    }
+    if (dec && warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(&tmem_base)),
+                     "r"(g.tmem_cols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+
+    if (dec) {
+        const uint32_t tmem = tmem_base;
+        const int rowsA = (s.nA + 7) & ~7, rowsB = (s.nB + 7) & ~7;
+        const uint32_t kb_tx = (uint32_t)(rowsA + rowsB) * 128u;
+        const int yA = (s.start + 2) >> 1, yB = (s.start + 1) >> 1;
+        const bool oddA = (s.start + 2) & 1, oddB = (s.start + 1) & 1;
+        // K-block kb of both halves into stage kb % S
+        auto produce = [&](int kb) {
+            const int st = kb % S;
+            const uint32_t bar = smem_addr(&bar_full[st]);
+            mbar_expect_tx(bar, kb_tx);
+            const uint32_t dA = smem_addr(regA + (size_t)st * g.kb_a), dB = smem_addr(regB + (size_t)st * g.kb_b);
+            for (int half = 0; half < 2; ++half) {
+                const int n = half ? s.nB : s.nA;
+                const bool odd = half ? oddB : oddA;
+                const int y0 = half ? yB : yA;
+                const uint32_t d0 = half ? dB : dA;
+                int done = 0;
+                for (; n - done >= 32; done += 32)
+                    tma_load_2d(d0 + done * 128, odd ? &maps.o32 : &maps.e32, kb * 64, y0 + done, bar);
+                for (; done < n; done += 8)
+                    tma_load_2d(d0 + done * 128, odd ? &maps.o8 : &maps.e8, kb * 64, y0 + done, bar);
+            }
+        };
+        if (tid == 0)
+            for (int kb = 0; kb < S && kb < nkb; ++kb) produce(kb);
+
+        // instruction descriptor: f32 accumulator, bf16 A and B, K-major, N = |B| rounded to 16, M = 128
+        const int npad = (s.nB + 15) & ~15;
+        const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(npad >> 3) << 17) | (8u << 24);
+        const bool isA = tid < 128;
+        const int row = isA ? tid : tid - 128;
+        const bool has_row = row < (isA ? s.nA : s.nB);
+        float ss = 0.0f, sc = 0.0f;
+        bool ok = true;
+        for (int kb = 0; kb < nkb; ++kb) {
+            const int st = kb % S;
+            const uint32_t par = (uint32_t)(kb / S) & 1u;
+            if (!mbar_wait(smem_addr(&bar_full[st]), par)) {
+                ok = false;
+                break;
+            }
+            if (tid == 32) {
+                const uint32_t a0 = smem_addr(regA + (size_t)st * g.kb_a), b0 = smem_addr(regB + (size_t)st * g.kb_b);
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                    umma_bf16(tmem, sw128_desc(a0 + k * 32), sw128_desc(b0 + k * 32), idesc, (kb | k) ? 1u : 0u);
+                umma_commit(smem_addr(&bar_empty[st]));
+                if (kb == nkb - 1) umma_commit(smem_addr(&bar_done));
+            }
+            if (has_row) {   // squared norm of this thread's row, chunk by chunk
+                const unsigned char *base = (isA ? regA + (size_t)st * g.kb_a : regB + (size_t)st * g.kb_b) + row * 128;
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    float f[8];
+                    chunk_to_f(*reinterpret_cast<const uint4 *>(base + ((j ^ (row & 7)) << 4)), f);
+                    float part = 0.0f;
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) part = fmaf(f[e], f[e], part);
+                    const float t = __fadd_rn(ss, part);   // Neumaier-compensated sum of the chunk sums
+                    sc = __fadd_rn(sc, fabsf(ss) >= fabsf(part) ? __fadd_rn(__fsub_rn(ss, t), part)
+                                                               : __fadd_rn(__fsub_rn(part, t), ss));
+                    ss = t;
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_addr(&bar_empty[st]));
+            if (tid == 0 && kb + S < nkb) {   // refill this stage once everyone is done with it
+                if (!mbar_wait(smem_addr(&bar_empty[st]), par)) {
+                    ok = false;
+                    break;
+                }
+                produce(kb + S);
+            }
+        }
+        if (!ok) atomicOr(&s_fail, 1);
+        if (has_row) {
+            const float sq = __fadd_rn(ss, sc);
+            if (!isfinite(sq)) raise_status(p.status, FUSION_DEV_NONFINITE);
+            const float inv = 1.0f / fmaxf(sqrtf(sq), 1e-12f);
+            if (isA)
+                m.inv_a[row] = inv;
+            else
+                m.inv_b[row] = inv;
+        }
+        __syncthreads();
+        bool mma_ok = s_fail == 0 && mbar_wait(smem_addr(&bar_done), 0);
+        if (!mma_ok) atomicOr(&s_fail, 2);
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        __syncthreads();
+        if (s_fail == 0) {
+            // epilogue: thread -> A row (tid % 128); the two warpgroups take the low / high columns
+            const int wg = tid >> 7;
+            const int r = tid & 127;
+            const int half_cols = ((npad / 16 + 1) / 2) * 16;
+            const int c_lo = wg ? half_cols : 0, c_hi = wg ? npad : half_cols;
+            const uint32_t lane_addr = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+            const float ia = r < s.nA ? m.inv_a[r] : 0.0f;
+            unsigned long long bk = 0ull;
+            for (int c0 = c_lo; c0 < c_hi; c0 += 16) {
+                uint32_t v[16];
+                tmem_ld16(lane_addr + (uint32_t)c0, v);
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    const int col = c0 + e;
+                    if (r < s.nA && col < s.nB) {
+                        const float cs = (__uint_as_float(v[e]) * ia) * m.inv_b[col];
+                        const unsigned long long k = rank_key(cs, col);
+                        bk = k > bk ? k : bk;
+                    }
+                }
+            }
+            if (wg == 1) half_best[r] = bk;
+            __syncthreads();
+            if (wg == 0 && r < s.nA) {
+                const unsigned long long o = half_best[r];
+                m.best[r] = o > bk ? o : bk;
+            }
+        } else {
+            if (tid == 0) raise_status(p.status, FUSION_DEV_TIMEOUT);
+        }
+        __syncthreads();
+        if (s_fail == 0) select_top_r<kTcThreads>(s, m);
+    }
+
+    if (s_fail == 0) {
+        const GlobalLoader<__nv_bfloat16> gl{reinterpret_cast<const __nv_bfloat16 *>(p.x), (long long)s.start, p.dim};
+        if (dec && g.stages >= g.n_kb && p.keys_alias) {
+            const SwizzledLoader ld{regA, regB, g.kb_a, g.kb_b, gl};
+            finish_sample<__nv_bfloat16, kTcThreads>(p, s, m, ld);
+        } else {
+            finish_sample<__nv_bfloat16, kTcThreads>(p, s, m, gl);
+        }
+    }
+    if (dec) {
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncthreads();
+        if (warp == 0)
+            asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(g.tmem_cols)
+                         : "memory");
+    }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static bool tried = false;
+    if (!tried) {
+        tried = true;
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(f);
+    }
+    return fn;
+}
+
+int ceil8(int v) { return (v + 7) & ~7; }
+
+}  // namespace
+
+TcGeometry image_tc_geometry(int dtype, int max_tokens, int kdim, long long max_rows, int do_merge,
+                             int stage_budget_kb) {
+    TcGeometry g{};
+    if (dtype != FUSION_BF16 || !do_merge || kdim % 64 != 0 || max_rows < 2) return g;
+    const int nAmax = (max_tokens - 1) / 2, nBmax = max_tokens / 2;
+    if (nAmax > 128 || nBmax > 128) return g;
+    g.n_kb = kdim / 64;
+    g.kb_a = (uint32_t)ceil8(nAmax > 0 ? nAmax : 1) * 128u;
+    g.kb_b = (uint32_t)ceil8(nBmax > 0 ? nBmax : 1) * 128u;
+    int cols = 32;
+    while (cols < ((nBmax + 15) & ~15)) cols <<= 1;
+    g.tmem_cols = cols;
+    const size_t meta = meta_layout(max_tokens, 0).total;
+    const size_t per_stage = g.kb_a + g.kb_b;
+    // the padded MMA rows of the last stage read past the end: 2 KB of tail
+    const size_t budget = (size_t)stage_budget_kb * 1024;
+    int S = g.n_kb;
+    while (S > 2 && (size_t)S * per_stage + 2048 + meta + 1024 > budget) --S;
+    if (S > kMaxStages) S = kMaxStages;
+    if ((size_t)S * per_stage + 2048 + meta + 1024 > 227 * 1024 - 4096) return g;
+    g.stages = S;
+    g.stage_a = 0;
+    g.stage_b = (uint32_t)(S * g.kb_a);
+    g.meta_base = (uint32_t)(S * per_stage + 2048);
+    // an M = 128 MMA reads 16 row groups (16 KB) of half A from the last stage on
+    const size_t a_reach = (size_t)(S - 1) * g.kb_a + 16384;
+    size_t total = meta_layout(max_tokens, g.meta_base).total;
+    if (a_reach > total) total = a_reach;
+    g.smem = total + 1024;
+    if (g.smem > 227 * 1024) return TcGeometry{};
+    g.ok = 1;
+    return g;
+}
+
+cudaError_t launch_image_tc(const ImageParams &p, const TcGeometry &g, cudaStream_t s) {
+    if (p.in.max_batch == 0) return cudaSuccess;
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    TcMaps maps;
+    const cuuint64_t rows_even = (cuuint64_t)((p.in.max_rows + 1) / 2), rows_odd = (cuuint64_t)(p.in.max_rows / 2);
+    const char *keys = reinterpret_cast<const char *>(p.keys);
+    for (int i = 0; i < 4; ++i) {
+        const int odd = i & 1, box_rows = i < 2 ? 32 : 8;
+        cuuint64_t dims[2] = {(cuuint64_t)p.kdim, odd ? rows_odd : rows_even};
+        cuuint64_t strides[1] = {(cuuint64_t)p.kdim * 2 * 2};   // every other row
+        cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
+        cuuint32_t estr[2] = {1, 1};
+        CUtensorMap *dst = i == 0 ? &maps.e32 : i == 1 ? &maps.o32 : i == 2 ? &maps.e8 : &maps.o8;
+        void *base = const_cast<char *>(keys + (odd ? (size_t)p.kdim * 2 : 0));
+        if (enc(dst, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
+    cudaError_t e = cudaFuncSetAttribute(k_image_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)g.smem);
+    if (e != cudaSuccess) return e;
+    k_image_tc<<<p.in.max_batch, kTcThreads, g.smem, s>>>(maps, p, g);
+    return cudaGetLastError();
+}
+
+}  // namespace fz

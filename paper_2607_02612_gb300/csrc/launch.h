@@ -72,4 +72,19 @@ struct ImageGeometry {
 ImageGeometry image_geometry(int dtype, int max_tokens, int kdim, int do_merge);
 cudaError_t launch_image(int dtype, const ImageParams &p, size_t smem, cudaStream_t s);
 
+// ---- per-sample kernel on TMA + tcgen05 (bf16, |A|, |B| <= 128, key width % 64 == 0) ----
+struct TcGeometry {
+    int ok;
+    int n_kb;          // key K-blocks of 64 dims
+    int stages;        // K-block stages in shared memory (all n_kb: the sample stays resident)
+    int tmem_cols;     // tensor-memory columns allocated per CTA
+    uint32_t kb_a, kb_b;             // bytes of one K-block of half A / half B
+    uint32_t stage_a, stage_b;       // offsets of the two halves' stages
+    uint32_t meta_base;              // offset of the per-sample metadata
+    size_t smem;                     // dynamic shared memory bytes (with 1 KB alignment slack)
+};
+TcGeometry image_tc_geometry(int dtype, int max_tokens, int kdim, long long max_rows, int do_merge,
+                             int stage_budget_kb);
+cudaError_t launch_image_tc(const ImageParams &p, const TcGeometry &g, cudaStream_t s);
+
 }  // namespace fz

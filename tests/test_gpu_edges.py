@@ -145,6 +145,26 @@ def test_ids_index_router_outputs():
     np.testing.assert_array_equal(g["ids"][:3], b.ids)
 
 
+def test_prune_keep_count_is_exact():
+    """k = ceil(rho * P) on the exact product, including rho one float step either side of
+    k/P (where a rounded product would land on the integer)."""
+    rng = np.random.default_rng(12)
+    counts, rhos = [], []
+    for P in (1, 2, 3, 5, 7, 10, 64, 96, 196, 576, 1023):
+        for kk in sorted({0, 1, P // 3, P // 2, P - 1, P}):
+            base = np.float32(kk / P)
+            for r in (np.nextafter(base, np.float32(0)), base, np.nextafter(base, np.float32(2))):
+                counts.append(P + 1)
+                rhos.append(r)
+    counts += [6, 11, 197]
+    rhos += [np.float32(0.4), np.float32(0.1), np.float32(0.7)]
+    b = make_batch(counts, 16, "f32", seed=13)
+    b.scores = rng.random(len(b.scores)).astype(np.float32)
+    spec = StageSpec(False, False, True, r=np.zeros(len(counts), np.int32), rho=np.array(rhos, np.float32))
+    g, o = run_stage_and_compare(b, spec, "keep counts")
+    np.testing.assert_array_equal(g["offsets"][:len(counts) + 1], o["offsets"])
+
+
 def test_largest_sample():
     b = make_batch([fz.FUSION_MAX_TOKENS, 3], 16, "bf16", seed=6)
     spec = StageSpec(True, False, True, r=np.array([300, 1], np.int32), rho=np.array([0.37, 1.0], np.float32))

@@ -124,10 +124,15 @@ ImageParams image_params(const fusion_ragged &in, const void *x, int32_t dim, co
     return p;
 }
 
+// Dynamic shared memory per CTA of the tcgen05 kernel: two CTAs share an SM's 228 KB
+// (1 KB of it reserved per CTA, plus the kernel's static shared memory), so that one
+// CTA's decisions and gather overlap the other's loads.
+constexpr int kTcSmemBudgetKb = 111;
+
 // The per-sample kernel: TMA + tcgen05 when the shape allows it, else the general one.
 cudaError_t launch_sample_kernel(int dtype, const ImageParams &p, const ImageGeometry &G, cudaStream_t s) {
     if (p.do_merge) {
-        const TcGeometry T = image_tc_geometry(dtype, p.in.max_tokens, p.kdim, p.in.max_rows, 1, 227);
+        const TcGeometry T = image_tc_geometry(dtype, p.in.max_tokens, p.kdim, p.in.max_rows, 1, kTcSmemBudgetKb);
         if (T.ok) return launch_image_tc(p, T, s);
     }
     return launch_image(dtype, p, G.smem, s);

@@ -102,7 +102,7 @@ struct SwizzledLoader {
     }
 };
 
-__global__ void __launch_bounds__(kTcThreads, 1)
+__global__ void __launch_bounds__(kTcThreads, 2)
     k_image_tc(const __grid_constant__ TcMaps maps, ImageParams p, TcGeometry g) {
     extern __shared__ unsigned char sm_raw[];
     unsigned char *sm = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~uintptr_t(1023));
@@ -114,13 +114,34 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     SampleInfo s;
     if (!sample_info(p, blockIdx.x, s)) return;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    MetaPtrs m(sm, meta_layout(p.in.max_tokens, g.meta_base));
-    meta_init<kTcThreads>(p, s, m);
     const bool dec = s.decide;
     const int S = g.stages, nkb = g.n_kb;
     unsigned char *regA = sm + g.stage_a;   // stage st, half A: regA + st * kbA
     unsigned char *regB = sm + g.stage_b;
+    const int rowsA = (s.nA + 7) & ~7, rowsB = (s.nB + 7) & ~7;
+    const uint32_t kb_tx = (uint32_t)(rowsA + rowsB) * 128u;
+    const int yA = (s.start + 2) >> 1, yB = (s.start + 1) >> 1;
+    const bool oddA = (s.start + 2) & 1, oddB = (s.start + 1) & 1;
+    // K-block kb of both halves into stage kb % S
+    auto produce = [&](int kb) {
+        const int st = kb % S;
+        const uint32_t bar = smem_addr(&bar_full[st]);
+        mbar_expect_tx(bar, kb_tx);
+        const uint32_t dA = smem_addr(regA + (size_t)st * g.kb_a), dB = smem_addr(regB + (size_t)st * g.kb_b);
+        for (int half = 0; half < 2; ++half) {
+            const int n = half ? s.nB : s.nA;
+            const bool odd = half ? oddB : oddA;
+            const int y0 = half ? yB : yA;
+            const uint32_t d0 = half ? dB : dA;
+            int done = 0;
+            for (; n - done >= 32; done += 32)
+                tma_load_2d(d0 + done * 128, odd ? &maps.o32 : &maps.e32, kb * 64, y0 + done, bar);
+            for (; done < n; done += 8)
+                tma_load_2d(d0 + done * 128, odd ? &maps.o8 : &maps.e8, kb * 64, y0 + done, bar);
+        }
+    };
 
+    // the first stages' loads go out before anything else
     if (tid == 0) {
         s_fail = 0;
         if (dec) {
@@ -131,8 +152,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             mbar_init(smem_addr(&bar_done), 1);
             asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            for (int kb = 0; kb < S && kb < nkb; ++kb) produce(kb);
         }
     }
+    MetaPtrs m(sm, meta_layout(p.in.max_tokens, g.meta_base));
+    meta_init<kTcThreads>(p, s, m);
+    __syncwarp();
     if (dec && warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(&tmem_base)),
                      "r"(g.tmem_cols)
@@ -145,30 +170,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 
     if (dec) {
         const uint32_t tmem = tmem_base;
-        const int rowsA = (s.nA + 7) & ~7, rowsB = (s.nB + 7) & ~7;
-        const uint32_t kb_tx = (uint32_t)(rowsA + rowsB) * 128u;
-        const int yA = (s.start + 2) >> 1, yB = (s.start + 1) >> 1;
-        const bool oddA = (s.start + 2) & 1, oddB = (s.start + 1) & 1;
-        // K-block kb of both halves into stage kb % S
-        auto produce = [&](int kb) {
-            const int st = kb % S;
-            const uint32_t bar = smem_addr(&bar_full[st]);
-            mbar_expect_tx(bar, kb_tx);
-            const uint32_t dA = smem_addr(regA + (size_t)st * g.kb_a), dB = smem_addr(regB + (size_t)st * g.kb_b);
-            for (int half = 0; half < 2; ++half) {
-                const int n = half ? s.nB : s.nA;
-                const bool odd = half ? oddB : oddA;
-                const int y0 = half ? yB : yA;
-                const uint32_t d0 = half ? dB : dA;
-                int done = 0;
-                for (; n - done >= 32; done += 32)
-                    tma_load_2d(d0 + done * 128, odd ? &maps.o32 : &maps.e32, kb * 64, y0 + done, bar);
-                for (; done < n; done += 8)
-                    tma_load_2d(d0 + done * 128, odd ? &maps.o8 : &maps.e8, kb * 64, y0 + done, bar);
-            }
-        };
-        if (tid == 0)
-            for (int kb = 0; kb < S && kb < nkb; ++kb) produce(kb);
 
         // instruction descriptor: f32 accumulator, bf16 A and B, K-major, N = |B| rounded to 16, M = 128
         const int npad = (s.nB + 15) & ~15;
@@ -328,11 +329,11 @@ TcGeometry image_tc_geometry(int dtype, int max_tokens, int kdim, long long max_
     const size_t meta = meta_layout(max_tokens, 0).total;
     const size_t per_stage = g.kb_a + g.kb_b;
     // the padded MMA rows of the last stage read past the end: 2 KB of tail
-    const size_t budget = (size_t)stage_budget_kb * 1024;
-    int S = g.n_kb;
+    size_t budget = (size_t)stage_budget_kb * 1024;
+    if (budget > 227 * 1024 - 4096) budget = 227 * 1024 - 4096;   // room for static shared memory
+    int S = g.n_kb < kMaxStages ? g.n_kb : kMaxStages;
     while (S > 2 && (size_t)S * per_stage + 2048 + meta + 1024 > budget) --S;
-    if (S > kMaxStages) S = kMaxStages;
-    if ((size_t)S * per_stage + 2048 + meta + 1024 > 227 * 1024 - 4096) return g;
+    if ((size_t)S * per_stage + 2048 + meta + 1024 > budget) return g;
     g.stages = S;
     g.stage_a = 0;
     g.stage_b = (uint32_t)(S * g.kb_a);

@@ -8,12 +8,20 @@
 
 namespace fz {
 
+// A and B indices are below FUSION_MAX_TOKENS / 2 <= 2^kKeyShift, so (B index, A index)
+// packs into one int that orders by B token first.
+constexpr int kKeyShift = 10;
+static_assert(FUSION_MAX_TOKENS / 2 <= (1 << kKeyShift), "token index does not fit the merge key");
+constexpr int kMergedCount = 36;   // tmp[] slot of the number of B tokens that receive sources
+constexpr int kGatherChunks = 2048;   // copy chunks in flight per CTA
+constexpr int kSrcU = 2;           // merge sources fetched ahead
+
 // ---------------------------------------------------------------------------
 // metadata in shared memory, after the kernel's staging area
 // ---------------------------------------------------------------------------
 struct Meta {
-    size_t best, rk, pk, inv_a, inv_b, match, sel, mflag, kflag, opos, srcpos, scnt, slist, msize, mscore, invd,
-        tsize, tscore, tmp, total;
+    size_t best, rk, pk, inv_a, inv_b, match, sel, mkey, mflag, kflag, opos, srcpos, scnt, slist, mlist, msize,
+        mscore, invd, tsize, tscore, tmp, total;
 };
 
 __host__ __device__ inline Meta meta_layout(int nmax, size_t base) {
@@ -28,12 +36,14 @@ __host__ __device__ inline Meta meta_layout(int nmax, size_t base) {
     L.inv_b = off;  off += sizeof(float) * nB;
     L.match = off;  off += sizeof(int) * nA;
     L.sel = off;    off += sizeof(int) * nA;
+    L.mkey = off;   off += sizeof(int) * nA;
     L.mflag = off;  off += sizeof(int) * nmax;
     L.kflag = off;  off += sizeof(int) * nmax;
     L.opos = off;   off += sizeof(int) * (nmax + 1);
     L.srcpos = off; off += sizeof(int) * nmax;
     L.scnt = off;   off += sizeof(int) * (nB + 1);
     L.slist = off;  off += sizeof(int) * nA;
+    L.mlist = off;  off += sizeof(int) * nB;
     L.msize = off;  off += sizeof(float) * nmax;
     L.mscore = off; off += sizeof(float) * nmax;
     off = (off + 7) / 8 * 8;
@@ -48,7 +58,7 @@ __host__ __device__ inline Meta meta_layout(int nmax, size_t base) {
 struct MetaPtrs {
     unsigned long long *best, *rk, *pk;
     float *inv_a, *inv_b;
-    int *match, *sel, *mflag, *kflag, *opos, *srcpos, *scnt, *slist;
+    int *match, *sel, *mkey, *mflag, *kflag, *opos, *srcpos, *scnt, *slist, *mlist;
     float *msize, *mscore;
     float2 *invd;
     float *tsize, *tscore;
@@ -61,12 +71,14 @@ struct MetaPtrs {
           inv_b(reinterpret_cast<float *>(sm + L.inv_b)),
           match(reinterpret_cast<int *>(sm + L.match)),
           sel(reinterpret_cast<int *>(sm + L.sel)),
+          mkey(reinterpret_cast<int *>(sm + L.mkey)),
           mflag(reinterpret_cast<int *>(sm + L.mflag)),
           kflag(reinterpret_cast<int *>(sm + L.kflag)),
           opos(reinterpret_cast<int *>(sm + L.opos)),
           srcpos(reinterpret_cast<int *>(sm + L.srcpos)),
           scnt(reinterpret_cast<int *>(sm + L.scnt)),
           slist(reinterpret_cast<int *>(sm + L.slist)),
+          mlist(reinterpret_cast<int *>(sm + L.mlist)),
           msize(reinterpret_cast<float *>(sm + L.msize)),
           mscore(reinterpret_cast<float *>(sm + L.mscore)),
           invd(reinterpret_cast<float2 *>(sm + L.invd)),
@@ -82,17 +94,21 @@ struct SampleInfo {
 
 // The input sample this CTA handles; false when there is nothing to do (beyond the
 // device batch count, an invalid call, or a sample that exited).
+// The grid has one CTA per possible sample (i < max_batch), so every load of the first
+// group is in bounds whatever the device batch count says; they issue together, and the
+// second group (which needs the output slot and the original id) follows.
 __device__ __forceinline__ bool sample_info(const ImageParams &p, int i, SampleInfo &s) {
-    const int B = device_batch(p.in);
-    if (B < 0 || i >= B) return false;
-    if (p.plan[0] == 0) return false;
+    const int bval = p.in.batch ? *p.in.batch : p.in.max_batch;
+    const int valid = p.plan[0];
     const int j = p.slot[i];
-    if (j < 0) return false;
-    s.start = p.in.offsets[i];
-    s.N = p.in.offsets[i + 1] - s.start;
+    const int o0 = p.in.offsets[i], o1 = p.in.offsets[i + 1];
+    const int id = p.in.ids ? p.in.ids[i] : i;
+    if (bval < 0 || bval > p.in.max_batch || i >= bval || valid == 0 || j < 0) return false;
+    s.start = o0;
+    s.N = o1 - o0;
     s.out_start = p.offsets_out[j];
     s.out_n = p.offsets_out[j + 1] - s.out_start;
-    s.id = p.in.ids ? p.in.ids[i] : i;
+    s.id = id;
     s.P = s.N - 1;
     s.nA = s.P / 2;
     s.nB = (s.P + 1) / 2;
@@ -110,6 +126,7 @@ __device__ __forceinline__ void meta_init(const ImageParams &p, const SampleInfo
         m.match[a] = 0;
     }
     for (int n = tid; n <= s.nB; n += NT) m.scnt[n] = 0;
+    if (tid == 0) m.tmp[kMergedCount] = 0;
     for (int pos = tid; pos < s.N; pos += NT) {
         m.tsize[pos] = p.sizes[s.start + pos];
         m.tscore[pos] = p.scores ? p.scores[s.start + pos] : 0.0f;
@@ -118,7 +135,8 @@ __device__ __forceinline__ void meta_init(const ImageParams &p, const SampleInfo
 
 // best[a] holds the packed (similarity, lowest B index) maximum of every A row.  Writes
 // match[a] and, when tokens merge, sel[a] for the r_eff A tokens of largest similarity
-// (lowest position on ties).  Ends with a barrier.
+// (lowest position on ties) and mkey[rank] = (match[a] << kKeyShift) | a for each of them.
+// Ends with a barrier.
 template <int NT>
 __device__ __forceinline__ void select_top_r(const SampleInfo &s, MetaPtrs &m) {
     const int tid = threadIdx.x;
@@ -133,6 +151,7 @@ __device__ __forceinline__ void select_top_r(const SampleInfo &s, MetaPtrs &m) {
 #pragma unroll 8
             for (int q = 0; q < s.nA; ++q) rank += m.rk[q] > ka ? 1 : 0;
             m.sel[a] = rank < s.r_eff ? 1 : 0;
+            if (rank < s.r_eff) m.mkey[rank] = (m.match[a] << kKeyShift) | a;
         }
     }
     __syncthreads();
@@ -144,13 +163,6 @@ __device__ __forceinline__ void select_top_r(const SampleInfo &s, MetaPtrs &m) {
 __device__ __forceinline__ uint4 pack_chunk(const F2 (&q)[4]) {
     return make_uint4(__float_as_uint(q[0].hi), __float_as_uint(q[1].hi), __float_as_uint(q[2].hi),
                       __float_as_uint(q[3].hi));
-}
-__device__ __forceinline__ uint4 pack_chunk(const F2 (&q)[8]) {
-    uint32_t w[4];
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-        w[k] = (uint32_t)f2_to_bf16_bits(q[2 * k]) | ((uint32_t)f2_to_bf16_bits(q[2 * k + 1]) << 16);
-    return make_uint4(w[0], w[1], w[2], w[3]);
 }
 
 // num / den for the merged mean, as a float-float value whose rounding to the
@@ -176,10 +188,28 @@ __device__ __forceinline__ F2 mean_of(F2 num, F2 den, F2 inv, __nv_bfloat16) {
 }
 __device__ __forceinline__ F2 mean_of(F2 num, F2 den, F2, float) { return f2_div(num, den); }
 
+// bf16 bits of num / den rounded to nearest even.  q1 = num.hi * inv.hi carries three
+// relative errors of at most 2^-24 each (num.lo dropped, inv.lo dropped, the product's
+// rounding), so it lies within 4 float32 ulps of the exact quotient: when it is more than
+// 8 ulps from every bf16 rounding midpoint it rounds like the exact quotient; otherwise
+// the float-float path above decides.
+__device__ __forceinline__ uint16_t mean_bits(F2 num, F2 den, F2 inv, __nv_bfloat16) {
+    const uint32_t u = __float_as_uint(__fmul_rn(num.hi, inv.hi));
+    const uint32_t low = u & 0xFFFFu;
+    const uint32_t dist = low > 0x8000u ? low - 0x8000u : 0x8000u - low;
+    if (dist > 8u && (u & 0x7F800000u) != 0x7F800000u) return (uint16_t)((u + 0x8000u) >> 16);
+    return f2_to_bf16_bits(mean_of(num, den, inv, __nv_bfloat16{}));
+}
+
 // Accumulator of exact products: hi parts summed with two_sum, the rounding errors and
 // product remainders summed plainly (about 44 correct bits for a few terms).
 struct Acc2 {
     float hi = 0.0f, lo = 0.0f;
+    __device__ __forceinline__ void first_prod(float a, float b) {   // add_prod from zero
+        const F2 pr = two_prod(a, b);
+        hi = pr.hi;
+        lo = pr.lo;
+    }
     __device__ __forceinline__ void add_prod(float a, float b) {
         const F2 pr = two_prod(a, b);
         const F2 sm = two_sum(hi, pr.hi);
@@ -188,6 +218,21 @@ struct Acc2 {
     }
     __device__ __forceinline__ F2 value() const { return quick_two_sum(hi, lo); }
 };
+
+__device__ __forceinline__ uint4 merged_pack(const Acc2 (&num)[8], F2 den, F2 inv, __nv_bfloat16) {
+    uint32_t w[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+        w[k] = (uint32_t)mean_bits(num[2 * k].value(), den, inv, __nv_bfloat16{}) |
+               ((uint32_t)mean_bits(num[2 * k + 1].value(), den, inv, __nv_bfloat16{}) << 16);
+    return make_uint4(w[0], w[1], w[2], w[3]);
+}
+__device__ __forceinline__ uint4 merged_pack(const Acc2 (&num)[4], F2 den, F2 inv, float) {
+    F2 q[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) q[e] = mean_of(num[e].value(), den, inv, 0.0f);
+    return pack_chunk(q);
+}
 
 // Loads the 16-byte chunk c of the input token at `pos` straight from global memory.
 template <typename T>
@@ -203,36 +248,102 @@ struct GlobalLoader {
 // ---------------------------------------------------------------------------
 // merged token set -> merged sizes / scores -> prune -> outputs
 // ---------------------------------------------------------------------------
-// Requires sel / match / scnt / tsize / tscore ready (after a barrier).  `load(pos, c)`
+// One chunk of a merged output row (Sec. III-C): chunk c of B token `pos` and of its
+// first kSrcU sources, fetched ahead of the arithmetic so the loads overlap other work.
+struct MergedItem {
+    int pos, c, q0, q1;   // pos < 0: nothing to do
+    uint4 self, av[kSrcU];
+};
+
+template <typename Loader>
+__device__ __forceinline__ void merged_fetch(const MetaPtrs &m, int t, int n_items, int ncx, const Loader &load,
+                                             MergedItem &it) {
+    it.pos = -1;
+    if (t >= n_items) return;
+    const int k = t / ncx;
+    const int pos = 1 + 2 * m.mlist[k];
+    if (!m.kflag[pos]) return;   // pruned after merging
+    it.pos = pos;
+    it.c = t - k * ncx;
+    const int n = (pos - 1) >> 1;
+    it.q0 = m.scnt[n];
+    it.q1 = m.scnt[n + 1];
+    it.self = load(pos, it.c);
+#pragma unroll
+    for (int u = 0; u < kSrcU; ++u)
+        if (it.q0 + u < it.q1) it.av[u] = load(2 + 2 * m.slist[it.q0 + u], it.c);
+}
+
+// The size-weighted mean of a fetched item: the B token first, then its sources in
+// ascending A order, products summed exactly enough that the result rounds once.
+template <typename T, typename Loader>
+__device__ __forceinline__ uint4 merged_compute(const MetaPtrs &m, const MergedItem &it, const Loader &load) {
+    constexpr int CH = Elem<T>::kPerChunk;
+    float f[CH];
+    chunk_to_f(it.self, f);
+    const float sb = m.tsize[it.pos];
+    Acc2 num[CH];
+#pragma unroll
+    for (int e = 0; e < CH; ++e) num[e].first_prod(sb, f[e]);
+    F2 den = {sb, 0.0f};
+#pragma unroll
+    for (int u = 0; u < kSrcU; ++u) {
+        if (it.q0 + u >= it.q1) break;
+        const float sa = m.tsize[2 + 2 * m.slist[it.q0 + u]];
+        den = f2_add_f(den, sa);
+        chunk_to_f(it.av[u], f);
+#pragma unroll
+        for (int e = 0; e < CH; ++e) num[e].add_prod(sa, f[e]);
+    }
+    for (int q = it.q0 + kSrcU; q < it.q1; ++q) {
+        const int ap = 2 + 2 * m.slist[q];
+        const float sa = m.tsize[ap];
+        den = f2_add_f(den, sa);
+        chunk_to_f(load(ap, it.c), f);
+#pragma unroll
+        for (int e = 0; e < CH; ++e) num[e].add_prod(sa, f[e]);
+    }
+    const float2 iv = m.invd[it.pos];
+    return merged_pack(num, den, {iv.x, iv.y}, T{});
+}
+
+// Requires sel / match / mkey / tsize / tscore ready (after a barrier).  `load(pos, c)`
 // returns the 16-byte chunk c of input token pos.  Returns false (after raising
 // FUSION_DEV_INTERNAL) if the token count disagrees with the plan; uniform per CTA.
 template <typename T, int NT, typename Loader>
 __device__ bool finish_sample(const ImageParams &p, const SampleInfo &s, MetaPtrs &m, const Loader &load) {
     constexpr int CH = Elem<T>::kPerChunk;
     const int tid = threadIdx.x;
-    const int N = s.N;
+    const int N = s.N, nB = s.nB, R = s.r_eff;
 
-    // merged token set: survivors keep ascending position
+    // merged token set: survivors keep ascending position (mflag 1; 0 = merged away).
+    // The selected A tokens, keyed (B index, A index), give every B token the slice
+    // scnt[n] .. scnt[n+1] of slist holding its sources in ascending A order.
     for (int pos = tid; pos < N; pos += NT)
         m.mflag[pos] = (pos >= 2 && !(pos & 1) && m.sel[(pos - 2) / 2]) ? 0 : 1;
-    if (s.r_eff > 0)
-        for (int a = tid; a < s.nA; a += NT)
-            if (m.sel[a]) atomicAdd(&m.scnt[m.match[a]], 1);
-    __syncthreads();
-    block_scan_excl(m.scnt, s.nB + 1, m.tmp);   // scnt[n] = first slot of B token n's sources
-    if (s.r_eff > 0) {
-        for (int a = tid; a < s.nA; a += NT) {
-            if (!m.sel[a]) continue;
-            const int n = m.match[a];
-            int before = 0;
-            for (int q = 0; q < a; ++q) before += (m.sel[q] && m.match[q] == n) ? 1 : 0;
-            m.slist[m.scnt[n] + before] = a;   // sources of every B token in ascending A order
+    if (R > 0) {
+        for (int t = tid; t < R; t += NT) {
+            const int key = m.mkey[t];
+            int slot = 0;
+            for (int u = 0; u < R; ++u) slot += m.mkey[u] < key ? 1 : 0;
+            m.slist[slot] = key & ((1 << kKeyShift) - 1);
         }
+        for (int n = tid; n < nB; n += NT) {
+            int lt = 0, eq = 0;
+            for (int u = 0; u < R; ++u) {
+                const int b = m.mkey[u] >> kKeyShift;
+                lt += b < n ? 1 : 0;
+                eq += b == n ? 1 : 0;
+            }
+            m.scnt[n] = lt;
+            if (eq > 0) m.mlist[atomicAdd(&m.tmp[kMergedCount], 1)] = n;
+        }
+        if (tid == 0) m.scnt[nB] = R;
     }
     __syncthreads();
 
     // merged sizes and scores: float-float sums over the sources (exact for a few terms),
-    // rounded once; merged B tokens also keep 1 / (sum of sizes) for the weighted mean
+    // rounded once; merged B tokens (mflag 2) also keep 1 / (sum of sizes) for the mean
     for (int pos = tid; pos < N; pos += NT) {
         if (!m.mflag[pos]) continue;
         F2 sz = {m.tsize[pos], 0.0f};
@@ -252,6 +363,7 @@ __device__ bool finish_sample(const ImageParams &p, const SampleInfo &s, MetaPtr
         if (merged) {
             const F2 inv = f2_div({1.0f, 0.0f}, sz);
             m.invd[pos] = make_float2(inv.hi, inv.lo);
+            m.mflag[pos] = 2;
         }
         if (p.scores && !isfinite(m.mscore[pos]) && pos > 0) raise_status(p.status, FUSION_DEV_NONFINITE);
     }
@@ -260,7 +372,7 @@ __device__ bool finish_sample(const ImageParams &p, const SampleInfo &s, MetaPtr
     // prune: CLS + the k highest merged scores, lowest position on ties
     if (p.do_prune) {
         bool nf = false;
-        const int k = keep_count(p.rho[s.id], N - s.r_eff - 1, nf);
+        const int k = keep_count(p.rho[s.id], N - R - 1, nf);
         // key 0 marks a non-candidate (CLS or merged away); every candidate key is > 0
         for (int pos = tid; pos < N; pos += NT)
             m.pk[pos] = (pos > 0 && m.mflag[pos]) ? rank_key(m.mscore[pos], pos) : 0ull;
@@ -281,8 +393,9 @@ __device__ bool finish_sample(const ImageParams &p, const SampleInfo &s, MetaPtr
         }
     } else {
         for (int pos = tid; pos < N; pos += NT) {
-            m.kflag[pos] = m.mflag[pos];
-            m.opos[pos] = m.mflag[pos];
+            const int keep = m.mflag[pos] ? 1 : 0;
+            m.kflag[pos] = keep;
+            m.opos[pos] = keep;
         }
     }
     __syncthreads();
@@ -291,14 +404,16 @@ __device__ bool finish_sample(const ImageParams &p, const SampleInfo &s, MetaPtr
         if (tid == 0) raise_status(p.status, FUSION_DEV_INTERNAL);
         return false;
     }
+    // source of every output row; merged rows are stored complemented (negative)
     for (int pos = tid; pos < N; pos += NT)
-        if (m.kflag[pos]) m.srcpos[m.opos[pos]] = pos;
+        if (m.kflag[pos]) m.srcpos[m.opos[pos]] = m.mflag[pos] == 2 ? ~pos : pos;
     __syncthreads();
 
     // index outputs
     const int start = s.start, out_start = s.out_start, out_n = s.out_n;
     for (int o = tid; o < out_n; o += NT) {
-        const int pos = m.srcpos[o];
+        const int sp = m.srcpos[o];
+        const int pos = sp < 0 ? ~sp : sp;
         const long long orow = (long long)out_start + o;
         p.sizes_out[orow] = m.msize[pos];
         if (p.scores_out) p.scores_out[orow] = m.mscore[pos];
@@ -314,49 +429,46 @@ __device__ bool finish_sample(const ImageParams &p, const SampleInfo &s, MetaPtr
             p.dst_map[start + pos] = out_start + m.opos[dest];
         }
 
-    // token rows: copies and size-weighted means, 16 bytes per thread.  (o, c) walks the
-    // output rows chunk by chunk without a division per step.
-    const int ncx = p.dim / CH;
+    // copied token rows, 16 bytes per thread and kGatherU chunks in flight; (o, c) walks
+    // the output rows chunk by chunk without a division per step
+    constexpr int kGatherU = kGatherChunks / NT;
+    const int dim = p.dim, ncx = dim / CH;
     const int ostep = NT / ncx, cstep = NT - ostep * ncx;
-    T *xo = reinterpret_cast<T *>(p.x_out);
+    T *xo = reinterpret_cast<T *>(p.x_out) + (long long)out_start * dim;
+    const int n_items = m.tmp[kMergedCount] * ncx;   // merged chunks
+    MergedItem cur;
+    merged_fetch(m, tid, n_items, ncx, load, cur);   // lands while the copies run
     int o = tid / ncx, c = tid - (tid / ncx) * ncx;
-    for (; o < out_n;) {
-        const int pos = m.srcpos[o];
-        const uint4 self = load(pos, c);
-        uint4 outv = self;
-        if (pos & 1) {
-            const int n = (pos - 1) / 2;
-            const int q0 = m.scnt[n], q1 = m.scnt[n + 1];
-            if (q1 > q0) {
-                float f[CH];
-                chunk_to_f(self, f);
-                const float sb = m.tsize[pos];
-                Acc2 num[CH];
+    while (o < out_n) {
+        int src[kGatherU], cc[kGatherU], dst[kGatherU];
 #pragma unroll
-                for (int e = 0; e < CH; ++e) num[e].add_prod(sb, f[e]);
-                F2 den = {sb, 0.0f};
-                for (int q = q0; q < q1; ++q) {
-                    const int apos = 2 + 2 * m.slist[q];
-                    const float sa = m.tsize[apos];
-                    den = f2_add_f(den, sa);
-                    chunk_to_f(load(apos, c), f);
-#pragma unroll
-                    for (int e = 0; e < CH; ++e) num[e].add_prod(sa, f[e]);
-                }
-                const float2 iv = m.invd[pos];
-                F2 qv[CH];
-#pragma unroll
-                for (int e = 0; e < CH; ++e) qv[e] = mean_of(num[e].value(), den, {iv.x, iv.y}, T{});
-                outv = pack_chunk(qv);
+        for (int u = 0; u < kGatherU; ++u) {
+            src[u] = o < out_n ? m.srcpos[o] : -1;   // < 0: merged row or past the end
+            cc[u] = c;
+            dst[u] = o * dim + c * CH;
+            o += ostep;
+            c += cstep;
+            if (c >= ncx) {
+                c -= ncx;
+                ++o;
             }
         }
-        *reinterpret_cast<uint4 *>(xo + ((long long)out_start + o) * p.dim + c * CH) = outv;
-        o += ostep;
-        c += cstep;
-        if (c >= ncx) {
-            c -= ncx;
-            ++o;
-        }
+        uint4 v[kGatherU];
+#pragma unroll
+        for (int u = 0; u < kGatherU; ++u)
+            if (src[u] >= 0) v[u] = load(src[u], cc[u]);
+#pragma unroll
+        for (int u = 0; u < kGatherU; ++u)
+            if (src[u] >= 0) *reinterpret_cast<uint4 *>(xo + dst[u]) = v[u];
+    }
+
+    // merged token rows: the size-weighted means, the next item's loads in flight
+    for (int t = tid; t < n_items; t += NT) {
+        MergedItem nxt;
+        merged_fetch(m, t + NT, n_items, ncx, load, nxt);
+        if (cur.pos >= 0)
+            *reinterpret_cast<uint4 *>(xo + m.opos[cur.pos] * dim + cur.c * CH) = merged_compute<T>(m, cur, load);
+        cur = nxt;
     }
     return true;
 }

@@ -129,6 +129,9 @@ ImageParams image_params(const fusion_ragged &in, const void *x, int32_t dim, co
 // CTA's decisions and gather overlap the other's loads.
 constexpr int kTcSmemBudgetKb = 111;
 
+// The plan runs inside the per-sample kernel when every CTA can afford to scan the batch.
+bool fuse_plan(const fusion_ragged &in) { return in.max_batch >= 1 && in.max_batch <= kFusedPlanMaxBatch; }
+
 // The per-sample kernel: TMA + tcgen05 when the shape allows it, else the general one.
 cudaError_t launch_sample_kernel(int dtype, const ImageParams &p, const ImageGeometry &G, cudaStream_t s) {
     if (p.do_merge) {
@@ -202,11 +205,12 @@ int fusion_merge(int dtype, fusion_ragged in, const void *x, int32_t dim, const 
     pa.plan = w.plan;
     pa.status = dev_status;
     record(ev.start, s);
-    FZ_TRY(cuda_rc(launch_plan(pa, s)));
+    if (!fuse_plan(in)) FZ_TRY(cuda_rc(launch_plan(pa, s)));
     record(ev.mid, s);
-    const ImageParams p = image_params(in, x, dim, keys, key_dim, sizes, scores, r, nullptr, 1, 0, w,
-                                       offsets_out, x_out, sizes_out, scores_out, keep_idx, dst_map,
-                                       a_match, dev_status, G);
+    ImageParams p = image_params(in, x, dim, keys, key_dim, sizes, scores, r, nullptr, 1, 0, w, offsets_out,
+                                 x_out, sizes_out, scores_out, keep_idx, dst_map, a_match, dev_status, G);
+    p.fused_plan = fuse_plan(in);
+    p.plan_args = pa;
     const int rc = cuda_rc(launch_sample_kernel(dtype, p, G, s));
     record(ev.end, s);
     return rc;
@@ -269,11 +273,12 @@ int fusion_prune(int dtype, fusion_ragged in, const void *x, int32_t dim, const 
     pa.status = dev_status;
     const ProfileEvents ev = take_profile();
     record(ev.start, s);
-    FZ_TRY(cuda_rc(launch_plan(pa, s)));
+    if (!fuse_plan(in)) FZ_TRY(cuda_rc(launch_plan(pa, s)));
     record(ev.mid, s);
-    const ImageParams p = image_params(in, x, dim, nullptr, dim, sizes, scores, nullptr, rho, 0, 1, w,
-                                       offsets_out, x_out, sizes_out, scores_out, keep_idx, nullptr,
-                                       nullptr, dev_status, G);
+    ImageParams p = image_params(in, x, dim, nullptr, dim, sizes, scores, nullptr, rho, 0, 1, w, offsets_out,
+                                 x_out, sizes_out, scores_out, keep_idx, nullptr, nullptr, dev_status, G);
+    p.fused_plan = fuse_plan(in);
+    p.plan_args = pa;
     const int rc = cuda_rc(launch_sample_kernel(dtype, p, G, s));
     record(ev.end, s);
     return rc;
@@ -307,11 +312,12 @@ int fusion_compact(int dtype, fusion_ragged in, const void *x, int32_t dim, cons
     pa.status = dev_status;
     const ProfileEvents ev = take_profile();
     record(ev.start, s);
-    FZ_TRY(cuda_rc(launch_plan(pa, s)));
+    if (!fuse_plan(in)) FZ_TRY(cuda_rc(launch_plan(pa, s)));
     record(ev.mid, s);
-    const ImageParams p = image_params(in, x, dim, nullptr, dim, sizes, scores, nullptr, nullptr, 0, 0, w,
-                                       offsets_out, x_out, sizes_out, scores_out, keep_idx, nullptr,
-                                       nullptr, dev_status, G);
+    ImageParams p = image_params(in, x, dim, nullptr, dim, sizes, scores, nullptr, nullptr, 0, 0, w, offsets_out,
+                                 x_out, sizes_out, scores_out, keep_idx, nullptr, nullptr, dev_status, G);
+    p.fused_plan = fuse_plan(in);
+    p.plan_args = pa;
     const int rc = cuda_rc(launch_sample_kernel(dtype, p, G, s));
     record(ev.end, s);
     return rc;
@@ -381,17 +387,19 @@ int fusion_stage(int dtype, int flags, fusion_ragged in, const void *x, int32_t 
         e.partials = w.partials;
         e.n_ctile = ceil_div(head.classes, kExitCT);
         e.n_btile = ceil_div(in.max_batch > 0 ? in.max_batch : 1, kExitBT);
-        e.do_plan = 1;
+        e.do_plan = !fuse_plan(in);
         e.plan = pa;
         e.status = dev_status;
         FZ_TRY(cuda_rc(launch_exit(dtype, e, s)));
-    } else {
+    } else if (!fuse_plan(in)) {
         FZ_TRY(cuda_rc(launch_plan(pa, s)));
     }
     record(ev.mid, s);
-    const ImageParams p = image_params(in, x, dim, do_merge ? keys : nullptr, key_dim, sizes, scores, r,
-                                       rho, do_merge, do_prune, w, offsets_out, x_out, sizes_out,
-                                       scores_out, keep_idx, nullptr, a_match, dev_status, G);
+    ImageParams p = image_params(in, x, dim, do_merge ? keys : nullptr, key_dim, sizes, scores, r, rho, do_merge,
+                                 do_prune, w, offsets_out, x_out, sizes_out, scores_out, keep_idx, nullptr, a_match,
+                                 dev_status, G);
+    p.fused_plan = fuse_plan(in);
+    p.plan_args = pa;
     const int rc = cuda_rc(launch_sample_kernel(dtype, p, G, s));
     record(ev.end, s);
     return rc;

@@ -268,7 +268,7 @@ __global__ void __launch_bounds__(kImageThreads, 1) k_image(ImageParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
     constexpr int CH = Elem<T>::kPerChunk;
     SampleInfo s;
-    if (!sample_info(p, blockIdx.x, s)) return;
+    if (!sample_begin<kImageThreads>(p, blockIdx.x, s)) return;
     const int tid = threadIdx.x;
     const int stage_chunks = p.resident ? p.kdim / CH : p.kc / CH;
     const size_t stage_b = p.do_merge ? stage_a_bytes(stage_chunks, p.ra) : 0;

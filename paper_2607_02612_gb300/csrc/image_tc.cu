@@ -22,6 +22,8 @@
 // FUSION_DEV_TIMEOUT, skips its outputs and frees its tensor memory.
 #include <cuda.h>
 
+#include <algorithm>
+
 #include "sample.cuh"
 
 namespace fz {
@@ -88,6 +90,22 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// ss + sc += part, Neumaier-compensated.
+__device__ __forceinline__ void neumaier_add(float &ss, float &sc, float part) {
+    const float t = __fadd_rn(ss, part);
+    sc = __fadd_rn(sc, fabsf(ss) >= fabsf(part) ? __fadd_rn(__fsub_rn(ss, t), part) : __fadd_rn(__fsub_rn(part, t), ss));
+    ss = t;
+}
+// Sum of squares of the 8 bf16 values of a 16-byte chunk.
+__device__ __forceinline__ float chunk_sq(uint4 v) {
+    float f[8];
+    chunk_to_f(v, f);
+    float part = 0.0f;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) part = fmaf(f[e], f[e], part);
+    return part;
+}
+
 // Chunk c of input token pos from the resident swizzled stages (CLS from global).
 struct SwizzledLoader {
     const unsigned char *regA, *regB;
@@ -111,59 +129,85 @@ __global__ void __launch_bounds__(kTcThreads, 2)
     __shared__ int s_fail;
     __shared__ unsigned long long half_best[kTcThreads / 2];
 
-    SampleInfo s;
-    if (!sample_info(p, blockIdx.x, s)) return;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const bool dec = s.decide;
-    const int S = g.stages, nkb = g.n_kb;
-    unsigned char *regA = sm + g.stage_a;   // stage st, half A: regA + st * kbA
-    unsigned char *regB = sm + g.stage_b;
-    const int rowsA = (s.nA + 7) & ~7, rowsB = (s.nB + 7) & ~7;
-    const uint32_t kb_tx = (uint32_t)(rowsA + rowsB) * 128u;
-    const int yA = (s.start + 2) >> 1, yB = (s.start + 1) >> 1;
-    const bool oddA = (s.start + 2) & 1, oddB = (s.start + 1) & 1;
-    // K-block kb of both halves into stage kb % S
-    auto produce = [&](int kb) {
-        const int st = kb % S;
-        const uint32_t bar = smem_addr(&bar_full[st]);
-        mbar_expect_tx(bar, kb_tx);
-        const uint32_t dA = smem_addr(regA + (size_t)st * g.kb_a), dB = smem_addr(regB + (size_t)st * g.kb_b);
-        for (int half = 0; half < 2; ++half) {
-            const int n = half ? s.nB : s.nA;
-            const bool odd = half ? oddB : oddA;
-            const int y0 = half ? yB : yA;
-            const uint32_t d0 = half ? dB : dA;
-            int done = 0;
-            for (; n - done >= 32; done += 32)
-                tma_load_2d(d0 + done * 128, odd ? &maps.o32 : &maps.e32, kb * 64, y0 + done, bar);
-            for (; done < n; done += 8)
-                tma_load_2d(d0 + done * 128, odd ? &maps.o8 : &maps.e8, kb * 64, y0 + done, bar);
-        }
-    };
-
-    // the first stages' loads go out before anything else
-    if (tid == 0) {
-        s_fail = 0;
-        if (dec) {
-            for (int st = 0; st < S; ++st) {
-                mbar_init(smem_addr(&bar_full[st]), 1);
-                mbar_init(smem_addr(&bar_empty[st]), 1 + kTcThreads / 32);
-            }
-            mbar_init(smem_addr(&bar_done), 1);
-            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            for (int kb = 0; kb < S && kb < nkb; ++kb) produce(kb);
-        }
-    }
-    MetaPtrs m(sm, meta_layout(p.in.max_tokens, g.meta_base));
-    meta_init<kTcThreads>(p, s, m);
-    __syncwarp();
-    if (dec && warp == 0) {
+    // Tensor memory first: an SM admits another CTA of a kernel that allocates tensor
+    // memory only once the resident one has given up its allocation permit.
+    if (warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(&tmem_base)),
                      "r"(g.tmem_cols)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
+    // the tensor maps' descriptors travel while the sample's metadata loads
+    if (tid >= 32 && tid < 36) {
+        const CUtensorMap *mp = tid == 32 ? &maps.e32 : tid == 33 ? &maps.o32 : tid == 34 ? &maps.e8 : &maps.o8;
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(mp)) : "memory");
+    }
+    SampleInfo s;
+    if (!sample_begin<kTcThreads>(p, blockIdx.x, s)) {   // uniform over the CTA
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncthreads();
+        if (warp == 0)
+            asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(g.tmem_cols)
+                         : "memory");
+        return;
+    }
+    const bool dec = s.decide;
+    const int nkb = g.n_kb;
+    const int rowsA = (s.nA + 7) & ~7, rowsB = (s.nB + 7) & ~7;
+    const int npad = (s.nB + 15) & ~15;   // MMA N: |B| rounded up to 16
+    // The ring is sized for this sample: stage st holds K-block kb (st = kb % S) of half A
+    // at st * kbs and of half B right after it.  An MMA reads 128 A rows and npad B rows
+    // from a stage, past its end when the sample is small, which stays inside the buffer.
+    const uint32_t kbs = (uint32_t)(rowsA + rowsB) * 128u;
+    const uint32_t reach = (uint32_t)max(16384, (rowsA + npad) * 128);
+    int S = min(min(nkb, kMaxStages), (int)(g.stage_region / kbs));
+    while (S > 1 && (uint32_t)(S - 1) * kbs + reach > g.usable) --S;
+    unsigned char *regA = sm;                       // stage st, half A: regA + st * kbs
+    unsigned char *regB = sm + (size_t)rowsA * 128;  // stage st, half B: regB + st * kbs
+    const uint32_t kb_tx = kbs;
+    const int yA = (s.start + 2) >> 1, yB = (s.start + 1) >> 1;
+    const bool oddA = (s.start + 2) & 1, oddB = (s.start + 1) & 1;
+    // The boxes of one K-block: half A then half B, each in 32-row boxes while 32 rows
+    // remain, then 8-row boxes.
+    const int nbA = (s.nA >> 5) + (((s.nA & 31) + 7) >> 3);
+    const int per_kb = nbA + (s.nB >> 5) + (((s.nB & 31) + 7) >> 3);
+    auto issue_box = [&](int kb, int b) {
+        const int st = kb % S;
+        const int half = b >= nbA ? 1 : 0;
+        const int q = half ? b - nbA : b;
+        const int n32 = (half ? s.nB : s.nA) >> 5;
+        const bool big = q < n32;
+        const int row0 = big ? q * 32 : n32 * 32 + (q - n32) * 8;
+        const bool odd = half ? oddB : oddA;
+        const CUtensorMap *map = big ? (odd ? &maps.o32 : &maps.e32) : (odd ? &maps.o8 : &maps.e8);
+        const uint32_t dst = smem_addr((half ? regB : regA) + (size_t)st * kbs + (size_t)row0 * 128);
+        tma_load_2d(dst, map, kb * 64, (half ? yB : yA) + row0, smem_addr(&bar_full[st]));
+    };
+    auto produce = [&](int kb) {   // a whole K-block from one thread
+        mbar_expect_tx(smem_addr(&bar_full[kb % S]), kb_tx);
+        for (int b = 0; b < per_kb; ++b) issue_box(kb, b);
+    };
+
+    // the first stages' loads go out before anything else, spread over warp 0
+    if (warp == 0) {
+        if (lane == 0) s_fail = 0;
+        if (dec) {
+            if (lane < S) {
+                mbar_init(smem_addr(&bar_full[lane]), 1);
+                mbar_init(smem_addr(&bar_empty[lane]), 1 + kTcThreads / 32);
+            }
+            if (lane == 31) mbar_init(smem_addr(&bar_done), 1);
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            __syncwarp();
+            const int S0 = min(S, nkb);
+            if (lane < S0) mbar_expect_tx(smem_addr(&bar_full[lane]), kb_tx);
+            for (int t = lane; t < S0 * per_kb; t += 32) issue_box(t / per_kb, t % per_kb);
+        }
+    }
+    MetaPtrs m(sm, meta_layout(p.in.max_tokens, g.meta_base));
+    meta_init<kTcThreads>(p, s, m);
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
@@ -172,11 +216,13 @@ __global__ void __launch_bounds__(kTcThreads, 2)
         const uint32_t tmem = tmem_base;
 
         // instruction descriptor: f32 accumulator, bf16 A and B, K-major, N = |B| rounded to 16, M = 128
-        const int npad = (s.nB + 15) & ~15;
         const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(npad >> 3) << 17) | (8u << 24);
+        // Squared row norms: for a sample that stays resident, after all stages landed with
+        // kT threads per row; otherwise one thread per row, K-block by K-block as the ring turns.
+        const bool resident = S >= nkb;
         const bool isA = tid < 128;
         const int row = isA ? tid : tid - 128;
-        const bool has_row = row < (isA ? s.nA : s.nB);
+        const bool has_row = !resident && row < (isA ? s.nA : s.nB);
         float ss = 0.0f, sc = 0.0f;
         bool ok = true;
         for (int kb = 0; kb < nkb; ++kb) {
@@ -187,7 +233,7 @@ __global__ void __launch_bounds__(kTcThreads, 2)
                 break;
             }
             if (tid == 32) {
-                const uint32_t a0 = smem_addr(regA + (size_t)st * g.kb_a), b0 = smem_addr(regB + (size_t)st * g.kb_b);
+                const uint32_t a0 = smem_addr(regA + (size_t)st * kbs), b0 = smem_addr(regB + (size_t)st * kbs);
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 #pragma unroll
                 for (int k = 0; k < 4; ++k)
@@ -196,19 +242,10 @@ __global__ void __launch_bounds__(kTcThreads, 2)
                 if (kb == nkb - 1) umma_commit(smem_addr(&bar_done));
             }
             if (has_row) {   // squared norm of this thread's row, chunk by chunk
-                const unsigned char *base = (isA ? regA + (size_t)st * g.kb_a : regB + (size_t)st * g.kb_b) + row * 128;
+                const unsigned char *base = (isA ? regA : regB) + (size_t)st * kbs + row * 128;
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    float f[8];
-                    chunk_to_f(*reinterpret_cast<const uint4 *>(base + ((j ^ (row & 7)) << 4)), f);
-                    float part = 0.0f;
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) part = fmaf(f[e], f[e], part);
-                    const float t = __fadd_rn(ss, part);   // Neumaier-compensated sum of the chunk sums
-                    sc = __fadd_rn(sc, fabsf(ss) >= fabsf(part) ? __fadd_rn(__fsub_rn(ss, t), part)
-                                                               : __fadd_rn(__fsub_rn(part, t), ss));
-                    ss = t;
-                }
+                for (int j = 0; j < 8; ++j)
+                    neumaier_add(ss, sc, chunk_sq(*reinterpret_cast<const uint4 *>(base + ((j ^ (row & 7)) << 4))));
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_addr(&bar_empty[st]));
@@ -221,14 +258,40 @@ __global__ void __launch_bounds__(kTcThreads, 2)
             }
         }
         if (!ok) atomicOr(&s_fail, 1);
-        if (has_row) {
+        int nrow = row;        // row of this thread: A rows, then B rows
+        bool owner = has_row;  // writes the row's inverse norm
+        if (resident) {   // uniform over the CTA: every lane reaches the shuffles
+            // kT threads per row (the largest power of two up to 8 that fits), each taking
+            // every kT-th chunk of the row; the partial sums meet by shuffles
+            const int R = s.nA + s.nB;
+            const int kT = R <= 32 ? 8 : R <= 64 ? 4 : R <= 128 ? 2 : 1;
+            const int r = tid / kT, part = tid % kT;
+            if (r < R) {
+                const bool rA = r < s.nA;
+                const int rr = rA ? r : r - s.nA;
+                const unsigned char *base = (rA ? regA : regB) + (size_t)rr * 128;
+                for (int c = part; c < nkb * 8; c += kT)
+                    neumaier_add(ss, sc, chunk_sq(*reinterpret_cast<const uint4 *>(
+                                             base + (size_t)(c >> 3) * kbs + (((c & 7) ^ (rr & 7)) << 4))));
+            }
+            for (int mk = 1; mk < kT; mk <<= 1) {   // kT divides 32: groups stay inside a warp
+                const float oss = __shfl_xor_sync(0xFFFFFFFFu, ss, mk), osc = __shfl_xor_sync(0xFFFFFFFFu, sc, mk);
+                neumaier_add(ss, sc, oss);
+                sc = __fadd_rn(sc, osc);
+            }
+            owner = r < R && part == 0;
+            nrow = r;
+        } else if (has_row) {
+            nrow = isA ? row : s.nA + row;
+        }
+        if (owner) {
             const float sq = __fadd_rn(ss, sc);
             if (!isfinite(sq)) raise_status(p.status, FUSION_DEV_NONFINITE);
             const float inv = 1.0f / fmaxf(sqrtf(sq), 1e-12f);
-            if (isA)
-                m.inv_a[row] = inv;
+            if (nrow < s.nA)
+                m.inv_a[nrow] = inv;
             else
-                m.inv_b[row] = inv;
+                m.inv_b[nrow - s.nA] = inv;
         }
         __syncthreads();
         bool mma_ok = s_fail == 0 && mbar_wait(smem_addr(&bar_done), 0);
@@ -272,20 +335,18 @@ __global__ void __launch_bounds__(kTcThreads, 2)
 
     if (s_fail == 0) {
         const GlobalLoader<__nv_bfloat16> gl{reinterpret_cast<const __nv_bfloat16 *>(p.x), (long long)s.start, p.dim};
-        if (dec && g.stages >= g.n_kb && p.keys_alias) {
-            const SwizzledLoader ld{regA, regB, g.kb_a, g.kb_b, gl};
+        if (dec && S >= nkb && p.keys_alias) {   // the whole sample is still in shared memory
+            const SwizzledLoader ld{regA, regB, kbs, kbs, gl};
             finish_sample<__nv_bfloat16, kTcThreads>(p, s, m, ld);
         } else {
             finish_sample<__nv_bfloat16, kTcThreads>(p, s, m, gl);
         }
     }
-    if (dec) {
-        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-        __syncthreads();
-        if (warp == 0)
-            asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(g.tmem_cols)
-                         : "memory");
-    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(g.tmem_cols)
+                     : "memory");
 }
 
 // ---------------------------------------------------------------------------
@@ -326,24 +387,24 @@ TcGeometry image_tc_geometry(int dtype, int max_tokens, int kdim, long long max_
     int cols = 32;
     while (cols < ((nBmax + 15) & ~15)) cols <<= 1;
     g.tmem_cols = cols;
-    const size_t meta = meta_layout(max_tokens, 0).total;
     const size_t per_stage = g.kb_a + g.kb_b;
-    // the padded MMA rows of the last stage read past the end: 2 KB of tail
+    // the largest read from a stage base: 128 A rows, or half A and npad B rows
+    const size_t npad_max = (size_t)((nBmax + 15) & ~15);
+    const size_t reach = std::max<size_t>(16384, g.kb_a + npad_max * 128);
     size_t budget = (size_t)stage_budget_kb * 1024;
     if (budget > 227 * 1024 - 4096) budget = 227 * 1024 - 4096;   // room for static shared memory
+    auto need = [&](int S) {   // usable bytes for S stages at max_tokens
+        const size_t meta_base = (size_t)S * per_stage + 2048;
+        return std::max(meta_layout(max_tokens, meta_base).total, (size_t)(S - 1) * per_stage + reach);
+    };
     int S = g.n_kb < kMaxStages ? g.n_kb : kMaxStages;
-    while (S > 2 && (size_t)S * per_stage + 2048 + meta + 1024 > budget) --S;
-    if ((size_t)S * per_stage + 2048 + meta + 1024 > budget) return g;
+    while (S > 2 && need(S) + 1024 > budget) --S;
+    if (need(S) + 1024 > budget) return g;
     g.stages = S;
-    g.stage_a = 0;
-    g.stage_b = (uint32_t)(S * g.kb_a);
+    g.stage_region = (uint32_t)(S * per_stage);
     g.meta_base = (uint32_t)(S * per_stage + 2048);
-    // an M = 128 MMA reads 16 row groups (16 KB) of half A from the last stage on
-    const size_t a_reach = (size_t)(S - 1) * g.kb_a + 16384;
-    size_t total = meta_layout(max_tokens, g.meta_base).total;
-    if (a_reach > total) total = a_reach;
-    g.smem = total + 1024;
-    if (g.smem > 227 * 1024) return TcGeometry{};
+    g.usable = (uint32_t)need(S);
+    g.smem = g.usable + 1024;
     g.ok = 1;
     return g;
 }
@@ -369,6 +430,9 @@ cudaError_t launch_image_tc(const ImageParams &p, const TcGeometry &g, cudaStrea
             return cudaErrorInvalidValue;
     }
     cudaError_t e = cudaFuncSetAttribute(k_image_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)g.smem);
+    if (e != cudaSuccess) return e;
+    // the largest shared-memory carveout, so that both CTAs of an SM are resident from the start
+    e = cudaFuncSetAttribute(k_image_tc, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     if (e != cudaSuccess) return e;
     k_image_tc<<<p.in.max_batch, kTcThreads, g.smem, s>>>(maps, p, g);
     return cudaGetLastError();

@@ -32,6 +32,10 @@ size_t exit_smem_bytes(int dtype, int dim);
 cudaError_t launch_plan(const PlanArgs &a, cudaStream_t s);
 
 // ---- per-sample merge / prune / gather -----------------------------------------
+// Batches of at most this many samples plan inside the per-sample kernel (every CTA
+// scans the batch), larger ones run the plan kernel first.
+constexpr int kFusedPlanMaxBatch = 1024;
+
 struct ImageParams {
     Ragged in;
     const void *x;
@@ -56,6 +60,10 @@ struct ImageParams {
     int *dst_map;
     int *a_match;
     int *status;
+    // fused_plan: no plan kernel ran; every CTA derives its sample's slot and output
+    // offset from plan_args (which also receives the plan's outputs)
+    int fused_plan;
+    PlanArgs plan_args;
     // staging geometry, fixed by the host from max_tokens and the key width
     int resident;        // every key dim staged at once
     int kc;              // key dims staged per chunk (multiple of 16)
@@ -76,12 +84,13 @@ cudaError_t launch_image(int dtype, const ImageParams &p, size_t smem, cudaStrea
 struct TcGeometry {
     int ok;
     int n_kb;          // key K-blocks of 64 dims
-    int stages;        // K-block stages in shared memory (all n_kb: the sample stays resident)
+    int stages;        // K-block stages of a sample of max_tokens tokens (more for smaller samples)
     int tmem_cols;     // tensor-memory columns allocated per CTA
-    uint32_t kb_a, kb_b;             // bytes of one K-block of half A / half B
-    uint32_t stage_a, stage_b;       // offsets of the two halves' stages
+    uint32_t kb_a, kb_b;             // bytes of one K-block of half A / half B at max_tokens
+    uint32_t stage_region;           // bytes of the K-block ring, from offset 0
     uint32_t meta_base;              // offset of the per-sample metadata
-    size_t smem;                     // dynamic shared memory bytes (with 1 KB alignment slack)
+    uint32_t usable;                 // bytes addressable after the 1 KB alignment
+    size_t smem;                     // dynamic shared memory bytes (usable + 1 KB alignment slack)
 };
 TcGeometry image_tc_geometry(int dtype, int max_tokens, int kdim, long long max_rows, int do_merge,
                              int stage_budget_kb);

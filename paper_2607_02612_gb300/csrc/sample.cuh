@@ -117,6 +117,125 @@ __device__ __forceinline__ bool sample_info(const ImageParams &p, int i, SampleI
     return true;
 }
 
+// The plan of one call computed inside the per-sample kernel, for batches of at most
+// kFusedPlanMaxBatch samples: every CTA runs through the whole batch (validation, which
+// samples continue, their output token counts) and keeps the exclusive prefix before its
+// own sample, so all CTAs agree on validity and no plan kernel runs first.  The loads of
+// the first group are in bounds for any j < max_batch, so they issue before the device
+// batch count is known.  CTA 0 writes the batch-level outputs and raises the status.
+// Must be called by every thread of the CTA.
+
+template <int NT>
+__device__ bool sample_plan(const ImageParams &p, int i, SampleInfo &s) {
+    const PlanArgs &a = p.plan_args;
+    constexpr int kW = NT / 32;
+    __shared__ int red[6][kW];
+    __shared__ int own[6];   // start, N, id, continues, count, merge count of sample i
+    const int t = threadIdx.x, lane = t & 31, w = t >> 5;
+    const int bval = a.in.batch ? *a.in.batch : a.in.max_batch;
+    int bad = 0, nf = 0, pre_s = 0, pre_r = 0, tot_s = 0, tot_r = 0;
+    for (int j0 = 0; j0 < a.in.max_batch; j0 += NT) {
+        const int j = j0 + t;
+        const bool inb = j < a.in.max_batch;
+        const int o0 = inb ? a.in.offsets[j] : 0, o1 = inb ? a.in.offsets[j + 1] : 0;
+        const int idr = inb ? (a.in.ids ? a.in.ids[j] : j) : 0;
+        const int ex = (inb && a.exit_mask) ? a.exit_mask[j] : 0;
+        if (!inb || j >= bval) continue;
+        const int N = o1 - o0;
+        const bool ok = o0 >= 0 && N >= 1 && N <= a.in.max_tokens && (long long)o1 <= a.in.max_rows;
+        const bool id_ok = idr >= 0 && idr < a.in.max_batch;
+        if (!ok) bad |= FUSION_DEV_BAD_OFFSETS;
+        if (!id_ok) bad |= FUSION_DEV_BAD_IDS;
+        const int surv = ex == 0 ? 1 : 0;
+        int cnt = 0, rm = 0;
+        if (ok && id_ok && surv) {
+            int n = N;
+            if (a.merge) {
+                rm = merge_count(a.r[idr], N - 1);
+                n -= rm;
+            }
+            if (a.prune) {
+                bool f = false;
+                n = 1 + keep_count(a.rho[idr], n - 1, f);
+                if (f) nf = 1;
+            }
+            cnt = n;
+        }
+        tot_s += surv;
+        tot_r += cnt;
+        if (j < i) {
+            pre_s += surv;
+            pre_r += cnt;
+        }
+        if (j == i) {
+            own[0] = o0;
+            own[1] = N;
+            own[2] = idr;
+            own[3] = surv;
+            own[4] = cnt;
+            own[5] = rm;
+        }
+    }
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) {
+        bad |= __shfl_xor_sync(0xFFFFFFFFu, bad, m);
+        nf |= __shfl_xor_sync(0xFFFFFFFFu, nf, m);
+        pre_s += __shfl_xor_sync(0xFFFFFFFFu, pre_s, m);
+        pre_r += __shfl_xor_sync(0xFFFFFFFFu, pre_r, m);
+        tot_s += __shfl_xor_sync(0xFFFFFFFFu, tot_s, m);
+        tot_r += __shfl_xor_sync(0xFFFFFFFFu, tot_r, m);
+    }
+    if (lane == 0) {
+        red[0][w] = bad;
+        red[1][w] = nf;
+        red[2][w] = pre_s;
+        red[3][w] = pre_r;
+        red[4][w] = tot_s;
+        red[5][w] = tot_r;
+    }
+    __syncthreads();
+    bad = nf = pre_s = pre_r = tot_s = tot_r = 0;
+#pragma unroll
+    for (int k = 0; k < kW; ++k) {
+        bad |= red[0][k];
+        nf |= red[1][k];
+        pre_s += red[2][k];
+        pre_r += red[3][k];
+        tot_s += red[4][k];
+        tot_r += red[5][k];
+    }
+    const bool batch_ok = bval >= 0 && bval <= a.in.max_batch;
+    if (!batch_ok) bad |= FUSION_DEV_BAD_BATCH;
+    if (i == 0 && t == 0) {
+        if (bad) raise_status(a.status, bad);
+        if (nf) raise_status(a.status, FUSION_DEV_NONFINITE);
+        a.offsets_out[bad ? 0 : tot_s] = bad ? 0 : tot_r;
+        if (a.batch_out) *a.batch_out = bad ? 0 : tot_s;
+    }
+    if (bad || i >= bval || !own[3]) return false;
+    if (t == 0) {
+        a.offsets_out[pre_s] = pre_r;
+        if (a.ids_out) a.ids_out[pre_s] = own[2];
+    }
+    s.start = own[0];
+    s.N = own[1];
+    s.out_start = pre_r;
+    s.out_n = own[4];
+    s.id = own[2];
+    s.P = s.N - 1;
+    s.nA = s.P / 2;
+    s.nB = (s.P + 1) / 2;
+    s.r_eff = p.do_merge ? own[5] : 0;   // the plan's merge flag is the call's
+    s.decide = p.do_merge && s.nA > 0 && (s.r_eff > 0 || p.need_match);
+    return true;
+}
+
+// Either the fused plan or the plan kernel's results.
+template <int NT>
+__device__ __forceinline__ bool sample_begin(const ImageParams &p, int i, SampleInfo &s) {
+    return p.fused_plan ? sample_plan<NT>(p, i, s) : sample_info(p, i, s);
+}
+
 template <int NT>
 __device__ __forceinline__ void meta_init(const ImageParams &p, const SampleInfo &s, MetaPtrs &m) {
     const int tid = threadIdx.x;
@@ -188,17 +307,24 @@ __device__ __forceinline__ F2 mean_of(F2 num, F2 den, F2 inv, __nv_bfloat16) {
 }
 __device__ __forceinline__ F2 mean_of(F2 num, F2 den, F2, float) { return f2_div(num, den); }
 
-// bf16 bits of num / den rounded to nearest even.  q1 = num.hi * inv.hi carries three
+// bf16 bits of num / den rounded to nearest even.  A power-of-two den (uniform over a
+// merged row; every merge of two unit-size tokens) scales num exactly, so the float-float
+// product rounds directly, as in mean_of.  Otherwise q1 = num.hi * inv.hi carries three
 // relative errors of at most 2^-24 each (num.lo dropped, inv.lo dropped, the product's
 // rounding), so it lies within 4 float32 ulps of the exact quotient: when it is more than
 // 8 ulps from every bf16 rounding midpoint it rounds like the exact quotient; otherwise
 // the float-float path above decides.
-__device__ __forceinline__ uint16_t mean_bits(F2 num, F2 den, F2 inv, __nv_bfloat16) {
+// The rare case near a midpoint, out of line so that the common path stays short.
+static __device__ __noinline__ uint16_t mean_bits_slow(F2 num, F2 den, F2 inv) {
+    return f2_to_bf16_bits(mean_of(num, den, inv, __nv_bfloat16{}));
+}
+__device__ __forceinline__ uint16_t mean_bits(F2 num, F2 den, F2 inv, bool pow2, __nv_bfloat16) {
+    if (pow2) return f2_to_bf16_bits(f2_mul(num, inv));
     const uint32_t u = __float_as_uint(__fmul_rn(num.hi, inv.hi));
     const uint32_t low = u & 0xFFFFu;
     const uint32_t dist = low > 0x8000u ? low - 0x8000u : 0x8000u - low;
     if (dist > 8u && (u & 0x7F800000u) != 0x7F800000u) return (uint16_t)((u + 0x8000u) >> 16);
-    return f2_to_bf16_bits(mean_of(num, den, inv, __nv_bfloat16{}));
+    return mean_bits_slow(num, den, inv);
 }
 
 // Accumulator of exact products: hi parts summed with two_sum, the rounding errors and
@@ -220,11 +346,12 @@ struct Acc2 {
 };
 
 __device__ __forceinline__ uint4 merged_pack(const Acc2 (&num)[8], F2 den, F2 inv, __nv_bfloat16) {
+    const bool pow2 = den.lo == 0.0f && (__float_as_uint(den.hi) & 0x007FFFFFu) == 0u;
     uint32_t w[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k)
-        w[k] = (uint32_t)mean_bits(num[2 * k].value(), den, inv, __nv_bfloat16{}) |
-               ((uint32_t)mean_bits(num[2 * k + 1].value(), den, inv, __nv_bfloat16{}) << 16);
+        w[k] = (uint32_t)mean_bits(num[2 * k].value(), den, inv, pow2, __nv_bfloat16{}) |
+               ((uint32_t)mean_bits(num[2 * k + 1].value(), den, inv, pow2, __nv_bfloat16{}) << 16);
     return make_uint4(w[0], w[1], w[2], w[3]);
 }
 __device__ __forceinline__ uint4 merged_pack(const Acc2 (&num)[4], F2 den, F2 inv, float) {

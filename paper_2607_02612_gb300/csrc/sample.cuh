@@ -56,6 +56,15 @@ __host__ __device__ inline Meta meta_layout(int nmax, size_t base) {
 }
 
 struct MetaPtrs {
+    MetaPtrs() = default;
+    // only the arrays a merged mean reads (sizes, source lists, inverse size sums)
+    __device__ static MetaPtrs views(const float *tsize, const int *slist, const float2 *invd) {
+        MetaPtrs m{};
+        m.tsize = const_cast<float *>(tsize);
+        m.slist = const_cast<int *>(slist);
+        m.invd = const_cast<float2 *>(invd);
+        return m;
+    }
     unsigned long long *best, *rk, *pk;
     float *inv_a, *inv_b;
     int *match, *sel, *mkey, *mflag, *kflag, *opos, *srcpos, *scnt, *slist, *mlist;
@@ -434,6 +443,93 @@ __device__ __forceinline__ uint4 merged_compute(const MetaPtrs &m, const MergedI
     return merged_pack(num, den, {iv.x, iv.y}, T{});
 }
 
+// A size whose product with any bf16 value (8 significant bits) is exact in float: at most
+// 16 significant bits, at least 1 (so products with subnormal values stay on the float
+// grid) and below 2^64.
+__device__ __forceinline__ bool short_size(float s) {
+    return s >= 1.0f && s < 0x1p64f && (__float_as_uint(s) & 0xFFu) == 0u;
+}
+
+// The exact float-float mean of a chunk, out of line; everything passed by value so the
+// caller keeps its state in registers.
+template <typename Loader>
+__device__ __noinline__ uint4 merged_exact_bf16(const float *tsize, const int *slist, const float2 *invd, int pos, int c,
+                                                int q0, int q1, uint4 self, uint4 av0, uint4 av1, Loader load) {
+    MergedItem it;
+    it.pos = pos;
+    it.c = c;
+    it.q0 = q0;
+    it.q1 = q1;
+    it.self = self;
+    it.av[0] = av0;
+    it.av[1] = av1;
+    MetaPtrs m = MetaPtrs::views(tsize, slist, invd);
+    return merged_compute<__nv_bfloat16>(m, it, load);
+}
+
+// A bf16 merged chunk, exactly rounded, in float.  When every size is short, every
+// product s x is exact; a two_sum chain over the products then shows whether their float
+// sum num is the exact numerator (it is unless the terms lie more than 2^24 apart).  With
+// num exact and den (the float sum of the sizes) exact:
+//  * q0 = num * inv.hi lies within a few float ulps of the exact mean t = num / den, so t
+//    lies in the bf16 interval [b, b+1] that holds q0 or within a few float ulps of its
+//    ends, where the rounding is that of the nearest end anyway;
+//  * m, the midpoint of that interval, decides the rounding: R = fma(m, -den, num) is
+//    num - m den rounded once, so its sign (and whether it is zero) is that of t - m:
+//    t beyond m rounds away from b, short of m to b, exactly on m to the even end.
+// Otherwise (long sizes, an inexact sum, non-finite values) the float-float computation
+// runs, out of line.
+template <typename Loader>
+__device__ __forceinline__ uint4 merged_fast_bf16(const MetaPtrs &m, const MergedItem &it, const Loader &load) {
+    const float sb = m.tsize[it.pos];
+    const float2 iv = m.invd[it.pos];   // 1 / den as float-float
+    float num[8], x[8];
+    chunk_to_f(it.self, x);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) num[e] = __fmul_rn(sb, x[e]);
+    float den = sb;
+    bool ok = short_size(sb);
+    for (int q = it.q0; q < it.q1; ++q) {
+        const int u = q - it.q0;
+        const int ap = 2 + 2 * m.slist[q];
+        const float sa = m.tsize[ap];
+        const F2 dd = two_sum(den, sa);
+        den = dd.hi;
+        ok = ok && short_size(sa) && dd.lo == 0.0f;
+        chunk_to_f(u == 0 ? it.av[0] : u == 1 ? it.av[1] : load(ap, it.c), x);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const F2 t = two_sum(num[e], __fmul_rn(sa, x[e]));
+            num[e] = t.hi;
+            ok = ok && t.lo == 0.0f;
+        }
+    }
+    uint32_t bits[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        const uint32_t uq = __float_as_uint(__fmul_rn(num[e], iv.x));
+        ok = ok && ((uq >> 23) & 0xFFu) != 0xFFu;
+        const float mid = __uint_as_float((uq & 0xFFFF0000u) | 0x8000u);
+        const float R = __fmaf_rn(mid, -den, num[e]);
+        const uint32_t b = uq >> 16;
+        const bool neg = (uq >> 31) != 0u;
+        const bool up = R == 0.0f ? (b & 1u) != 0u : ((R > 0.0f) != neg);
+        bits[e] = b + (up ? 1u : 0u);
+    }
+    if (!ok)
+        return merged_exact_bf16(m.tsize, m.slist, m.invd, it.pos, it.c, it.q0, it.q1, it.self, it.av[0], it.av[1], load);
+    return make_uint4(bits[0] | (bits[1] << 16), bits[2] | (bits[3] << 16), bits[4] | (bits[5] << 16),
+                      bits[6] | (bits[7] << 16));
+}
+
+template <typename T, typename Loader>
+__device__ __forceinline__ uint4 merged_value(const MetaPtrs &m, const MergedItem &it, const Loader &load) {
+    if constexpr (Elem<T>::kBytes == 2)
+        return merged_fast_bf16(m, it, load);
+    else
+        return merged_compute<T>(m, it, load);
+}
+
 // Requires sel / match / mkey / tsize / tscore ready (after a barrier).  `load(pos, c)`
 // returns the 16-byte chunk c of input token pos.  Returns false (after raising
 // FUSION_DEV_INTERNAL) if the token count disagrees with the plan; uniform per CTA.
@@ -594,7 +690,7 @@ __device__ bool finish_sample(const ImageParams &p, const SampleInfo &s, MetaPtr
         MergedItem nxt;
         merged_fetch(m, t + NT, n_items, ncx, load, nxt);
         if (cur.pos >= 0)
-            *reinterpret_cast<uint4 *>(xo + m.opos[cur.pos] * dim + cur.c * CH) = merged_compute<T>(m, cur, load);
+            *reinterpret_cast<uint4 *>(xo + m.opos[cur.pos] * dim + cur.c * CH) = merged_value<T>(m, cur, load);
         cur = nxt;
     }
     return true;

@@ -103,6 +103,42 @@ def test_identical_keys_zero_norm_and_signed_zero(dtype):
     run_stage_and_compare(b2, spec2, f"zero-key {dtype}")
 
 
+def _grid_batch(counts, dim, seed, scale=1.0):
+    """bf16 tokens on a coarse grid (multiples of 2^-5 in [-4, 4), times `scale`), so that
+    size-weighted means land exactly on, or right next to, bf16 rounding midpoints; sizes
+    mix integers and halves (power-of-two and other sums); keys are unit vectors that send
+    A token a to B token f(a), with one, two or three sources per destination."""
+    rng = np.random.default_rng(seed)
+    counts = np.asarray(counts)
+    offs = np.concatenate([[0], np.cumsum(counts)]).astype(np.int32)
+    T = int(offs[-1])
+    x32 = (rng.integers(-128, 128, (T, dim)) / 32.0 * scale).astype(np.float32)
+    k32 = np.zeros((T, dim), np.float32)
+    for i in range(len(counts)):
+        N = int(counts[i]); base = int(offs[i]); nB = N // 2
+        for pos in range(1, N):
+            if pos % 2 == 1:
+                k32[base + pos, ((pos - 1) // 2) % dim] = 1.0
+            else:
+                a = (pos - 2) // 2
+                dest = a if a < nB // 3 else (a // 2 if a < 2 * nB // 3 else a // 3)
+                k32[base + pos, min(dest, nB - 1) % dim] = 1.0
+        k32[base, :] = 1.0
+    sz = rng.choice(np.array([1, 1, 1, 2, 3, 0.5, 1.5, 7], np.float32), T).astype(np.float32)
+    sc = rng.random(T).astype(np.float32)
+    return Batch("bf16", offs, f32_to_bf16_bits(x32), f32_to_bf16_bits(k32), sz, sc)
+
+
+@pytest.mark.parametrize("scale", [1.0, 2.0 ** -100, 2.0 ** -110])
+def test_merged_mean_rounding_ties_and_near_ties(scale):
+    """bf16 merged tokens must be the exactly rounded weighted mean, ties to even, whatever
+    path the kernel takes (two-term power-of-two sums, the bounded float path, the exact
+    float-float path for three sources or near-midpoint and tiny values)."""
+    b = _grid_batch([65, 129, 97, 33, 65], 64, seed=21, scale=scale)
+    r = np.array([32, 64, 40, 16, 20], np.int32)
+    run_stage_and_compare(b, StageSpec(True, False, False, r=r), f"grid means scale={scale}")
+
+
 @pytest.mark.parametrize("tau", [0.0, 2.0])
 def test_all_or_no_samples_exit(tau):
     b = make_batch([10] * 37, 64, "bf16", seed=3)
@@ -213,6 +249,43 @@ def test_bad_batch_and_ids_raise_status():
     st, o = _stage_raw(b, db, ids=torch.tensor([0, 7], dtype=torch.int32, device="cuda"))
     assert st & fz.FUSION_DEV_BAD_IDS
     assert torch.all(o["keep_idx"] == -5)
+
+
+def _stage_raw_exit(db, offsets=None, batch=None, ids=None):
+    """bf16 merge + exit + prune on the tcgen05 per-sample kernel, with malformed inputs."""
+    head = runner.head_tensors(make_head(db.dim, 10, "bf16", 0.5), "bf16")
+    f = runner.Fusion(db.max_batch, 10)
+    o = f.stage_outputs(db, 7, head)
+    o["x"].fill_(7)
+    o["keep_idx"].fill_(-5)
+    rr = torch.full((db.max_batch,), 2, dtype=torch.int32, device="cuda")
+    rho = torch.full((db.max_batch,), 0.5, dtype=torch.float32, device="cuda")
+    rg = fz.ragged(db.max_batch, db.max_tokens, db.max_rows, offsets if offsets is not None else db.offsets,
+                   batch, ids)
+    fz.check(fz.fusion_stage(fz.FUSION_BF16, 7, rg, db.x, db.dim, db.keys, db.key_dim, db.sizes, db.scores, rr,
+                             rho, head.c_struct(), o["exit_mask"], o["logits"], o["max_prob"], o["x"], o["sizes"],
+                             o["scores"], o["offsets"], o["ids"], o["batch"], o["keep_idx"], None, f.workspace,
+                             f.ws_bytes, f.status))
+    torch.cuda.synchronize()
+    return int(f.status.item()), o
+
+
+def test_malformed_inputs_with_exit_check_write_nothing():
+    b = make_batch([20, 20, 20], 64, "bf16", seed=11)
+    db = P.device_batch(b)
+    st, o = _stage_raw_exit(db)
+    assert st == 0
+    for bad in ([0, 20, 10, 60], [0, 20, 40, 99], [-3, 20, 40, 60], [0, 0, 40, 60]):
+        st, o = _stage_raw_exit(db, offsets=torch.tensor(bad, dtype=torch.int32, device="cuda"))
+        assert st & fz.FUSION_DEV_BAD_OFFSETS, bad
+        assert torch.all(o["keep_idx"] == -5) and torch.all(o["x"] == 7), bad
+        assert int(o["batch"][0]) == 0 and int(o["offsets"][0]) == 0, bad
+    st, o = _stage_raw_exit(db, batch=torch.full((1,), 4, dtype=torch.int32, device="cuda"))
+    assert st & fz.FUSION_DEV_BAD_BATCH
+    assert torch.all(o["keep_idx"] == -5) and torch.all(o["x"] == 7)
+    st, o = _stage_raw_exit(db, ids=torch.tensor([0, 9, 1], dtype=torch.int32, device="cuda"))
+    assert st & fz.FUSION_DEV_BAD_IDS
+    assert torch.all(o["keep_idx"] == -5) and torch.all(o["x"] == 7)
 
 
 def test_nonfinite_keys_raise_status():

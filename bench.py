@@ -10,7 +10,9 @@ and every stage reads its input from HBM, as it would after a real block.
 
 value     images/s per stage: images entering each stage, summed over the step's
           stages and over all ranks, divided by the (max over ranks) sum of the
-          stages' CUDA-event times.
+          stages' CUDA-event times.  A step (flushes, events and stages) is captured
+          once as a CUDA graph and replayed, as a serving loop would launch it
+          (--eager launches every kernel from the host instead).
 roofline  the per-sample kernel (merge + prune + gather), which moves almost all
           bytes: algorithmic bytes / event-timed duration vs the measured HBM copy
           bandwidth.
@@ -55,6 +57,7 @@ def parse_args():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--e2e-steps", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--eager", action="store_true", help="launch every step from the host instead of a CUDA graph")
     ap.add_argument("--ref-sample", type=int, default=16, help="images per reference step")
     return ap.parse_args()
 
@@ -285,34 +288,60 @@ def main():
             import torch.distributed as dist
             dist.barrier()
 
+    # the mid event only where a first kernel runs (the exit check, or the plan kernel of a
+    # batch too large for the fused plan): an empty start-to-mid interval still costs an
+    # event record on the stream
+    has_first = [bool(specs[s].exit) or b.batch > fz.FUSION_FUSED_PLAN_MAX_BATCH for s in range(S)]
+
     def run_step(evs):
         for s in range(S):
             flush.fill_(s & 0xFF)
-            fz.fusion_profile_next(*evs[s])
+            e0, e1, e2 = evs[s]
+            fz.fusion_profile_next(e0, e1 if has_first[s] else None, e2)
             chain.run_stage(s)
 
     mk = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
-    warm_evs = [(mk(), mk(), mk()) for _ in range(S)]
-    for _ in range(args.warmup):
-        run_step(warm_evs)
+    step_evs = [(mk(), mk(), mk()) for _ in range(S)]
+    for trio in step_evs:      # create the CUDA events outside any capture
+        for e in trio:
+            e.record()
+    run_step(step_evs)         # one eager step: first launches, kernel attributes
     torch.cuda.synchronize()
     st = int(fus.status.item())
     if st != 0:
         raise SystemExit(f"device status {st} ({fz.fusion_status_string(st)})")
+    graph = None
+    if not args.eager:
+        # one step (flushes, events, stages) as a CUDA graph: the launch path a serving loop
+        # would use; the events are graph nodes and record at every replay
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            run_step(step_evs)
+    one = graph.replay if graph is not None else (lambda: run_step(step_evs))
+    for _ in range(args.warmup):
+        one()
+    torch.cuda.synchronize()
 
-    evs = [[(mk(), mk(), mk()) for _ in range(S)] for _ in range(args.steps)]
+    def read(trio_list):
+        return ([t[0].elapsed_time(t[2]) for t in trio_list],
+                [t[0].elapsed_time(t[1]) if has_first[s] else 0.0 for s, t in enumerate(trio_list)])
+
+    stage_rows, first_rows = [], []
     barrier()
     torch.cuda.synchronize()
     with ClockSampler(local) as clk:
         t0 = time.perf_counter()
         for k in range(args.steps):
-            run_step(evs[k])
-        torch.cuda.synchronize()
+            one()
+            torch.cuda.synchronize()   # the step's events are read before the next replay
+            a_, b_ = read(step_evs)
+            stage_rows.append(a_)
+            first_rows.append(b_)
         wall = time.perf_counter() - t0
     barrier()
-    stage_ms = np.array([[evs[k][s][0].elapsed_time(evs[k][s][2]) for s in range(S)] for k in range(args.steps)])
-    first_ms = np.array([[evs[k][s][0].elapsed_time(evs[k][s][1]) for s in range(S)] for k in range(args.steps)])
-    image_ms = np.array([[evs[k][s][1].elapsed_time(evs[k][s][2]) for s in range(S)] for k in range(args.steps)])
+    stage_ms = np.array(stage_rows)
+    first_ms = np.array(first_rows)
+    image_ms = stage_ms - first_ms
     clocks = clk.summary()
 
     # images entering each stage and algorithmic bytes, from the (deterministic) outputs
@@ -362,7 +391,8 @@ def main():
         "config": {"workload": args.workload, "batch": b.batch, "tokens": int(np.diff(b.offsets).max()),
                    "dim": b.dim, "stages": S, "exit_blocks": list(w.spec.exit_blocks),
                    "l2": "flushed before every stage (512 MB write, untimed)",
-                   "timing": "CUDA events around each stage's kernels, summed"},
+                   "timing": ("CUDA events around each stage's kernels, summed; " +
+                              ("eager launches" if args.eager else "one step captured as a CUDA graph and replayed"))},
         "roofline": {"bound": "hbm", "kernel": "k_image (merge + prune + gather)", "achieved": achieved,
                      "peak": peak, "unit": "GB/s", "frac": achieved / peak, "peak_source": peak_src,
                      "traffic": (tr["dram_bytes_per_launch"] if tr else None),

@@ -89,6 +89,9 @@ extern "C" {
 
 #define FUSION_MAX_TOKENS 1024
 #define FUSION_MAX_DIM 1024
+/* batches of at most this many samples run their plan (validation, output offsets)
+   inside the per-sample kernel; larger ones launch a plan kernel first */
+#define FUSION_FUSED_PLAN_MAX_BATCH 1024
 
 /* A ragged batch as seen by the device.  All pointers are device memory. */
 typedef struct fusion_ragged {
@@ -123,8 +126,9 @@ const char *fusion_version(void);
  * from the calling host thread to record up to three CUDA events (cudaEvent_t
  * passed as void*, NULL to skip) on that call's stream: `start` before its first
  * kernel, `mid` between its first kernel (plan or exit check) and its
- * per-sample kernel, `end` after its last kernel.  The events are created and
- * owned by the caller.  Returns FUSION_OK.
+ * per-sample kernel, `end` after its last kernel.  Inside a stream capture the
+ * events are recorded by graph nodes, at every replay.  The events are created
+ * and owned by the caller.  Returns FUSION_OK.
  */
 int fusion_profile_next(void *start, void *mid, void *end);
 

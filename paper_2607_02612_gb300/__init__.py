@@ -20,6 +20,7 @@ from ._binding import (  # noqa: F401
     FUSION_ERR_SHAPE,
     FUSION_ERR_WORKSPACE,
     FUSION_F32,
+    FUSION_FUSED_PLAN_MAX_BATCH,
     FUSION_MAX_DIM,
     FUSION_MAX_TOKENS,
     FUSION_OK,

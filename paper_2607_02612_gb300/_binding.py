@@ -35,6 +35,7 @@ FUSION_STAGE_MERGE = 1
 FUSION_STAGE_EXIT = 2
 FUSION_STAGE_PRUNE = 4
 FUSION_MAX_TOKENS = 1024
+FUSION_FUSED_PLAN_MAX_BATCH = 1024
 FUSION_MAX_DIM = 1024
 
 EXPORTED = ("fusion_status_string", "fusion_version", "fusion_profile_next", "fusion_workspace_size",

@@ -1,13 +1,18 @@
 // Exit check (Sec. III-D, Eq. 6-7): u = LayerNorm(CLS), logits = W u + b,
 // c = max_k softmax(logits)_k, exit iff c >= tau.
 //
-// Grid: (class tiles of kExitCT) x (sample tiles of kExitBT).  Every CTA computes
+// Two kernels.  The cluster kernel (heads of at most 8 class tiles) is described below.
+// The general one: grid (class tiles of kExitCT) x (sample tiles of kExitBT).  Every CTA computes
 // the LayerNorm of its samples' CLS rows, one logits tile (bf16: mma.sync tensor
 // cores with float32 accumulation; f32: FFMA) and a partial softmax (tile max and
 // sum of exponentials) per sample.  The last CTA of a sample tile to finish
 // (atomic counter, no waiting) merges the partials into c and the exit mask; the
 // last sample tile to finish runs the compaction plan for the fused stage.
+#include <cooperative_groups.h>
+
 #include "launch.h"
+
+namespace cg = cooperative_groups;
 
 namespace fz {
 namespace {
@@ -86,6 +91,116 @@ struct ExitSmem {
         return t > plan ? t : plan;
     }
 };
+
+// The logits tile [kExitBT samples] x [kExitCT classes] of one CTA, K chunks of the head
+// double-buffered (chunks 0 and 1 already in flight): bf16 mma.sync with float32
+// accumulation, f32 FFMA.  u_s holds the LayerNorm rows (16 rows for the bf16 A tile).
+template <typename T>
+__device__ __forceinline__ void exit_gemm(const ExitParams &p, const T *u_s, unsigned char *w_region, int c0, int dim,
+                                          int C, int n_k, float (&acc)[4], float (&acc2)[4]) {
+    using S = ExitSmem<T>;
+    constexpr int KC = S::KC;
+    constexpr bool kBf16 = (Elem<T>::kBytes == 2);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int u_stride = S::u_stride(dim);
+    for (int kc = 0; kc < n_k; ++kc) {
+        const int k0 = kc * KC;
+        const int kw = min(KC, dim - k0);
+        unsigned char *wbuf = w_region + (kc & 1) * S::w_stage;
+        if (kc + 1 < n_k)
+            asm volatile("cp.async.wait_group 1;\n" ::: "memory");
+        else
+            cp_async_wait_all();
+        __syncthreads();
+        if constexpr (kBf16) {
+            // warp -> the 16-row sample tile (rows 8..15 are zero) x 16 classes
+            float t0[4] = {0.0f, 0.0f, 0.0f, 0.0f}, t1[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+            const uint32_t ubase = smem_addr(u_s);
+            const uint32_t wbase = smem_addr(wbuf);
+            const int arow = (lane & 7) + ((lane >> 3) & 1) * 8;
+            const int brow = warp * 16 + (lane >> 4) * 8 + (lane & 7);
+            for (int kk = 0; kk < kw; kk += 16) {
+                uint32_t af[4], b0, b1, b2, b3;
+                ldsm_x4(ubase + (uint32_t)((arow * u_stride + k0 + kk + (lane >> 4) * 8) * 2), af[0], af[1],
+                        af[2], af[3]);
+                ldsm_x4(wbase + (uint32_t)((brow * S::w_stride + kk + ((lane >> 3) & 1) * 8) * 2), b0, b1, b2, b3);
+                mma_bf16_16816(t0, af, b0, b1);
+                mma_bf16_16816(t1, af, b2, b3);
+                if ((kk & 63) == 48) {   // flush the partial sums every 64 dims
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        acc[e] += t0[e];
+                        acc2[e] += t1[e];
+                        t0[e] = t1[e] = 0.0f;
+                    }
+                }
+            }
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                acc[e] += t0[e];
+                acc2[e] += t1[e];
+            }
+        } else {
+            // warp -> sample `warp`; lane -> classes lane + 32 q
+            const float *ur = reinterpret_cast<const float *>(u_s) + (size_t)warp * u_stride + k0;
+            const float *ws = reinterpret_cast<const float *>(wbuf);
+            float t[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+            for (int kk = 0; kk < kw; kk += 4) {
+                const float4 uv = *reinterpret_cast<const float4 *>(ur + kk);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float4 wv = *reinterpret_cast<const float4 *>(ws + (lane + 32 * q) * S::w_stride + kk);
+                    t[q] = fmaf(uv.x, wv.x, t[q]);
+                    t[q] = fmaf(uv.y, wv.y, t[q]);
+                    t[q] = fmaf(uv.z, wv.z, t[q]);
+                    t[q] = fmaf(uv.w, wv.w, t[q]);
+                }
+                if ((kk & 15) == 12) {   // flush every 16 dims
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        acc[q] += t[q];
+                        t[q] = 0.0f;
+                    }
+                }
+            }
+#pragma unroll
+            for (int q = 0; q < 4; ++q) acc[q] += t[q];
+        }
+        __syncthreads();   // everyone is done with this stage buffer
+        if (kc + 2 < n_k) issue_w_chunk<T>(p, wbuf, c0, k0 + 2 * KC, dim, C, tid);
+    }
+}
+
+// Logits (+ bias) into shared memory (padded classes get -inf) and to p.logits.
+template <typename T>
+__device__ __forceinline__ void exit_logits(const ExitParams &p, float *lg_s, const float *bias_s, const float (&acc)[4],
+                                            const float (&acc2)[4], int s0, int c0, int B, int C) {
+    constexpr bool kBf16 = (Elem<T>::kBytes == 2);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    // ---- logits (+ bias) into shared memory; padded classes get -inf ---------------
+    if constexpr (kBf16) {
+        const int g = lane >> 2, t4 = lane & 3;   // fragment rows g (valid) and g + 8 (padding)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            const int col0 = warp * 16 + 2 * t4 + e, col1 = col0 + 8;
+            lg_s[g * kExitCT + col0] = (c0 + col0 < C) ? acc[e] + bias_s[col0] : -INFINITY;
+            lg_s[g * kExitCT + col1] = (c0 + col1 < C) ? acc2[e] + bias_s[col1] : -INFINITY;
+        }
+    } else {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int col = lane + 32 * q;
+            lg_s[warp * kExitCT + col] = (c0 + col < C) ? acc[q] + bias_s[col] : -INFINITY;
+        }
+    }
+    __syncthreads();
+    if (p.logits) {
+        for (int it = tid; it < kExitBT * kExitCT; it += kExitThreads) {
+            const int sl = it / kExitCT, col = it - sl * kExitCT;
+            if (s0 + sl < B && c0 + col < C) p.logits[(size_t)(s0 + sl) * C + c0 + col] = lg_s[it];
+        }
+    }
+}
 
 template <typename T>
 __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
@@ -206,96 +321,8 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
     float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};   // bf16: two m16n8 fragments' valid rows; f32: 4 classes
     float acc2[4] = {0.0f, 0.0f, 0.0f, 0.0f};
     if (active) {
-        for (int kc = 0; kc < n_k; ++kc) {
-            const int k0 = kc * KC;
-            const int kw = min(KC, dim - k0);
-            unsigned char *wbuf = w_region + (kc & 1) * S::w_stage;
-            if (kc + 1 < n_k)
-                asm volatile("cp.async.wait_group 1;\n" ::: "memory");
-            else
-                cp_async_wait_all();
-            __syncthreads();
-            if constexpr (kBf16) {
-                // warp -> the 16-row sample tile (rows 8..15 are zero) x 16 classes
-                float t0[4] = {0.0f, 0.0f, 0.0f, 0.0f}, t1[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-                const uint32_t ubase = smem_addr(u_s);
-                const uint32_t wbase = smem_addr(wbuf);
-                const int arow = (lane & 7) + ((lane >> 3) & 1) * 8;
-                const int brow = warp * 16 + (lane >> 4) * 8 + (lane & 7);
-                for (int kk = 0; kk < kw; kk += 16) {
-                    uint32_t af[4], b0, b1, b2, b3;
-                    ldsm_x4(ubase + (uint32_t)((arow * u_stride + k0 + kk + (lane >> 4) * 8) * 2), af[0], af[1],
-                            af[2], af[3]);
-                    ldsm_x4(wbase + (uint32_t)((brow * S::w_stride + kk + ((lane >> 3) & 1) * 8) * 2), b0, b1, b2, b3);
-                    mma_bf16_16816(t0, af, b0, b1);
-                    mma_bf16_16816(t1, af, b2, b3);
-                    if ((kk & 63) == 48) {   // flush the partial sums every 64 dims
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            acc[e] += t0[e];
-                            acc2[e] += t1[e];
-                            t0[e] = t1[e] = 0.0f;
-                        }
-                    }
-                }
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    acc[e] += t0[e];
-                    acc2[e] += t1[e];
-                }
-            } else {
-                // warp -> sample `warp`; lane -> classes lane + 32 q
-                const float *ur = reinterpret_cast<const float *>(u_s) + (size_t)warp * u_stride + k0;
-                const float *ws = reinterpret_cast<const float *>(wbuf);
-                float t[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-                for (int kk = 0; kk < kw; kk += 4) {
-                    const float4 uv = *reinterpret_cast<const float4 *>(ur + kk);
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const float4 wv = *reinterpret_cast<const float4 *>(ws + (lane + 32 * q) * S::w_stride + kk);
-                        t[q] = fmaf(uv.x, wv.x, t[q]);
-                        t[q] = fmaf(uv.y, wv.y, t[q]);
-                        t[q] = fmaf(uv.z, wv.z, t[q]);
-                        t[q] = fmaf(uv.w, wv.w, t[q]);
-                    }
-                    if ((kk & 15) == 12) {   // flush every 16 dims
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            acc[q] += t[q];
-                            t[q] = 0.0f;
-                        }
-                    }
-                }
-#pragma unroll
-                for (int q = 0; q < 4; ++q) acc[q] += t[q];
-            }
-            __syncthreads();   // everyone is done with this stage buffer
-            if (kc + 2 < n_k) issue_w_chunk<T>(p, wbuf, c0, k0 + 2 * KC, dim, C, tid);
-        }
-
-        // ---- logits (+ bias) into shared memory; padded classes get -inf ---------------
-        if constexpr (kBf16) {
-            const int g = lane >> 2, t4 = lane & 3;   // fragment rows g (valid) and g + 8 (padding)
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-                const int col0 = warp * 16 + 2 * t4 + e, col1 = col0 + 8;
-                lg_s[g * kExitCT + col0] = (c0 + col0 < C) ? acc[e] + bias_s[col0] : -INFINITY;
-                lg_s[g * kExitCT + col1] = (c0 + col1 < C) ? acc2[e] + bias_s[col1] : -INFINITY;
-            }
-        } else {
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int col = lane + 32 * q;
-                lg_s[warp * kExitCT + col] = (c0 + col < C) ? acc[q] + bias_s[col] : -INFINITY;
-            }
-        }
-        __syncthreads();
-        if (p.logits) {
-            for (int it = tid; it < kExitBT * kExitCT; it += kExitThreads) {
-                const int sl = it / kExitCT, col = it - sl * kExitCT;
-                if (s0 + sl < B && c0 + col < C) p.logits[(size_t)(s0 + sl) * C + c0 + col] = lg_s[it];
-            }
-        }
+        exit_gemm<T>(p, u_s, w_region, c0, dim, C, n_k, acc, acc2);
+        exit_logits<T>(p, lg_s, bias_s, acc, acc2, s0, c0, B, C);
         // ---- partial softmax of this class tile: warp -> sample ------------------------
         {
             const int sl = warp, s = s0 + sl;
@@ -360,13 +387,291 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
     if (p.do_plan) run_plan(p.plan, reinterpret_cast<int *>(sm));
 }
 
+__device__ __forceinline__ float to_float(float v) { return v; }
+__device__ __forceinline__ float to_float(__nv_bfloat16 v) { return __bfloat162float(v); }
+
+// ---------------------------------------------------------------------------
+// The exit check as thread-block clusters: the n_ctile (<= 8) class tiles of one sample
+// tile form a cluster.  Cluster rank r computes the LayerNorm of the tile's samples
+// r, r + n_ctile, ... with several warps per row (one pass: sum and sum of squares in
+// float-float, var = E[x^2] - mean^2) and stores the normalised row into the shared
+// memory of every CTA of the cluster; each CTA then computes its logits tile and partial
+// softmax, sends (max, sum of exponentials) to the sample's owner, and the owner merges
+// them.  The head's weight chunks load while the LayerNorm runs; no global atomics
+// unless the plan kernel's work runs here (batches above the fused-plan bound).
+// ---------------------------------------------------------------------------
+template <typename T>
+struct ExitClSmem {
+    static constexpr int EB = Elem<T>::kBytes;
+    using B = ExitSmem<T>;
+    // u rows (16, the GEMM's A tile) | own raw CLS rows (kExitBT) | gamma | beta | W stages (2)
+    // | bias | partials [kExitBT][8] | reduction scratch
+    static __host__ __device__ size_t x_off(int dim) { return B::u_bytes(dim); }
+    static __host__ __device__ size_t g_off(int dim) { return x_off(dim) + (size_t)kExitBT * B::u_stride(dim) * EB; }
+    static __host__ __device__ size_t be_off(int dim) { return g_off(dim) + ((size_t)dim * EB + 15) / 16 * 16; }
+    static __host__ __device__ size_t w_off(int dim) { return be_off(dim) + ((size_t)dim * EB + 15) / 16 * 16; }
+    static __host__ __device__ size_t bias_off(int dim) { return w_off(dim) + 2 * B::w_stage; }
+    static __host__ __device__ size_t part_off(int dim) { return bias_off(dim) + kExitCT * sizeof(float); }
+    static __host__ __device__ size_t red_off(int dim) { return part_off(dim) + (size_t)kExitBT * 8 * sizeof(float2); }
+    static __host__ __device__ size_t total(int dim) {
+        const size_t t = red_off(dim) + (size_t)(kExitThreads / 32) * 8 * sizeof(float);
+        const size_t plan = w_off(dim) + (4 * kExitThreads + 40) * sizeof(int);   // run_plan reuses the W stages
+        return t > plan ? t : plan;
+    }
+};
+
+template <typename T>
+__global__ void __launch_bounds__(kExitThreads) k_exit_cl(ExitParams p) {
+    extern __shared__ __align__(16) unsigned char sm[];
+    using S = ExitSmem<T>;
+    using L = ExitClSmem<T>;
+    constexpr int CH = Elem<T>::kPerChunk;
+    constexpr int EB = Elem<T>::kBytes;
+    constexpr int KC = S::KC;
+    constexpr bool kBf16 = (EB == 2);
+    constexpr int kWarps = kExitThreads / 32;
+    cg::cluster_group cl = cg::this_cluster();
+    const int ncl = (int)cl.num_blocks(), rank = (int)cl.block_rank();
+    const int dim = p.dim, nchunk = dim / CH, u_stride = S::u_stride(dim);
+    T *u_s = reinterpret_cast<T *>(sm);
+    T *x_s = reinterpret_cast<T *>(sm + L::x_off(dim));
+    T *g_s = reinterpret_cast<T *>(sm + L::g_off(dim));
+    T *be_s = reinterpret_cast<T *>(sm + L::be_off(dim));
+    unsigned char *w_region = sm + L::w_off(dim);
+    float *lg_s = reinterpret_cast<float *>(w_region);   // [kExitBT][kExitCT], reused after the GEMM
+    float *bias_s = reinterpret_cast<float *>(sm + L::bias_off(dim));
+    float2 *part_s = reinterpret_cast<float2 *>(sm + L::part_off(dim));
+    float *red = reinterpret_cast<float *>(sm + L::red_off(dim));
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int ct = blockIdx.x, bt = blockIdx.y;
+    const int s0 = bt * kExitBT, c0 = ct * kExitCT;
+    const int C = p.head.classes;
+    const int Bdev = device_batch(p.in);
+    const int B = Bdev < 0 ? 0 : Bdev;
+    const bool active = s0 < B;   // uniform over the cluster (same sample tile)
+    const int n_k = (dim + KC - 1) / KC;
+    // rows of this CTA: slot j -> sample slot sl = rank + j * ncl; G warps per row
+    int nrp = 1;
+    while (nrp * ncl < kExitBT) nrp <<= 1;
+    const int G = kWarps / nrp;
+    const int j = warp / G, gt = tid - j * G * 32;   // row slot of this warp, thread index in its group
+    const int sl = rank + j * ncl;
+    const bool has_row = sl < kExitBT;
+    const int s = s0 + sl;
+
+    if (active) {
+        // own CLS rows, gamma and beta first (group 0), then weight chunks 0 and 1
+        for (int it = tid; it < kExitBT * nchunk; it += kExitThreads) {
+            const int jj = it / nchunk, c = it - jj * nchunk;
+            const int sli = rank + jj * ncl, si = s0 + sli;
+            T *dst = x_s + (size_t)jj * u_stride + c * CH;
+            long long row = -1;
+            if (sli < kExitBT && si < B) {
+                row = p.in.offsets[si];
+                if (row < 0 || row >= p.in.max_rows) row = -1;
+            }
+            if (row >= 0)
+                cp_async16(dst, reinterpret_cast<const T *>(p.x) + row * dim + c * CH);
+            else
+                *reinterpret_cast<uint4 *>(dst) = make_uint4(0, 0, 0, 0);
+        }
+        for (int c = tid; c < 2 * nchunk; c += kExitThreads) {
+            const bool isg = c < nchunk;
+            const int cc = isg ? c : c - nchunk;
+            cp_async16((isg ? g_s : be_s) + cc * CH,
+                       reinterpret_cast<const T *>(isg ? p.head.gamma : p.head.beta) + cc * CH);
+        }
+        cp_async_commit();
+        for (int c = tid; c < kExitCT; c += kExitThreads) bias_s[c] = (c0 + c < C) ? p.head.bias[c0 + c] : 0.0f;
+        // padding rows 8..15 of the GEMM's A tile
+        for (int it = tid; it < 8 * nchunk; it += kExitThreads) {
+            const int r = 8 + it / nchunk, c = it % nchunk;
+            *reinterpret_cast<uint4 *>(u_s + (size_t)r * u_stride + c * CH) = make_uint4(0, 0, 0, 0);
+        }
+    }
+    cl.sync();   // every CTA of the cluster runs before any remote shared-memory store
+    if (active) {
+        cp_async_wait_all();
+        __syncthreads();
+        // the head's first two weight chunks load while the LayerNorm runs (issued only now:
+        // every CTA's 64 KB at once would hold up the CLS rows above)
+        issue_w_chunk<T>(p, w_region, c0, 0, dim, C, tid);
+        if (n_k > 1) issue_w_chunk<T>(p, w_region + S::w_stage, c0, KC, dim, C, tid);
+
+        // ---- LayerNorm, G warps per row: one pass of sum and sum of squares -----------
+        bool ok = has_row && s < B;
+        if (ok) {
+            const long long row = p.in.offsets[s];
+            if (row < 0 || row >= p.in.max_rows) {
+                if (gt == 0) raise_status(p.status, FUSION_DEV_BAD_OFFSETS);
+                ok = false;
+            }
+        }
+        const T *xr = x_s + (size_t)j * u_stride;
+        float s1 = 0.0f, c1 = 0.0f, s2 = 0.0f, c2 = 0.0f, l2 = 0.0f;
+        if (ok) {
+            for (int e = gt; e < dim; e += G * 32) {
+                const float v = to_float(xr[e]);
+                neu_add(s1, c1, v);
+                const F2 sq = two_prod(v, v);
+                neu_add(s2, c2, sq.hi);
+                l2 = __fadd_rn(l2, sq.lo);
+            }
+        }
+        F2 a1 = warp_sum_f2(two_sum(s1, c1));
+        F2 a2 = warp_sum_f2(f2_add_f(two_sum(s2, c2), l2));
+        if (lane == 0) {
+            red[warp * 8 + 0] = a1.hi;
+            red[warp * 8 + 1] = a1.lo;
+            red[warp * 8 + 2] = a2.hi;
+            red[warp * 8 + 3] = a2.lo;
+        }
+        __syncthreads();
+        if (ok) {
+            F2 t1 = {0.0f, 0.0f}, t2 = {0.0f, 0.0f};
+            for (int w = j * G; w < j * G + G; ++w) {   // the group's warps, in order
+                t1 = f2_add(t1, {red[w * 8 + 0], red[w * 8 + 1]});
+                t2 = f2_add(t2, {red[w * 8 + 2], red[w * 8 + 3]});
+            }
+            const F2 fdim = {(float)dim, 0.0f};
+            const F2 mean = f2_div(t1, fdim);
+            const F2 ex2 = f2_div(t2, fdim);
+            const F2 m2 = f2_mul(mean, mean);
+            F2 var = f2_add(ex2, {-m2.hi, -m2.lo});
+            if (var.hi < 0.0f) var = {0.0f, 0.0f};
+            const F2 rstd = f2_rsqrt(f2_add_f(var, p.head.eps));
+            if (gt == 0 && !(isfinite(mean.hi) && isfinite(var.hi))) raise_status(p.status, FUSION_DEV_NONFINITE);
+            for (int c = gt; c < nchunk; c += G * 32) {
+                float f[CH], gf[CH], bf[CH];
+                chunk_to_f(*reinterpret_cast<const uint4 *>(xr + c * CH), f);
+                chunk_to_f(*reinterpret_cast<const uint4 *>(g_s + c * CH), gf);
+                chunk_to_f(*reinterpret_cast<const uint4 *>(be_s + c * CH), bf);
+                uint4 outv;
+                if constexpr (kBf16) {
+                    uint32_t w4[4];
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        w4[q] = (uint32_t)ln_out_bf16(f[2 * q], mean, rstd, gf[2 * q], bf[2 * q]) |
+                                ((uint32_t)ln_out_bf16(f[2 * q + 1], mean, rstd, gf[2 * q + 1], bf[2 * q + 1]) << 16);
+                    outv = make_uint4(w4[0], w4[1], w4[2], w4[3]);
+                } else {
+                    outv = make_uint4(__float_as_uint(ln_out_f32(f[0], mean, rstd, gf[0], bf[0])),
+                                      __float_as_uint(ln_out_f32(f[1], mean, rstd, gf[1], bf[1])),
+                                      __float_as_uint(ln_out_f32(f[2], mean, rstd, gf[2], bf[2])),
+                                      __float_as_uint(ln_out_f32(f[3], mean, rstd, gf[3], bf[3])));
+                }
+                T *dst = u_s + (size_t)sl * u_stride + c * CH;
+                for (int r = 0; r < ncl; ++r) *reinterpret_cast<uint4 *>(cl.map_shared_rank(dst, r)) = outv;
+            }
+        } else if (has_row) {
+            for (int c = gt; c < nchunk; c += G * 32) {
+                T *dst = u_s + (size_t)sl * u_stride + c * CH;
+                for (int r = 0; r < ncl; ++r)
+                    *reinterpret_cast<uint4 *>(cl.map_shared_rank(dst, r)) = make_uint4(0, 0, 0, 0);
+            }
+        }
+    }
+    cl.sync();   // all LayerNorm rows are in every CTA's shared memory
+
+    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    float acc2[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    if (active) {
+        exit_gemm<T>(p, u_s, w_region, c0, dim, C, n_k, acc, acc2);
+        exit_logits<T>(p, lg_s, bias_s, acc, acc2, s0, c0, B, C);
+        // partial softmax of this class tile, warp -> sample slot; to the sample's owner
+        {
+            const int slw = warp, sw = s0 + slw;
+            float m = -INFINITY;
+            for (int col = lane; col < kExitCT; col += 32) m = fmaxf(m, lg_s[slw * kExitCT + col]);
+#pragma unroll
+            for (int o = 16; o >= 1; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+            float z = 0.0f;
+            for (int col = lane; col < kExitCT; col += 32) {
+                const float l = lg_s[slw * kExitCT + col];
+                if (l != -INFINITY) z += expf(l - m);
+            }
+#pragma unroll
+            for (int o = 16; o >= 1; o >>= 1) z += __shfl_xor_sync(0xFFFFFFFFu, z, o);
+            if (lane == 0 && sw < B) *cl.map_shared_rank(part_s + slw * 8 + rank, slw % ncl) = make_float2(m, z);
+        }
+    }
+    cl.sync();   // every partial is with its owner
+    if (active) {
+        const int slw = warp, sw = s0 + slw;
+        if (slw % ncl == rank && sw < B) {
+            float m = -INFINITY;
+            for (int q = lane; q < ncl; q += 32) m = fmaxf(m, part_s[slw * 8 + q].x);
+#pragma unroll
+            for (int o = 16; o >= 1; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+            float z = 0.0f;
+            for (int q = lane; q < ncl; q += 32) {
+                const float2 pz = part_s[slw * 8 + q];
+                z += pz.y * expf(pz.x - m);
+            }
+#pragma unroll
+            for (int o = 16; o >= 1; o >>= 1) z += __shfl_xor_sync(0xFFFFFFFFu, z, o);
+            if (lane == 0) {
+                const float c = 1.0f / z;   // max_k softmax = exp(l_max - l_max) / sum
+                p.exit_mask[sw] = (c >= p.head.tau) ? 1 : 0;
+                if (p.max_prob) p.max_prob[sw] = c;
+                if (!isfinite(m)) raise_status(p.status, FUSION_DEV_NONFINITE);
+            }
+        }
+    }
+    if (!p.do_plan) {
+        if (Bdev < 0 && bt == 0 && rank == 0 && tid == 0) raise_status(p.status, FUSION_DEV_BAD_BATCH);
+        return;
+    }
+    // ---- the last cluster to finish runs the plan (batches above the fused-plan bound) ----
+    __threadfence();
+    cl.sync();   // this cluster's exit masks are written
+    __shared__ int s_last;
+    if (tid == 0) {
+        s_last = 0;
+        if (rank == 0) {
+            __threadfence();
+            s_last = (atomicAdd(&p.counters[p.n_btile], 1) == p.n_btile - 1);
+        }
+    }
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    if (tid == 0) p.counters[p.n_btile] = 0;
+    run_plan(p.plan, reinterpret_cast<int *>(w_region));
+}
+
 }  // namespace
 
 size_t exit_smem_bytes(int dtype, int dim) {
     return dtype == FUSION_BF16 ? ExitSmem<__nv_bfloat16>::total(dim) : ExitSmem<float>::total(dim);
 }
 
+template <typename T>
+cudaError_t launch_exit_cluster(const ExitParams &p, cudaStream_t s) {
+    const size_t smem = ExitClSmem<T>::total(p.dim);
+    cudaError_t e = cudaFuncSetAttribute(k_exit_cl<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(p.n_ctile, p.n_btile);
+    cfg.blockDim = dim3(kExitThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = p.n_ctile;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k_exit_cl<T>, p);
+}
+
 cudaError_t launch_exit(int dtype, const ExitParams &p, cudaStream_t s) {
+    // the class tiles of a sample tile as one cluster (portable size: at most 8 tiles,
+    // 1024 classes); larger heads take the kernel with a global last-CTA merge
+    if (p.n_ctile <= 8 && p.n_btile > 0)
+        return dtype == FUSION_BF16 ? launch_exit_cluster<__nv_bfloat16>(p, s) : launch_exit_cluster<float>(p, s);
     const size_t smem = exit_smem_bytes(dtype, p.dim);
     const dim3 grid(p.n_ctile, p.n_btile);
     if (dtype == FUSION_BF16) {

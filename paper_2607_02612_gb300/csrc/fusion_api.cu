@@ -77,8 +77,15 @@ ProfileEvents take_profile() {
     return e;
 }
 
+// Under stream capture a plain record only orders the graph; an external record becomes a
+// node that records the event at every replay.
 void record(cudaEvent_t e, cudaStream_t s) {
-    if (e) cudaEventRecord(e, s);
+    if (!e) return;
+    cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(s, &st) == cudaSuccess && st == cudaStreamCaptureStatusActive)
+        cudaEventRecordWithFlags(e, s, cudaEventRecordExternal);
+    else
+        cudaEventRecord(e, s);
 }
 
 #define FZ_TRY(expr)                    \

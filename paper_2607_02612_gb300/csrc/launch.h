@@ -34,7 +34,7 @@ cudaError_t launch_plan(const PlanArgs &a, cudaStream_t s);
 // ---- per-sample merge / prune / gather -----------------------------------------
 // Batches of at most this many samples plan inside the per-sample kernel (every CTA
 // scans the batch), larger ones run the plan kernel first.
-constexpr int kFusedPlanMaxBatch = 1024;
+constexpr int kFusedPlanMaxBatch = FUSION_FUSED_PLAN_MAX_BATCH;
 
 struct ImageParams {
     Ragged in;

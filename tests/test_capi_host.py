@@ -144,3 +144,13 @@ def test_binding_refuses_host_tensors(lib):
 def test_missing_library_fails_loudly(tmp_path):
     with pytest.raises(fz.FusionError):
         fb.load(str(tmp_path / "libfusion.so"))
+
+
+def test_binding_constants_match_header():
+    """The Python mirrors of the header's #define values stay in step with it."""
+    with open(os.path.join(ROOT, "include", "fusion.h")) as f:
+        text = f.read()
+    defs = dict(re.findall(r"#define\s+(FUSION_[A-Z0-9_]+)\s+(-?\d+)", text))
+    for name in ("FUSION_MAX_TOKENS", "FUSION_MAX_DIM", "FUSION_FUSED_PLAN_MAX_BATCH", "FUSION_STAGE_MERGE",
+                 "FUSION_STAGE_EXIT", "FUSION_STAGE_PRUNE", "FUSION_DEV_TIMEOUT"):
+        assert int(defs[name]) == getattr(fb, name), name

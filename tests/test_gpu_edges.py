@@ -149,6 +149,20 @@ def test_all_or_no_samples_exit(tau):
     assert g["offsets"][0] == 0
 
 
+@pytest.mark.parametrize("dtype,classes", [("bf16", 1100), ("f32", 1100), ("bf16", 300), ("f32", 7)])
+def test_exit_check_head_sizes(dtype, classes):
+    """Heads of up to 8 class tiles run as one cluster per sample tile, larger ones (1100
+    classes: 9 tiles) on the kernel with a global last-CTA merge; both against the oracle."""
+    b = make_batch([9, 17, 33, 5, 12, 40, 7, 21, 3, 30], 64, dtype, seed=13)
+    r, rho = np.full(10, 3, np.int32), np.full(10, 0.6, np.float32)
+    # tau halfway between the 5th and 6th largest max-probability: half the samples exit
+    probe = oracle.stage(b, StageSpec(True, True, True, r=r, rho=rho, head=make_head(64, classes, dtype, 2.0, scale=0.5)))
+    mp = np.sort(probe["max_prob"])
+    spec = StageSpec(True, True, True, r=r, rho=rho, head=make_head(64, classes, dtype, float(mp[4] + mp[5]) / 2, scale=0.5))
+    g, o = run_stage_and_compare(b, spec, f"head {dtype} C={classes}")
+    assert int(g["batch"][0]) == 5
+
+
 def test_empty_batch_and_device_count():
     b = make_batch([5, 7, 9, 11], 32, "f32", seed=8)
     db = P.device_batch(b)

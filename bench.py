@@ -45,7 +45,6 @@ METRIC = "images/s per merge→exit→prune stage (DeiT-S, b256); % of HBM roofl
 UNIT = "images/s"
 DEFAULT_WORKLOAD = "deit_s_chain12_bf16_b256"
 FLUSH_BYTES = 512 << 20
-KERNELS_PER_STAGE = 2      # plan or exit check, then the per-sample kernel
 
 
 def parse_args():
@@ -360,8 +359,10 @@ def main():
         bytes_image += im
         units_step += len(in_off) - 1
         per_stage.append({"stage": s + 1, "images_in": len(in_off) - 1, "tokens_in": int(in_off[-1]),
-                          "ms": float(np.median(stage_ms[:, s])), "image_kernel_ms": float(np.median(image_ms[:, s])),
-                          "image_kernel_bytes": im})
+                          "ms": float(np.median(stage_ms[:, s])),
+                          "ms_p10_p90": [float(np.percentile(stage_ms[:, s], 10)), float(np.percentile(stage_ms[:, s], 90))],
+                          "image_kernel_ms": float(np.median(image_ms[:, s])),
+                          "image_kernel_bytes": im, "first_kernel_bytes": f1})
         in_off, in_ids = out_off, out_ids
 
     step_ms = stage_ms.sum(axis=1)
@@ -380,6 +381,17 @@ def main():
     achieved = bytes_image * args.steps / img_s / 1e9
     step_achieved = (bytes_first + bytes_image) * args.steps / (float(stage_ms.sum()) / 1e3) / 1e9
     tr = recorded_traffic(args.workload)
+    # the full stages (exit check -> compaction -> prune, blocks 4/6/8/10): images/s and the
+    # fraction of the HBM roofline over all their kernels, per the measurement contract
+    full = [s for s in range(S) if specs[s].exit]
+    full_stats = None
+    if full:
+        t_full = float(stage_ms[:, full].sum()) / 1e3
+        b_full = sum(per_stage[s]["first_kernel_bytes"] + per_stage[s]["image_kernel_bytes"] for s in full) * args.steps
+        full_stats = {"stages": [s + 1 for s in full],
+                      "images_per_s": sum(per_stage[s]["images_in"] for s in full) * args.steps / t_full,
+                      "achieved_gbs": b_full / t_full / 1e9, "frac": b_full / t_full / 1e9 / peak}
+    solo = run_solo_full_stage(args, fz, runner, w, b, dev, flush, peak) if full else None
 
     # ---- end to end through the C ABI with host buffers -------------------------------
     e2e = run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world)
@@ -400,8 +412,10 @@ def main():
                      "whole_step_frac": step_achieved / peak},
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": KERNELS_PER_STAGE * S * args.steps,
+        "gpu_launches": sum(1 + int(has_first[s]) for s in range(S)) * args.steps,
         "clocks": clocks,
+        "full_stages": full_stats,
+        "solo_full_stage": solo,
         "stages": per_stage,
         "kernel_ms_per_step": {"first (exit check or plan)": float(first_ms.sum(axis=1).mean()),
                                "k_image": float(image_ms.sum(axis=1).mean())},
@@ -414,6 +428,54 @@ def main():
         import torch.distributed as dist
         dist.destroy_process_group()
     return 0
+
+
+def run_solo_full_stage(args, fz, runner, w, b, dev, flush, peak):
+    """One full stage (merge -> exit check -> compaction -> prune) on the N = 197 input batch with
+    the first full stage's router outputs and head: the stand-alone stage beside the schedule."""
+    import torch
+    spec = next(s for s in w.stages if s.exit)
+    r = torch.from_numpy(spec.r).to(dev)
+    rho = torch.from_numpy(spec.rho).to(dev)
+    head = runner.head_tensors(spec.head, b.dtype, dev)
+    flags = fz.FUSION_STAGE_MERGE | fz.FUSION_STAGE_EXIT | fz.FUSION_STAGE_PRUNE
+    fus = runner.Fusion(b.batch, spec.head.classes, dev)
+    db = runner.device_batch(b.dtype, b.offsets, b.x, b.keys, b.sizes, b.scores, device=dev)
+    ch = runner.Chain(fus, db, [runner.ChainStage(flags, r, rho, head)])
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    for e in ev:
+        e.record()
+
+    def one():
+        flush.fill_(7)
+        fz.fusion_profile_next(ev[0], None, ev[1])
+        ch.run_stage(0)
+
+    one()
+    torch.cuda.synchronize()
+    g = None
+    if not args.eager:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            one()
+    run = g.replay if g is not None else one
+    for _ in range(args.warmup):
+        run()
+    ms = []
+    for _ in range(args.steps):
+        run()
+        torch.cuda.synchronize()
+        ms.append(ev[0].elapsed_time(ev[1]))
+    o = ch.outs[0]
+    nb = int(o["batch"].item())
+    out_off = o["offsets"][:nb + 1].cpu().numpy()
+    out_ids = o["ids"][:nb].cpu().numpy()
+    f1, im = stage_bytes(spec, b.dtype, b.dim, b.offsets, np.arange(b.batch, dtype=np.int32), out_off, out_ids,
+                         spec.head.classes)
+    t = float(np.median(ms)) / 1e3
+    return {"batch": b.batch, "tokens": int(np.diff(b.offsets).max()), "ms": t * 1e3,
+            "ms_p10_p90": [float(np.percentile(ms, 10)), float(np.percentile(ms, 90))],
+            "images_per_s": b.batch / t, "achieved_gbs": (f1 + im) / t / 1e9, "frac": (f1 + im) / t / 1e9 / peak}
 
 
 def run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world):

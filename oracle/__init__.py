@@ -48,6 +48,8 @@ def configure(lib):
     lib.orc_exit.argtypes = [i32, i32, P, i32, P, P, P, dbl, P, P, i32, dbl, P, P, P, P, P]
     lib.orc_prune.argtypes = [i32, i32, P, i32, P, P, P, P, P, P, P, P, P, P]
     lib.orc_compact.argtypes = [i32, i32, P, i32, P, P, P, P, P, P, P, P, P, P, P, P]
+    lib.orc_merge_router.argtypes = [i32, i32, P, P, i32, P, P, dbl, dbl, dbl, P, P, P]
+    lib.orc_merge_router.restype = ctypes.c_int
     lib.orc_double_to_bf16.argtypes = [dbl]
     lib.orc_double_to_bf16.restype = ctypes.c_uint16
     lib.orc_bf16_to_double.argtypes = [ctypes.c_uint16]
@@ -151,6 +153,31 @@ def exit_check(dtype: str, offsets, x, head) -> Dict[str, np.ndarray]:
                       _p(mask), _p(logits), _p(maxp), _p(gap), _p(u))
     _check(rc, "exit")
     return dict(exit_mask=mask, logits=logits, max_prob=maxp, exit_gap=gap, u=u)
+
+
+def merge_router(dtype: str, offsets, x, w, beta: float, tau_tgt: float, tau_ref: float, ids=None,
+                 n_ids: Optional[int] = None) -> Dict[str, np.ndarray]:
+    """Sec. III-C router with profile scaling (Eq. 4-5) on the CLS row of every sample:
+    r = floor(clamp(sigmoid(w . z_CLS + beta) (1 - tau_tgt) / (1 - tau_ref), 0, 1) N / 2).
+    The arguments beta, tau_tgt, tau_ref are taken as float32 values (the library's
+    argument type).  Returns r (int32), mt (the scaled ratio) and r_gap (margin of the
+    floor decision), each indexed by original sample id (ids, or the position)."""
+    lib = _load()
+    et = _elem_dtype(dtype)
+    offsets = _c(offsets, np.int32)
+    x = _c(x, et)
+    B = len(offsets) - 1
+    d = x.shape[1]
+    ids_a = None if ids is None else _c(ids, np.int32)
+    n = n_ids if n_ids is not None else (int(ids_a.max()) + 1 if ids_a is not None and B > 0 else B)
+    r = np.zeros(n, np.int32)
+    mt = np.zeros(n, np.float64)
+    gap = np.full(n, np.inf)
+    rc = lib.orc_merge_router(_DT[dtype], B, _p(offsets), _p(ids_a), d, _p(x), _p(_c(w, et)),
+                              float(np.float32(beta)), float(np.float32(tau_tgt)), float(np.float32(tau_ref)),
+                              _p(r), _p(mt), _p(gap))
+    _check(rc, "merge_router")
+    return dict(r=r, mt=mt, r_gap=gap)
 
 
 def prune(dtype: str, offsets, x, sizes, scores, rho) -> Dict[str, np.ndarray]:

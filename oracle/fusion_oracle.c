@@ -21,6 +21,10 @@
  *           tokens by score (CLS-attention scores supplied as input).
  *   compact Drop the exited samples (Algorithm 1 returns early for them) and pack
  *           the survivors into a ragged, offset-indexed batch.
+ *   router  Sec. III-C, Eq. 4 and Eq. 5 (the merge count's source, upstream of
+ *           merge): m = sigmoid(w . z_CLS + beta), scaled by the profile ratio
+ *           (1 - tau_tgt) / (1 - tau_ref), clamped to [0, 1]; r = floor(m N / 2)
+ *           with N the sample's current token count.
  *
  * Readings of points the paper leaves open (fixed here, mirrored by the CUDA path):
  *   - positions within a sample: 0 is CLS, 1..P are patches; half B holds the odd
@@ -459,5 +463,50 @@ int orc_compact(int dtype, int B, const int32_t *offsets, int d, const void *x,
         ++j;
     }
     *n_out = j;
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------------------- */
+/* merge router with profile scaling (Sec. III-C, Eq. 4 and Eq. 5)             */
+/* ------------------------------------------------------------------------- */
+/*
+ * For every sample i (rows offsets[i]..offsets[i+1]-1, CLS first):
+ *   m_i  = sigmoid(w . z_i + beta)                          (Eq. 4, z_i the CLS row)
+ *   mt_i = m_i * (1 - tau_tgt) / (1 - tau_ref), clamped to [0, 1]   (Eq. 5)
+ *   r_i  = floor(mt_i * N_i / 2), N_i the sample's token count, CLS included
+ * Outputs are indexed by the sample's original id (ids[i], or i when ids is NULL):
+ * r_out, mt_out (may be NULL) and r_gap (may be NULL) = distance of mt_i N_i / 2 to
+ * the nearest integer, the margin of the floor decision.  tau_ref must be below 1.
+ */
+int orc_merge_router(int dtype, int B, const int32_t *offsets, const int32_t *ids, int d, const void *x,
+                     const void *w, double beta, double tau_tgt, double tau_ref, int32_t *r_out,
+                     double *mt_out, double *r_gap)
+{
+    if (B < 0 || d <= 0 || !(tau_ref < 1.0))
+        return ORC_ERR_ARG;
+    const double scale = (1.0 - tau_tgt) / (1.0 - tau_ref);
+    for (int i = 0; i < B; ++i) {
+        const int64_t row = offsets[i];
+        const int N = offsets[i + 1] - offsets[i];
+        double z = 0.0;
+        for (int j = 0; j < d; ++j)
+            z += load_elem(dtype, w, j) * load_elem(dtype, x, row * d + j);
+        const double m = 1.0 / (1.0 + exp(-(z + beta)));
+        double mt = m * scale;
+        if (mt < 0.0)
+            mt = 0.0;
+        if (mt > 1.0)
+            mt = 1.0;
+        const double v = mt * (0.5 * (double)N);
+        const double r = floor(v);
+        const int id = ids ? ids[i] : i;
+        r_out[id] = (int32_t)r;
+        if (mt_out)
+            mt_out[id] = mt;
+        if (r_gap) {
+            const double f = v - r;
+            r_gap[id] = f < 1.0 - f ? f : 1.0 - f;
+        }
+    }
     return ORC_OK;
 }

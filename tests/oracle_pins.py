@@ -505,6 +505,62 @@ def pin_stage_composition():
     np.testing.assert_array_equal(res["x"][untouched], b.x[res["keep_idx"][untouched]])
 
 
+# ---------------------------------------------------------------------------
+# merge router with profile scaling (Sec. III-C, Eq. 4-5)
+# ---------------------------------------------------------------------------
+def _router_batch(cls, Ns):
+    """One sample per N, each with `cls` as its CLS row and zero patch rows."""
+    d = len(cls)
+    offs = np.concatenate([[0], np.cumsum(Ns)]).astype(np.int32)
+    x = np.zeros((int(offs[-1]), d), np.float32)
+    x[offs[:-1]] = np.asarray(cls, np.float32)
+    return offs, x
+
+
+def pin_router_worked_examples():
+    for ex in _golden()["router"]:
+        Ns = [c["N"] for c in ex["cases"]]
+        offs, x = _router_batch(ex["cls"], Ns)
+        o = oracle.merge_router("f32", offs, x, np.array(ex["w"], np.float32), ex["beta"], ex["tau_tgt"], ex["tau_ref"])
+        np.testing.assert_array_equal(o["r"], [c["r"] for c in ex["cases"]], err_msg=ex["name"])
+        assert np.all(np.abs(o["mt"] - ex["mt"]) < 1e-7), (ex["name"], o["mt"])
+
+
+def pin_router_special_cases():
+    Ns = [1, 2, 3, 8, 65, 197, 577]
+    offs, x = _router_batch([0.7, -1.3, 2.0], Ns)
+    w0 = np.zeros(3, np.float32)
+    # w = 0, beta = 0, equal profiles: mt = 1/2, r = floor(N / 4)
+    o = oracle.merge_router("f32", offs, x, w0, 0.0, 0.3, 0.3)
+    np.testing.assert_array_equal(o["r"], [N // 4 for N in Ns])
+    # a saturated sigmoid merges every pair (floor(N / 2)) or none
+    o = oracle.merge_router("f32", offs, x, w0, 60.0, 0.3, 0.3)
+    np.testing.assert_array_equal(o["r"], [N // 2 for N in Ns])
+    o = oracle.merge_router("f32", offs, x, w0, -60.0, 0.3, 0.3)
+    np.testing.assert_array_equal(o["r"], [0] * len(Ns))
+    # r grows with beta and with the profile's merge budget (lower target keep ratio)
+    w = np.array([0.3, 0.1, -0.2], np.float32)
+    prev = None
+    for beta in np.linspace(-6, 6, 25):
+        r = oracle.merge_router("f32", offs, x, w, float(beta), 0.5, 0.5)["r"]
+        assert prev is None or np.all(r >= prev), beta
+        prev = r
+    prev = None
+    for tt in np.linspace(1.0, 0.0, 11):
+        r = oracle.merge_router("f32", offs, x, w, 0.5, float(tt), 0.4)["r"]
+        assert prev is None or np.all(r >= prev), tt
+        prev = r
+    # bf16 inputs: values exactly representable in bf16 give the same counts as float32
+    xb, wb = f32_to_bf16_bits(x), f32_to_bf16_bits(w)
+    np.testing.assert_array_equal(oracle.merge_router("bf16", offs, xb, wb, 0.5, 0.25, 0.4)["r"],
+                                  oracle.merge_router("f32", offs, x, w, 0.5, 0.25, 0.4)["r"])
+    # outputs land at the original sample id
+    ids = np.array([6, 0, 5, 1, 4, 2, 3], np.int32)
+    o1 = oracle.merge_router("f32", offs, x, w, 0.5, 0.25, 0.4)
+    o2 = oracle.merge_router("f32", offs, x, w, 0.5, 0.25, 0.4, ids=ids)
+    np.testing.assert_array_equal(o2["r"][ids], o1["r"])
+
+
 ALL_PINS = [
     pin_bf16_rounding_table,
     pin_bf16_rounding_vs_torch,
@@ -522,4 +578,6 @@ ALL_PINS = [
     pin_compact_examples,
     pin_stage_exit_sees_merged_cls,
     pin_stage_composition,
+    pin_router_worked_examples,
+    pin_router_special_cases,
 ]

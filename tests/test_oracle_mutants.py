@@ -36,6 +36,13 @@ MUTANTS = {
     "prune_floor": ("double kk = ceil((double)rho[i] * (double)P);", "double kk = floor((double)rho[i] * (double)P);"),
     "prune_drops_cls": ("if (p > 0 && !kept[p - 1])", "if (p == 0 || !kept[p - 1])"),
     "compact_keeps_exited": ("if (exit_mask[i])\n            continue;", "if (0)\n            continue;"),
+    "router_no_profile_scale": ("double mt = m * scale;", "double mt = m;"),
+    "router_ceil": ("const double r = floor(v);", "const double r = ceil(v);"),
+    "router_sigmoid_sign": ("exp(-(z + beta))", "exp(z + beta)"),
+    "router_drops_beta": ("exp(-(z + beta))", "exp(-z)"),
+    "router_patch_count": ("mt * (0.5 * (double)N)", "mt * (0.5 * (double)(N - 1))"),
+    "router_no_clamp": ("if (mt > 1.0)\n            mt = 1.0;", "if (0)\n            mt = 1.0;"),
+    "router_scale_inverted": ("(1.0 - tau_tgt) / (1.0 - tau_ref)", "(1.0 - tau_ref) / (1.0 - tau_tgt)"),
 }
 
 

@@ -392,6 +392,7 @@ def main():
                       "images_per_s": sum(per_stage[s]["images_in"] for s in full) * args.steps / t_full,
                       "achieved_gbs": b_full / t_full / 1e9, "frac": b_full / t_full / 1e9 / peak}
     solo = run_solo_full_stage(args, fz, runner, w, b, dev, flush, peak) if full else None
+    router = run_router(args, fz, runner, b, dev, flush, peak)
 
     # ---- end to end through the C ABI with host buffers -------------------------------
     e2e = run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world)
@@ -416,6 +417,7 @@ def main():
         "clocks": clocks,
         "full_stages": full_stats,
         "solo_full_stage": solo,
+        "router": router,
         "stages": per_stage,
         "kernel_ms_per_step": {"first (exit check or plan)": float(first_ms.sum(axis=1).mean()),
                                "k_image": float(image_ms.sum(axis=1).mean())},
@@ -476,6 +478,48 @@ def run_solo_full_stage(args, fz, runner, w, b, dev, flush, peak):
     return {"batch": b.batch, "tokens": int(np.diff(b.offsets).max()), "ms": t * 1e3,
             "ms_p10_p90": [float(np.percentile(ms, 10)), float(np.percentile(ms, 90))],
             "images_per_s": b.batch / t, "achieved_gbs": (f1 + im) / t / 1e9, "frac": (f1 + im) / t / 1e9 / peak}
+
+
+def run_router(args, fz, runner, b, dev, flush, peak):
+    """The merge router with profile scaling (Eq. 4-5) on the step's input batch: one
+    dot product per CLS row; bytes = CLS rows + router weight + offsets/ids + r and mt."""
+    import torch
+    from workloads import make_router
+    rs = make_router(np.random.default_rng(2607), b.dim, b.dtype)
+    wt = torch.from_numpy(rs.w.view(np.int16).copy() if b.dtype == "bf16" else rs.w.copy()).to(dev)
+    fus = runner.Fusion(b.batch, 1, dev)
+    db = runner.device_batch(b.dtype, b.offsets, b.x, b.keys, b.sizes, b.scores, device=dev)
+    out = dict(r=torch.zeros(b.batch, dtype=torch.int32, device=dev), m=torch.zeros(b.batch, device=dev))
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    for e in ev:
+        e.record()
+
+    def one():
+        flush.fill_(3)
+        fz.fusion_profile_next(ev[0], None, ev[1])
+        fus.merge_router(db, wt, rs.beta, rs.tau_tgt, rs.tau_ref, out=out)
+
+    one()
+    torch.cuda.synchronize()
+    g = None
+    if not args.eager:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            one()
+    run = g.replay if g is not None else one
+    for _ in range(args.warmup):
+        run()
+    ms = []
+    for _ in range(args.steps):
+        run()
+        torch.cuda.synchronize()
+        ms.append(ev[0].elapsed_time(ev[1]))
+    eb = 2 if b.dtype == "bf16" else 4
+    nbytes = b.batch * (b.dim * eb + 8 + 8) + b.dim * eb
+    t = float(np.median(ms)) / 1e3
+    return {"batch": b.batch, "ms": t * 1e3, "images_per_s": b.batch / t, "algorithmic_bytes": nbytes,
+            "achieved_gbs": nbytes / t / 1e9, "frac": nbytes / t / 1e9 / peak,
+            "note": "one CLS dot product per image in double: launch- and latency-bound by design"}
 
 
 def run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world):

@@ -237,6 +237,28 @@ int fusion_compact(int dtype, fusion_ragged in, const void *x, int32_t dim, cons
                    int32_t *dev_status, void *stream);
 
 /*
+ * fusion_merge_router: the per-sample merge counts from the merge router with
+ * profile scaling (Sec. III-C, Eq. 4 and Eq. 5), the input r of fusion_merge and
+ * fusion_stage:
+ *   m_i  = sigmoid(w . z_i + beta), z_i the CLS row of sample i          (Eq. 4)
+ *   mt_i = m_i (1 - tau_tgt) / (1 - tau_ref), clamped to [0, 1]          (Eq. 5)
+ *   r_i  = floor(mt_i N_i / 2), N_i the sample's token count, CLS included
+ * (the merge then clamps r_i to |A|).  tau_tgt is the target keep ratio of the
+ * operating profile, tau_ref that of the reference profile the router was
+ * trained at.  Evaluated in double, so r_i differs from an exact evaluation only
+ * when mt_i N_i / 2 lies within about 1e-15 of an integer.
+ * w: [dim] device, the tokens' dtype.  Outputs by original id (in.ids, or the
+ * position): r_out [max_batch] int32, m_out [max_batch] float (mt_i; may be
+ * NULL).  Samples beyond the device batch count are not written.
+ * Errors: FUSION_ERR_INVALID_ARG for NULL pointers or tau_ref >= 1 or a
+ * non-finite beta / tau; device bits BAD_BATCH, BAD_OFFSETS, BAD_IDS, NONFINITE
+ * (that sample's r is 0).  No workspace.
+ */
+int fusion_merge_router(int dtype, fusion_ragged in, const void *x, int32_t dim, const void *w,
+                        float beta, float tau_tgt, float tau_ref, int32_t *r_out, float *m_out,
+                        int32_t *dev_status, void *stream);
+
+/*
  * fusion_stage: one block's whole adaptation stage, fused (Algorithm 1 body):
  * merge (FUSION_STAGE_MERGE) -> exit check (FUSION_STAGE_EXIT; exited samples
  * leave the batch) -> prune (FUSION_STAGE_PRUNE) -> compacted output.  The

@@ -40,7 +40,7 @@ FUSION_MAX_DIM = 1024
 
 EXPORTED = ("fusion_status_string", "fusion_version", "fusion_profile_next", "fusion_workspace_size",
             "fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune", "fusion_compact",
-            "fusion_stage")
+            "fusion_stage", "fusion_merge_router")
 
 
 class FusionError(RuntimeError):
@@ -94,8 +94,10 @@ def load(path: Optional[str] = None):
     lib.fusion_compact.argtypes = [ctypes.c_int, R, V, I32, V, V, V, V, V, V, V, V, V, V, V, SZ, V, V]
     lib.fusion_stage.argtypes = [ctypes.c_int, ctypes.c_int, R, V, I32, V, I32, V, V, V, V, H, V, V, V,
                                  V, V, V, V, V, V, V, V, V, SZ, V, V]
+    lib.fusion_merge_router.argtypes = [ctypes.c_int, R, V, I32, V, ctypes.c_float, ctypes.c_float, ctypes.c_float,
+                                        V, V, V, V]
     for name in ("fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune",
-                 "fusion_compact", "fusion_stage"):
+                 "fusion_compact", "fusion_stage", "fusion_merge_router"):
         getattr(lib, name).restype = ctypes.c_int
     del I64, F
     if path is None:
@@ -190,6 +192,13 @@ def fusion_exit_check_noalloc(dtype, in_, x, dim, head, exit_mask, logits, max_p
     """fusion_exit_check with the library's built-in scratch (for callers that cannot allocate)."""
     return load().fusion_exit_check_noalloc(int(dtype), in_, _ptr(x), int(dim), head, _ptr(exit_mask),
                                             _ptr(logits), _ptr(max_prob), _ptr(dev_status), _stream(stream))
+
+
+def fusion_merge_router(dtype, in_, x, dim, w, beta, tau_tgt, tau_ref, r_out, m_out, dev_status,
+                        stream=None) -> int:
+    """Merge counts from the router with profile scaling (Sec. III-C, Eq. 4-5), by original id."""
+    return load().fusion_merge_router(int(dtype), in_, _ptr(x), int(dim), _ptr(w), float(beta), float(tau_tgt),
+                                      float(tau_ref), _ptr(r_out), _ptr(m_out), _ptr(dev_status), _stream(stream))
 
 
 def fusion_prune(dtype, in_, x, dim, sizes, scores, rho, x_out, sizes_out, scores_out, offsets_out,

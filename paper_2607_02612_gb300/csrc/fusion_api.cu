@@ -3,6 +3,8 @@
 // check fails.
 #include <stdint.h>
 
+#include <cmath>
+
 #include "launch.h"
 
 using namespace fz;
@@ -326,6 +328,35 @@ int fusion_compact(int dtype, fusion_ragged in, const void *x, int32_t dim, cons
     p.fused_plan = fuse_plan(in);
     p.plan_args = pa;
     const int rc = cuda_rc(launch_sample_kernel(dtype, p, G, s));
+    record(ev.end, s);
+    return rc;
+}
+
+int fusion_merge_router(int dtype, fusion_ragged in, const void *x, int32_t dim, const void *w,
+                        float beta, float tau_tgt, float tau_ref, int32_t *r_out, float *m_out,
+                        int32_t *dev_status, void *stream) {
+    FZ_TRY(check_dtype(dtype));
+    FZ_TRY(check_ragged(in));
+    FZ_TRY(check_dim(dim));
+    if (!x || !w || !r_out) return FUSION_ERR_INVALID_ARG;
+    if (!std::isfinite(beta) || !std::isfinite(tau_tgt) || !std::isfinite(tau_ref) || !(tau_ref < 1.0f))
+        return FUSION_ERR_INVALID_ARG;
+    RouterParams p{};
+    p.in = dev(in);
+    p.x = x;
+    p.dim = dim;
+    p.w = w;
+    p.beta = beta;
+    p.tau_tgt = tau_tgt;
+    p.tau_ref = tau_ref;
+    p.r_out = r_out;
+    p.m_out = m_out;
+    p.status = dev_status;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const ProfileEvents ev = take_profile();
+    record(ev.start, s);
+    record(ev.mid, s);
+    const int rc = cuda_rc(launch_router(dtype, p, s));
     record(ev.end, s);
     return rc;
 }

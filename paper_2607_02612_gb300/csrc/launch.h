@@ -28,6 +28,19 @@ struct ExitParams {
 cudaError_t launch_exit(int dtype, const ExitParams &p, cudaStream_t s);
 size_t exit_smem_bytes(int dtype, int dim);
 
+// ---- merge router with profile scaling ----------------------------------------------
+struct RouterParams {
+    Ragged in;
+    const void *x;
+    int dim;
+    const void *w;    // router weight [dim], the tokens' dtype
+    float beta, tau_tgt, tau_ref;
+    int *r_out;       // [max_batch] merge counts by original id
+    float *m_out;     // [max_batch] scaled merge ratios by original id, or NULL
+    int *status;
+};
+cudaError_t launch_router(int dtype, const RouterParams &p, cudaStream_t s);
+
 // ---- stand-alone plan ----------------------------------------------------------
 cudaError_t launch_plan(const PlanArgs &a, cudaStream_t s);
 

@@ -124,6 +124,16 @@ class Fusion:
                                  o["dst_map"], o["a_match"], self.workspace, self.ws_bytes, self.status))
         return o
 
+    def merge_router(self, b: DeviceBatch, w: torch.Tensor, beta: float, tau_tgt: float, tau_ref: float,
+                     out: Optional[Dict[str, torch.Tensor]] = None) -> Dict[str, torch.Tensor]:
+        """Merge counts r (by original id) from the router with profile scaling (Eq. 4-5)."""
+        o = out if out is not None else dict(
+            r=torch.zeros(b.max_batch, dtype=torch.int32, device=self.device),
+            m=torch.zeros(b.max_batch, dtype=torch.float32, device=self.device))
+        fb.check(fb.fusion_merge_router(DTYPE_CODE[b.dtype], b.ragged(), b.x, b.dim, w, beta, tau_tgt, tau_ref,
+                                        o["r"], o["m"], self.status))
+        return o
+
     def exit_check(self, b: DeviceBatch, head: HeadTensors) -> Dict[str, torch.Tensor]:
         dev = self.device
         o = dict(exit_mask=torch.zeros(b.max_batch, dtype=torch.uint8, device=dev),

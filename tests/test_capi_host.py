@@ -154,3 +154,17 @@ def test_binding_constants_match_header():
     for name in ("FUSION_MAX_TOKENS", "FUSION_MAX_DIM", "FUSION_FUSED_PLAN_MAX_BATCH", "FUSION_STAGE_MERGE",
                  "FUSION_STAGE_EXIT", "FUSION_STAGE_PRUNE", "FUSION_DEV_TIMEOUT"):
         assert int(defs[name]) == getattr(fb, name), name
+
+
+def test_merge_router_rejects_bad_arguments(lib):
+    def call(**kw):
+        args = dict(dtype=fz.FUSION_BF16, in_=_r(), x=FAKE, dim=384, w=FAKE, beta=0.0, tau_tgt=0.5, tau_ref=0.3,
+                    r_out=FAKE, m_out=None, dev_status=FAKE, stream=0)
+        args.update(kw)
+        return fz.fusion_merge_router(*args.values())
+    assert call(dtype=3) == fz.FUSION_ERR_DTYPE
+    assert call(dim=20) == fz.FUSION_ERR_SHAPE
+    assert call(in_=_r(offsets=None)) == fz.FUSION_ERR_INVALID_ARG
+    for kw in (dict(x=None), dict(w=None), dict(r_out=None), dict(tau_ref=1.0), dict(tau_ref=1.5),
+               dict(beta=float("nan")), dict(tau_tgt=float("inf"))):
+        assert call(**kw) == fz.FUSION_ERR_INVALID_ARG, kw

@@ -8,9 +8,11 @@ from .synth import (  # noqa: F401
     CONFIGS,
     Batch,
     Head,
+    RouterSpec,
     StageSpec,
     Workload,
     bf16_bits_to_f32,
     f32_to_bf16_bits,
+    make_router,
     make_workload,
 )

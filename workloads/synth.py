@@ -230,6 +230,25 @@ def make_head(rng: np.random.Generator, classes: int, dim: int, tau: float, alph
                 tau=float(tau))
 
 
+@dataclass
+class RouterSpec:
+    """Merge-router parameters (Sec. III-C, Eq. 4-5): weight w [dim] (the tokens' dtype),
+    bias beta, target keep ratio tau_tgt of the operating profile and tau_ref of the
+    reference profile."""
+    w: np.ndarray
+    beta: float
+    tau_tgt: float
+    tau_ref: float
+
+
+def make_router(rng: np.random.Generator, dim: int, dtype: str, tau_tgt: float = 0.5,
+                tau_ref: float = 0.3) -> RouterSpec:
+    """Random router weights with w . z of unit scale for unit-variance CLS rows (no trained
+    router exists here): w ~ N(0, 1/dim), beta ~ N(0, 0.25^2)."""
+    w = (rng.standard_normal(dim) / np.sqrt(dim)).astype(np.float32)
+    return RouterSpec(_round(w, dtype), float(np.float32(rng.normal(0.0, 0.25))), tau_tgt, tau_ref)
+
+
 def ragged_counts_from_sizes(rng: np.random.Generator, batch: int, max_tokens: int):
     """Ragged variant of the non-uniform-size config: draw patch sizes uniform in {1..4}
     until the next one would push the image's total (CLS included) past max_tokens."""

@@ -61,6 +61,20 @@ def parse_args():
     return ap.parse_args()
 
 
+def reduce_over_ranks(time_value, units, world, device):
+    """The job's time is the slowest rank's and its work the sum of all ranks' (each rank runs
+    its own shard of images; no data crosses ranks)."""
+    if world <= 1:
+        return float(time_value), float(units)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(time_value)], dtype=torch.float64, device=device)
+    u = torch.tensor([float(units)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(u.item())
+
+
 def dist_env():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -368,13 +382,7 @@ def main():
     step_ms = stage_ms.sum(axis=1)
     total_ms = float(step_ms.sum())
     units = units_step * args.steps
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([total_ms], device=dev)
-        u = torch.tensor([float(units)], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        dist.all_reduce(u, op=dist.ReduceOp.SUM)
-        total_ms, units = float(t.item()), float(u.item())
+    total_ms, units = reduce_over_ranks(total_ms, units, world, dev)
     value = units / (total_ms / 1e3)
     peak, peak_src = peaks()
     img_s = float(image_ms.sum()) / 1e3
@@ -563,12 +571,8 @@ def run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world):
     torch.cuda.synchronize()
     dt = time.perf_counter() - t0
     barrier()
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([dt], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        dt = float(t.item())
-    return {"value": units_step * steps * world / dt, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+    dt, units = reduce_over_ranks(dt, units_step * steps, world, dev)
+    return {"value": units / dt, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h_bytes[-1]), "steps": steps,
             "note": "pinned host inputs, C-ABI chain (no L2 flush), host reads the survivor count then the results"}
 

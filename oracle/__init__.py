@@ -50,6 +50,8 @@ def configure(lib):
     lib.orc_compact.argtypes = [i32, i32, P, i32, P, P, P, P, P, P, P, P, P, P, P, P]
     lib.orc_merge_router.argtypes = [i32, i32, P, P, i32, P, P, dbl, dbl, dbl, P, P, P]
     lib.orc_merge_router.restype = ctypes.c_int
+    lib.orc_token_scores.argtypes = [i32, i32, P, i32, P, P, dbl, P]
+    lib.orc_token_scores.restype = ctypes.c_int
     lib.orc_double_to_bf16.argtypes = [dbl]
     lib.orc_double_to_bf16.restype = ctypes.c_uint16
     lib.orc_bf16_to_double.argtypes = [ctypes.c_uint16]
@@ -178,6 +180,20 @@ def merge_router(dtype: str, offsets, x, w, beta: float, tau_tgt: float, tau_ref
                               _p(r), _p(mt), _p(gap))
     _check(rc, "merge_router")
     return dict(r=r, mt=mt, r_gap=gap)
+
+
+def token_scores(dtype: str, offsets, x, w, b: float) -> np.ndarray:
+    """Sec. III-E, Eq. 8 pruning router with a linear scoring head: s = w . z + b for every
+    token row of the batch (double, rounded once to float32; b taken as a float32 value)."""
+    lib = _load()
+    et = _elem_dtype(dtype)
+    offsets = _c(offsets, np.int32)
+    x = _c(x, et)
+    B = len(offsets) - 1
+    out = np.zeros(x.shape[0], np.float32)
+    _check(lib.orc_token_scores(_DT[dtype], B, _p(offsets), x.shape[1], _p(x), _p(_c(w, et)),
+                                float(np.float32(b)), _p(out)), "token_scores")
+    return out
 
 
 def prune(dtype: str, offsets, x, sizes, scores, rho) -> Dict[str, np.ndarray]:

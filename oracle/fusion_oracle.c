@@ -21,6 +21,9 @@
  *           tokens by score (CLS-attention scores supplied as input).
  *   compact Drop the exited samples (Algorithm 1 returns early for them) and pack
  *           the survivors into a ragged, offset-indexed batch.
+ *   scores  Sec. III-E, Eq. 8 (the prune scores' source): s_i = h_b(z_i) with a
+ *           linear scoring head, s = w . z + b for every token, rounded once to
+ *           float32.
  *   router  Sec. III-C, Eq. 4 and Eq. 5 (the merge count's source, upstream of
  *           merge): m = sigmoid(w . z_CLS + beta), scaled by the profile ratio
  *           (1 - tau_tgt) / (1 - tau_ref), clamped to [0, 1]; r = floor(m N / 2)
@@ -508,5 +511,28 @@ int orc_merge_router(int dtype, int B, const int32_t *offsets, const int32_t *id
             r_gap[id] = f < 1.0 - f ? f : 1.0 - f;
         }
     }
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------------------- */
+/* pruning router: token scores (Sec. III-E, Eq. 8)                             */
+/* ------------------------------------------------------------------------- */
+/*
+ * s_t = w . z_t + b for every token row t of the B samples (rows offsets[0] ..
+ * offsets[B] - 1), accumulated in double and rounded once to float32.  Rows outside
+ * the samples are not written.
+ */
+int orc_token_scores(int dtype, int B, const int32_t *offsets, int d, const void *x, const void *w, double b,
+                     float *scores_out)
+{
+    if (B < 0 || d <= 0)
+        return ORC_ERR_ARG;
+    for (int i = 0; i < B; ++i)
+        for (int64_t t = offsets[i]; t < offsets[i + 1]; ++t) {
+            double acc = 0.0;
+            for (int j = 0; j < d; ++j)
+                acc += load_elem(dtype, w, j) * load_elem(dtype, x, t * d + j);
+            scores_out[t] = (float)(acc + b);
+        }
     return ORC_OK;
 }

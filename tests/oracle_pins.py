@@ -561,6 +561,70 @@ def pin_router_special_cases():
     np.testing.assert_array_equal(o2["r"][ids], o1["r"])
 
 
+def _scores_batch(Ns, d, rng, lo=-9, hi=10, lead=0, tail=0):
+    offs = (lead + np.concatenate([[0], np.cumsum(Ns)])).astype(np.int32)
+    x = rng.integers(lo, hi, size=(int(offs[-1]) + tail, d)).astype(np.float32)
+    return offs, x
+
+
+def pin_scores_integer_brute_force():
+    """Linear pruning-router scores (Eq. 8) on integer-valued tokens and weights are exact:
+    each one equals Python's integer dot product plus the bias, row by row.  Rows before
+    offsets[0] and after offsets[B] keep their initial zero (a legitimate score here ends in
+    .5, never 0)."""
+    rng = np.random.default_rng(31)
+    d = 7
+    offs, x = _scores_batch([1, 3, 2, 5, 1], d, rng, lead=2, tail=3)
+    w = rng.integers(-5, 6, size=d).astype(np.float32)
+    b = -3.5
+    s = oracle.token_scores("f32", offs, x, w, b)
+    for t in range(x.shape[0]):
+        if offs[0] <= t < offs[-1]:
+            exact = sum(int(w[j]) * int(x[t, j]) for j in range(d)) + b
+            assert s[t] == exact, (t, s[t], exact)
+        else:
+            assert s[t] == 0.0, t
+
+
+def pin_scores_correctly_rounded():
+    """Real-valued float32 tokens: each product is exact in double, so math.fsum of the
+    products and the bias (the correctly rounded double of the exact sum), rounded to
+    float32, is the score to the last bit; the oracle agrees on every row of this draw."""
+    rng = np.random.default_rng(32)
+    T, d = 300, 384
+    x = rng.standard_normal((T, d)).astype(np.float32)
+    w = (rng.standard_normal(d) / np.sqrt(d)).astype(np.float32)
+    b = float(np.float32(0.37))
+    offs = np.array([0, 100, 197, 300], np.int32)
+    s = oracle.token_scores("f32", offs, x, w, b)
+    wd = [float(v) for v in w]
+    for t in range(T):
+        ref = np.float32(math.fsum([wd[j] * float(x[t, j]) for j in range(d)] + [b]))
+        assert s[t] == ref, (t, s[t], ref)
+
+
+def pin_scores_special_cases():
+    """A one-hot head reads one coordinate (s = x[t, j] + b rounded once); values exactly
+    representable in bf16 score the same in both element types; an empty batch scores
+    nothing."""
+    rng = np.random.default_rng(33)
+    T, d = 40, 16
+    x = rng.standard_normal((T, d)).astype(np.float32)
+    offs = np.array([0, 17, 40], np.int32)
+    for j in (0, 5, d - 1):
+        w = np.zeros(d, np.float32)
+        w[j] = 1.0
+        s = oracle.token_scores("f32", offs, x, w, 0.25)
+        np.testing.assert_array_equal(s, (x[:, j].astype(np.float64) + 0.25).astype(np.float32))
+    xr = bf16_bits_to_f32(f32_to_bf16_bits(x))
+    wr = bf16_bits_to_f32(f32_to_bf16_bits(rng.standard_normal(d).astype(np.float32)))
+    np.testing.assert_array_equal(
+        oracle.token_scores("bf16", offs, f32_to_bf16_bits(xr), f32_to_bf16_bits(wr), -1.5),
+        oracle.token_scores("f32", offs, xr, wr, -1.5))
+    s = oracle.token_scores("f32", np.array([0], np.int32), x, wr, 3.0)
+    assert not s.any()
+
+
 ALL_PINS = [
     pin_bf16_rounding_table,
     pin_bf16_rounding_vs_torch,
@@ -580,4 +644,7 @@ ALL_PINS = [
     pin_stage_composition,
     pin_router_worked_examples,
     pin_router_special_cases,
+    pin_scores_integer_brute_force,
+    pin_scores_correctly_rounded,
+    pin_scores_special_cases,
 ]

@@ -43,6 +43,13 @@ MUTANTS = {
     "router_patch_count": ("mt * (0.5 * (double)N)", "mt * (0.5 * (double)(N - 1))"),
     "router_no_clamp": ("if (mt > 1.0)\n            mt = 1.0;", "if (0)\n            mt = 1.0;"),
     "router_scale_inverted": ("(1.0 - tau_tgt) / (1.0 - tau_ref)", "(1.0 - tau_ref) / (1.0 - tau_tgt)"),
+    "scores_dropped_bias": ("scores_out[t] = (float)(acc + b);", "scores_out[t] = (float)acc;"),
+    "scores_reversed_weights": ("acc += load_elem(dtype, w, j) * load_elem(dtype, x, t * d + j);",
+                                "acc += load_elem(dtype, w, d - 1 - j) * load_elem(dtype, x, t * d + j);"),
+    "scores_float_accumulator": ("acc += load_elem(dtype, w, j) * load_elem(dtype, x, t * d + j);",
+                                 "acc = (float)(acc + load_elem(dtype, w, j) * load_elem(dtype, x, t * d + j));"),
+    "scores_skip_last_row": ("for (int64_t t = offsets[i]; t < offsets[i + 1]; ++t) {",
+                             "for (int64_t t = offsets[i]; t < offsets[i + 1] - 1; ++t) {"),
 }
 
 

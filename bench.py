@@ -401,6 +401,7 @@ def main():
                       "achieved_gbs": b_full / t_full / 1e9, "frac": b_full / t_full / 1e9 / peak}
     solo = run_solo_full_stage(args, fz, runner, w, b, dev, flush, peak) if full else None
     router = run_router(args, fz, runner, b, dev, flush, peak)
+    scores = run_token_scores(args, fz, runner, b, dev, flush, peak)
 
     # ---- end to end through the C ABI with host buffers -------------------------------
     e2e = run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world)
@@ -426,6 +427,7 @@ def main():
         "full_stages": full_stats,
         "solo_full_stage": solo,
         "router": router,
+        "pruning_router": scores,
         "stages": per_stage,
         "kernel_ms_per_step": {"first (exit check or plan)": float(first_ms.sum(axis=1).mean()),
                                "k_image": float(image_ms.sum(axis=1).mean())},
@@ -528,6 +530,50 @@ def run_router(args, fz, runner, b, dev, flush, peak):
     return {"batch": b.batch, "ms": t * 1e3, "images_per_s": b.batch / t, "algorithmic_bytes": nbytes,
             "achieved_gbs": nbytes / t / 1e9, "frac": nbytes / t / 1e9 / peak,
             "note": "one CLS dot product per image in double: launch- and latency-bound by design"}
+
+
+def run_token_scores(args, fz, runner, b, dev, flush, peak):
+    """The linear pruning router (Eq. 8) on every token row of the step's input batch, L2
+    flushed before each launch; bytes = token rows + one float32 score per row + head weight
+    + offsets."""
+    import torch
+    from workloads import make_score_head
+    h = make_score_head(np.random.default_rng(2608), b.dim, b.dtype)
+    wt = torch.from_numpy(h.w.view(np.int16).copy() if b.dtype == "bf16" else h.w.copy()).to(dev)
+    fus = runner.Fusion(b.batch, 1, dev)
+    db = runner.device_batch(b.dtype, b.offsets, b.x, b.keys, b.sizes, b.scores, device=dev)
+    out = torch.zeros(db.max_rows, dtype=torch.float32, device=dev)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    for e in ev:
+        e.record()
+
+    def one():
+        flush.fill_(3)
+        fz.fusion_profile_next(ev[0], None, ev[1])
+        fus.token_scores(db, wt, h.b, out=out)
+
+    one()
+    torch.cuda.synchronize()
+    g = None
+    if not args.eager:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            one()
+    run = g.replay if g is not None else one
+    for _ in range(args.warmup):
+        run()
+    ms = []
+    for _ in range(args.steps):
+        run()
+        torch.cuda.synchronize()
+        ms.append(ev[0].elapsed_time(ev[1]))
+    eb = 2 if b.dtype == "bf16" else 4
+    rows = int(b.offsets[-1])
+    nbytes = rows * (b.dim * eb + 4) + b.dim * eb + (b.batch + 1) * 4
+    t = float(np.median(ms)) / 1e3
+    return {"kernel": "k_token_scores", "rows": rows, "ms": t * 1e3, "ms_p10_p90": [float(np.percentile(ms, 10)),
+            float(np.percentile(ms, 90))], "algorithmic_bytes": nbytes, "achieved_gbs": nbytes / t / 1e9,
+            "frac": nbytes / t / 1e9 / peak, "tokens_per_s": rows / t}
 
 
 def run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world):

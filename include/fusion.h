@@ -259,6 +259,28 @@ int fusion_merge_router(int dtype, fusion_ragged in, const void *x, int32_t dim,
                         int32_t *dev_status, void *stream);
 
 /*
+ * fusion_token_scores: the prune scores from a pruning router with a linear
+ * scoring head (Sec. III-E, Eq. 8, s_i = h_b(z_i) with h_b(z) = w . z + b),
+ * the input `scores` of fusion_prune and fusion_stage:
+ *   scores_out[t] = w . x[t] + b   for every row t in [offsets[0], offsets[B])
+ * B the device batch count.  Accumulated in float32 (products of two bf16 values
+ * are exact) along a summation tree of depth at most 24, so
+ * |error| <= 2^-18 * (sum_j |w_j x[t]_j| + |b|).
+ * x: [rows, dim] device, 16-byte aligned; w: [dim] device, the tokens' dtype,
+ * 16-byte aligned; b: the head's bias.  scores_out: [max_rows] float32; rows
+ * outside [offsets[0], offsets[B]) are not written.  in.ids is ignored (a row's
+ * score depends only on the row).
+ * Errors: FUSION_ERR_INVALID_ARG for NULL or misaligned pointers or a
+ * non-finite b; device bits: BAD_BATCH (nothing written), BAD_OFFSETS (when
+ * offsets[0] < 0, offsets[B] < offsets[0] or offsets[B] > max_rows nothing is
+ * written; per-sample defects - a decreasing pair, an empty or longer than
+ * max_tokens sample - are flagged while every row of the range is still
+ * scored), NONFINITE (a non-finite score, written as computed).  No workspace.
+ */
+int fusion_token_scores(int dtype, fusion_ragged in, const void *x, int32_t dim, const void *w,
+                        float b, float *scores_out, int32_t *dev_status, void *stream);
+
+/*
  * fusion_stage: one block's whole adaptation stage, fused (Algorithm 1 body):
  * merge (FUSION_STAGE_MERGE) -> exit check (FUSION_STAGE_EXIT; exited samples
  * leave the batch) -> prune (FUSION_STAGE_PRUNE) -> compacted output.  The

@@ -35,6 +35,7 @@ from ._binding import (  # noqa: F401
     fusion_exit_check_noalloc,
     fusion_merge,
     fusion_merge_router,
+    fusion_token_scores,
     fusion_profile_next,
     fusion_prune,
     fusion_stage,

@@ -40,7 +40,7 @@ FUSION_MAX_DIM = 1024
 
 EXPORTED = ("fusion_status_string", "fusion_version", "fusion_profile_next", "fusion_workspace_size",
             "fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune", "fusion_compact",
-            "fusion_stage", "fusion_merge_router")
+            "fusion_stage", "fusion_merge_router", "fusion_token_scores")
 
 
 class FusionError(RuntimeError):
@@ -96,8 +96,9 @@ def load(path: Optional[str] = None):
                                  V, V, V, V, V, V, V, V, V, SZ, V, V]
     lib.fusion_merge_router.argtypes = [ctypes.c_int, R, V, I32, V, ctypes.c_float, ctypes.c_float, ctypes.c_float,
                                         V, V, V, V]
+    lib.fusion_token_scores.argtypes = [ctypes.c_int, R, V, I32, V, ctypes.c_float, V, V, V]
     for name in ("fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune",
-                 "fusion_compact", "fusion_stage", "fusion_merge_router"):
+                 "fusion_compact", "fusion_stage", "fusion_merge_router", "fusion_token_scores"):
         getattr(lib, name).restype = ctypes.c_int
     del I64, F
     if path is None:
@@ -199,6 +200,12 @@ def fusion_merge_router(dtype, in_, x, dim, w, beta, tau_tgt, tau_ref, r_out, m_
     """Merge counts from the router with profile scaling (Sec. III-C, Eq. 4-5), by original id."""
     return load().fusion_merge_router(int(dtype), in_, _ptr(x), int(dim), _ptr(w), float(beta), float(tau_tgt),
                                       float(tau_ref), _ptr(r_out), _ptr(m_out), _ptr(dev_status), _stream(stream))
+
+
+def fusion_token_scores(dtype, in_, x, dim, w, b, scores_out, dev_status, stream=None) -> int:
+    """Prune scores from a linear pruning router, s = w . z + b per token row (Sec. III-E, Eq. 8)."""
+    return load().fusion_token_scores(int(dtype), in_, _ptr(x), int(dim), _ptr(w), float(b), _ptr(scores_out),
+                                      _ptr(dev_status), _stream(stream))
 
 
 def fusion_prune(dtype, in_, x, dim, sizes, scores, rho, x_out, sizes_out, scores_out, offsets_out,

@@ -361,6 +361,30 @@ int fusion_merge_router(int dtype, fusion_ragged in, const void *x, int32_t dim,
     return rc;
 }
 
+int fusion_token_scores(int dtype, fusion_ragged in, const void *x, int32_t dim, const void *w, float b,
+                        float *scores_out, int32_t *dev_status, void *stream) {
+    FZ_TRY(check_dtype(dtype));
+    FZ_TRY(check_ragged(in));
+    FZ_TRY(check_dim(dim));
+    if (!x || !w || !scores_out || !aligned16(x) || !aligned16(w)) return FUSION_ERR_INVALID_ARG;
+    if (!std::isfinite(b)) return FUSION_ERR_INVALID_ARG;
+    ScoreParams p{};
+    p.in = dev(in);
+    p.x = x;
+    p.dim = dim;
+    p.w = w;
+    p.b = b;
+    p.scores_out = scores_out;
+    p.status = dev_status;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const ProfileEvents ev = take_profile();
+    record(ev.start, s);
+    record(ev.mid, s);
+    const int rc = cuda_rc(launch_token_scores(dtype, p, s));
+    record(ev.end, s);
+    return rc;
+}
+
 int fusion_stage(int dtype, int flags, fusion_ragged in, const void *x, int32_t dim,
                  const void *keys, int32_t key_dim, const float *sizes, const float *scores,
                  const int32_t *r, const float *rho, fusion_exit_head head, uint8_t *exit_mask,

@@ -41,6 +41,24 @@ struct RouterParams {
 };
 cudaError_t launch_router(int dtype, const RouterParams &p, cudaStream_t s);
 
+// ---- pruning router: linear token scores ------------------------------------------------
+struct ScoreParams {
+    Ragged in;
+    const void *x;
+    int dim;
+    const void *w;      // scoring head weight [dim], the tokens' dtype
+    float b;            // scoring head bias
+    float *scores_out;  // [max_rows]
+    int group;          // lanes per row (set by the launcher)
+    int *status;
+};
+struct ScoreLayout {
+    int group;    // lanes per row
+    int chunks;   // 16-byte chunks per lane
+};
+ScoreLayout score_layout(int dtype, int dim);
+cudaError_t launch_token_scores(int dtype, const ScoreParams &p, cudaStream_t s);
+
 // ---- stand-alone plan ----------------------------------------------------------
 cudaError_t launch_plan(const PlanArgs &a, cudaStream_t s);
 

@@ -134,6 +134,13 @@ class Fusion:
                                         o["r"], o["m"], self.status))
         return o
 
+    def token_scores(self, b: DeviceBatch, w: torch.Tensor, bias: float,
+                     out: Optional[torch.Tensor] = None) -> torch.Tensor:
+        """Prune scores s = w . z + bias of every token row from a linear pruning router (Eq. 8)."""
+        o = out if out is not None else torch.zeros(b.max_rows, dtype=torch.float32, device=self.device)
+        fb.check(fb.fusion_token_scores(DTYPE_CODE[b.dtype], b.ragged(), b.x, b.dim, w, bias, o, self.status))
+        return o
+
     def exit_check(self, b: DeviceBatch, head: HeadTensors) -> Dict[str, torch.Tensor]:
         dev = self.device
         o = dict(exit_mask=torch.zeros(b.max_batch, dtype=torch.uint8, device=dev),

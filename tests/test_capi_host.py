@@ -168,3 +168,18 @@ def test_merge_router_rejects_bad_arguments(lib):
     for kw in (dict(x=None), dict(w=None), dict(r_out=None), dict(tau_ref=1.0), dict(tau_ref=1.5),
                dict(beta=float("nan")), dict(tau_tgt=float("inf"))):
         assert call(**kw) == fz.FUSION_ERR_INVALID_ARG, kw
+
+
+def test_token_scores_rejects_bad_arguments(lib):
+    def call(**kw):
+        args = dict(dtype=fz.FUSION_BF16, in_=_r(), x=FAKE, dim=384, w=FAKE, b=0.0, scores_out=FAKE,
+                    dev_status=FAKE, stream=0)
+        args.update(kw)
+        return fz.fusion_token_scores(*args.values())
+    assert call(dtype=5) == fz.FUSION_ERR_DTYPE
+    assert call(dim=24) == fz.FUSION_ERR_SHAPE
+    assert call(in_=_r(max_tokens=0)) == fz.FUSION_ERR_SHAPE
+    assert call(in_=_r(offsets=None)) == fz.FUSION_ERR_INVALID_ARG
+    for kw in (dict(x=None), dict(w=None), dict(scores_out=None), dict(x=FAKE + 4), dict(w=FAKE + 8),
+               dict(b=float("nan")), dict(b=float("-inf"))):
+        assert call(**kw) == fz.FUSION_ERR_INVALID_ARG, kw

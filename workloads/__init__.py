@@ -9,10 +9,12 @@ from .synth import (  # noqa: F401
     Batch,
     Head,
     RouterSpec,
+    ScoreHeadSpec,
     StageSpec,
     Workload,
     bf16_bits_to_f32,
     f32_to_bf16_bits,
     make_router,
+    make_score_head,
     make_workload,
 )

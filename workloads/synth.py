@@ -249,6 +249,21 @@ def make_router(rng: np.random.Generator, dim: int, dtype: str, tau_tgt: float =
     return RouterSpec(_round(w, dtype), float(np.float32(rng.normal(0.0, 0.25))), tau_tgt, tau_ref)
 
 
+@dataclass
+class ScoreHeadSpec:
+    """Linear pruning-router scoring head (Sec. III-E, Eq. 8): weight w [dim] (the tokens'
+    dtype) and bias b; a token's score is w . z + b."""
+    w: np.ndarray
+    b: float
+
+
+def make_score_head(rng: np.random.Generator, dim: int, dtype: str) -> ScoreHeadSpec:
+    """Random scoring-head weights with scores of unit scale for unit-variance tokens (no
+    trained head exists here): w ~ N(0, 1/dim), b ~ N(0, 0.25^2)."""
+    w = (rng.standard_normal(dim) / np.sqrt(dim)).astype(np.float32)
+    return ScoreHeadSpec(_round(w, dtype), float(np.float32(rng.normal(0.0, 0.25))))
+
+
 def ragged_counts_from_sizes(rng: np.random.Generator, batch: int, max_tokens: int):
     """Ragged variant of the non-uniform-size config: draw patch sizes uniform in {1..4}
     until the next one would push the image's total (CLS included) past max_tokens."""

@@ -51,6 +51,9 @@ def configure(lib):
     lib.orc_merge_router.argtypes = [i32, i32, P, P, i32, P, P, dbl, dbl, dbl, P, P, P]
     lib.orc_merge_router.restype = ctypes.c_int
     lib.orc_token_scores.argtypes = [i32, i32, P, i32, P, P, dbl, P]
+    lib.orc_exit_mlp.argtypes = [i32, i32, P, i32, P, P, i32, P, P, dbl, P, P, i32, P, P, i32, dbl,
+                                 P, P, P, P, P, P]
+    lib.orc_exit_mlp.restype = ctypes.c_int
     lib.orc_token_scores.restype = ctypes.c_int
     lib.orc_double_to_bf16.argtypes = [dbl]
     lib.orc_double_to_bf16.restype = ctypes.c_uint16
@@ -155,6 +158,32 @@ def exit_check(dtype: str, offsets, x, head) -> Dict[str, np.ndarray]:
                       _p(mask), _p(logits), _p(maxp), _p(gap), _p(u))
     _check(rc, "exit")
     return dict(exit_mask=mask, logits=logits, max_prob=maxp, exit_gap=gap, u=u)
+
+
+def exit_mlp(dtype: str, offsets, x, sizes, head) -> Dict[str, np.ndarray]:
+    """Sec. III-D exit check with an MLP exit head (``workloads.MlpHead``): pool (CLS row or
+    size-weighted patch mean) -> LayerNorm -> W1, GELU -> W2 -> softmax maximum.  Returns
+    exit_mask, logits, max_prob, exit_gap, pool (the head input), hidden."""
+    lib = _load()
+    et = _elem_dtype(dtype)
+    offsets = _c(offsets, np.int32)
+    x = _c(x, et)
+    B = len(offsets) - 1
+    d = x.shape[1]
+    W1, W2 = _c(head.w1, et), _c(head.w2, et)
+    H, C = W1.shape[0], W2.shape[0]
+    mask = np.zeros(B, np.uint8)
+    logits = np.zeros((B, C), np.float32)
+    maxp = np.zeros(B, np.float32)
+    gap = np.full(B, np.inf)
+    z = np.zeros((B, d), np.float64)
+    hid = np.zeros((B, H), np.float64)
+    rc = lib.orc_exit_mlp(_DT[dtype], B, _p(offsets), d, _p(x), _p(_c(sizes, np.float32)), int(head.pool),
+                          _p(_c(head.gamma, et)), _p(_c(head.beta, et)), float(head.eps), _p(W1),
+                          _p(_c(head.b1, np.float32)), H, _p(W2), _p(_c(head.b2, np.float32)), C,
+                          float(np.float32(head.tau)), _p(mask), _p(logits), _p(maxp), _p(gap), _p(z), _p(hid))
+    _check(rc, "exit_mlp")
+    return dict(exit_mask=mask, logits=logits, max_prob=maxp, exit_gap=gap, pool=z, hidden=hid)
 
 
 def merge_router(dtype: str, offsets, x, w, beta: float, tau_tgt: float, tau_ref: float, ids=None,

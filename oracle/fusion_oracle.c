@@ -21,6 +21,9 @@
  *           tokens by score (CLS-attention scores supplied as input).
  *   compact Drop the exited samples (Algorithm 1 returns early for them) and pack
  *           the survivors into a ragged, offset-indexed batch.
+ *   exit (MLP heads)  Sec. III-D, Eq. 6 and Eq. 7 with the paper's two exit heads
+ *           (Sec. III-G, Sec. IV-I: a SpatialPool head at block 8, a CLS-only head at block 10,
+ *           each a 2-layer MLP): head(z) = W2 GELU(W1 LN(pool(z)) + b1) + b2.
  *   scores  Sec. III-E, Eq. 8 (the prune scores' source): s_i = h_b(z_i) with a
  *           linear scoring head, s = w . z + b for every token, rounded once to
  *           float32.
@@ -41,6 +44,10 @@
  *     top-k pruning the lowest position;
  *   - surviving tokens keep ascending original position, CLS first;
  *   - LayerNorm: biased variance, eps supplied (1e-6 in every workload);
+ *   - MLP exit heads: SpatialPool is the size-weighted mean of the patch tokens
+ *     (sum s_t x_t / sum s_t; the CLS row when a sample has no patch), GELU is the
+ *     erf form, and for bf16 the LayerNorm output and the hidden activations are
+ *     rounded to bf16 (the operands of the two products);
  *   - bf16 storage: keys enter the dot products as stored; the LayerNorm output
  *     is rounded to bf16 before the head; merged tokens are rounded to bf16 once,
  *     after the weighted mean; everything else is accumulated in double.
@@ -534,5 +541,114 @@ int orc_token_scores(int dtype, int B, const int32_t *offsets, int d, const void
                 acc += load_elem(dtype, w, j) * load_elem(dtype, x, t * d + j);
             scores_out[t] = (float)(acc + b);
         }
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------------------- */
+/* exit check with the MLP heads (Sec. III-D, Eq. 6-7; Sec. III-G, Sec. IV-I)     */
+/* ------------------------------------------------------------------------- */
+/*
+ * head(z) = W2 GELU(W1 LN(pool(z)) + b1) + b2, c = max_k softmax(head(z))_k, exit iff
+ * c >= tau.  pool 0 (CLS-only head): the CLS row; pool 1 (SpatialPool head): the
+ * size-weighted mean of the patch rows (positions 1..N-1), the CLS row when N = 1.
+ * GELU(a) = a (1 + erf(a / sqrt 2)) / 2.  W1 [H, d] and W2 [C, H] row-major, gamma and
+ * beta [d], all in dtype; b1 [H], b2 [C] f32.  Outputs as in orc_exit, plus pool_out
+ * [B, d] and hidden_out [B, H] (after the bf16 rounding; both double, may be NULL).
+ */
+int orc_exit_mlp(int dtype, int B, const int32_t *offsets, int d, const void *x, const float *sizes, int pool,
+                 const void *gamma, const void *beta, double eps, const void *W1, const float *b1, int H,
+                 const void *W2, const float *b2, int C, double tau, uint8_t *exit_mask, float *logits,
+                 float *max_prob, double *exit_gap, double *pool_out, double *hidden_out)
+{
+    if (B < 0 || d <= 0 || H <= 0 || C <= 0 || (pool != 0 && pool != 1))
+        return ORC_ERR_ARG;
+    double *z = malloc(sizeof(double) * (size_t)d);
+    double *u = malloc(sizeof(double) * (size_t)d);
+    double *h = malloc(sizeof(double) * (size_t)H);
+    double *l = malloc(sizeof(double) * (size_t)C);
+    if (!z || !u || !h || !l) {
+        free(z);
+        free(u);
+        free(h);
+        free(l);
+        return ORC_ERR_NOMEM;
+    }
+    for (int i = 0; i < B; ++i) {
+        const int64_t o = offsets[i], n = offsets[i + 1] - offsets[i];
+        /* pool */
+        if (pool == 0 || n < 2) {
+            for (int j = 0; j < d; ++j)
+                z[j] = load_elem(dtype, x, o * d + j);
+        } else {
+            double wsum = 0.0;
+            for (int j = 0; j < d; ++j)
+                z[j] = 0.0;
+            for (int64_t t = o + 1; t < o + n; ++t) {
+                wsum += (double)sizes[t];
+                for (int j = 0; j < d; ++j)
+                    z[j] += (double)sizes[t] * load_elem(dtype, x, t * d + j);
+            }
+            for (int j = 0; j < d; ++j)
+                z[j] /= wsum;
+        }
+        if (pool_out)
+            memcpy(pool_out + (int64_t)i * d, z, sizeof(double) * (size_t)d);
+        /* LayerNorm */
+        double mean = 0.0;
+        for (int j = 0; j < d; ++j)
+            mean += z[j];
+        mean /= d;
+        double var = 0.0;
+        for (int j = 0; j < d; ++j)
+            var += (z[j] - mean) * (z[j] - mean);
+        var /= d;
+        const double rstd = 1.0 / sqrt(var + eps);
+        for (int j = 0; j < d; ++j) {
+            double v = (z[j] - mean) * rstd * load_elem(dtype, gamma, j) + load_elem(dtype, beta, j);
+            if (dtype == ORC_BF16)
+                v = bf16_to_double(double_to_bf16(v));
+            u[j] = v;
+        }
+        /* first layer and GELU */
+        for (int k = 0; k < H; ++k) {
+            double a = 0.0;
+            for (int j = 0; j < d; ++j)
+                a += load_elem(dtype, W1, (int64_t)k * d + j) * u[j];
+            a += (double)b1[k];
+            double g = 0.5 * a * (1.0 + erf(a / sqrt(2.0)));
+            if (dtype == ORC_BF16)
+                g = bf16_to_double(double_to_bf16(g));
+            h[k] = g;
+            if (hidden_out)
+                hidden_out[(int64_t)i * H + k] = g;
+        }
+        /* second layer, softmax maximum, exit rule */
+        double lmax = -INFINITY;
+        for (int c = 0; c < C; ++c) {
+            double acc = 0.0;
+            for (int k = 0; k < H; ++k)
+                acc += load_elem(dtype, W2, (int64_t)c * H + k) * h[k];
+            l[c] = acc + (double)b2[c];
+            if (l[c] > lmax)
+                lmax = l[c];
+        }
+        double S = 0.0;
+        for (int c = 0; c < C; ++c)
+            S += exp(l[c] - lmax);
+        const double cmax = 1.0 / S;
+        if (exit_mask)
+            exit_mask[i] = (cmax >= tau) ? 1 : 0;
+        if (max_prob)
+            max_prob[i] = (float)cmax;
+        if (exit_gap)
+            exit_gap[i] = fabs(cmax - tau);
+        if (logits)
+            for (int c = 0; c < C; ++c)
+                logits[(int64_t)i * C + c] = (float)l[c];
+    }
+    free(z);
+    free(u);
+    free(h);
+    free(l);
     return ORC_OK;
 }

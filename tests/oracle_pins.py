@@ -22,7 +22,7 @@ import numpy as np
 import torch
 
 import oracle
-from workloads import Head, bf16_bits_to_f32, f32_to_bf16_bits
+from workloads import POOL_CLS, POOL_SPATIAL, Head, MlpHead, bf16_bits_to_f32, f32_to_bf16_bits
 
 GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "worked_examples.json")
 
@@ -625,6 +625,113 @@ def pin_scores_special_cases():
     assert not s.any()
 
 
+def _mlp_case(rng, dtype, pool, B=7, d=32, H=48, C=29, Ns=(1, 2, 5, 9, 4, 3, 6)):
+    """A small ragged batch with sizes in {1..4} and an MLP head, as stored and as float64."""
+    offsets = np.concatenate([[0], np.cumsum(Ns[:B])]).astype(np.int32)
+    T = int(offsets[-1])
+    x32 = (rng.standard_normal((T, d)) * 1.5 + 0.3).astype(np.float32)
+    sizes = rng.integers(1, 5, T).astype(np.float32)
+    parts = dict(g=1 + 0.1 * rng.standard_normal(d), b=0.1 * rng.standard_normal(d),
+                 w1=rng.standard_normal((H, d)) / np.sqrt(d), w2=rng.standard_normal((C, H)) * 2 / np.sqrt(H))
+    parts = {k: v.astype(np.float32) for k, v in parts.items()}
+    b1 = (0.1 * rng.standard_normal(H)).astype(np.float32)
+    b2 = (0.1 * rng.standard_normal(C)).astype(np.float32)
+    if dtype == "bf16":
+        xs = f32_to_bf16_bits(x32)
+        st = {k: f32_to_bf16_bits(v) for k, v in parts.items()}
+        fl = {k: bf16_bits_to_f32(v).astype(np.float64) for k, v in st.items()}
+        xf = bf16_bits_to_f32(xs).astype(np.float64)
+    else:
+        xs, st = x32, parts
+        fl = {k: v.astype(np.float64) for k, v in parts.items()}
+        xf = x32.astype(np.float64)
+    head = MlpHead(pool, st["g"], st["b"], 1e-6, st["w1"], b1, st["w2"], b2, 0.08)
+    return offsets, xs, xf, sizes, head, fl, b1.astype(np.float64), b2.astype(np.float64)
+
+
+def pin_exit_mlp_vs_torch():
+    """MLP exit heads (pool -> LayerNorm -> W1, GELU -> W2 -> softmax max) against torch
+    float64 library routines: weighted mean, layer_norm, linear, gelu (erf form), softmax.
+    For bf16 the oracle's separately pinned rounding is applied to torch's LayerNorm output
+    and hidden activations."""
+    rng = np.random.default_rng(41)
+    T_ = torch.from_numpy
+    F = torch.nn.functional
+    rnd = np.vectorize(lambda v: oracle.bf16_to_double(oracle.double_to_bf16(v)))
+    for dtype in ("f32", "bf16"):
+        for pool in (POOL_CLS, POOL_SPATIAL):
+            offsets, xs, xf, sizes, head, fl, b1, b2 = _mlp_case(rng, dtype, pool)
+            e = oracle.exit_mlp(dtype, offsets, xs, sizes, head)
+            for i in range(len(offsets) - 1):
+                o, n = offsets[i], offsets[i + 1] - offsets[i]
+                if pool == POOL_CLS or n < 2:
+                    z = T_(xf[o])
+                else:
+                    w = T_(sizes[o + 1:o + n].astype(np.float64))
+                    z = (w[:, None] * T_(xf[o + 1:o + n])).sum(0) / w.sum()
+                np.testing.assert_allclose(e["pool"][i], z.numpy(), rtol=1e-13, atol=1e-13)
+                u = F.layer_norm(z[None], (z.shape[0],), T_(fl["g"]), T_(fl["b"]), eps=1e-6)
+                if dtype == "bf16":
+                    u = T_(rnd(u.numpy()))
+                h = F.gelu(F.linear(u, T_(fl["w1"]), T_(b1)))
+                if dtype == "bf16":
+                    h_ref = rnd(h.numpy())
+                    # a pre-rounding value this close to a bf16 midpoint may round either way
+                    near = np.abs(h.numpy() - h_ref) > 0.5 * np.abs(h_ref) * 2.0 ** -8 * (1 - 1e-9)
+                    ok = (e["hidden"][i] == h_ref[0]) | near[0]
+                    assert ok.all(), (dtype, pool, i)
+                    h = T_(e["hidden"][i][None])
+                else:
+                    np.testing.assert_allclose(e["hidden"][i], h.numpy()[0], rtol=1e-12, atol=1e-12)
+                lg = F.linear(h, T_(fl["w2"]), T_(b2))
+                c = torch.softmax(lg, dim=1).max().item()
+                np.testing.assert_allclose(e["logits"][i], lg.numpy()[0], rtol=1e-6, atol=1e-6)
+                np.testing.assert_allclose(e["max_prob"][i], c, rtol=1e-6)
+                assert e["exit_mask"][i] == (c >= float(np.float32(head.tau))) or abs(c - head.tau) < 1e-9
+
+
+def pin_exit_mlp_special_cases():
+    """Closed forms of the MLP heads: SpatialPool weights by size and skips CLS (a two-patch
+    sample pools to (a + 3 b) / 4); it pools the CLS row when there is no patch; equal patch
+    tokens pool to themselves; with W1 = I and b1 = +40 the GELU is the identity (in double)
+    and the head reduces to the separately pinned linear exit head; with b1 = -40 the hidden
+    layer is 0 and the logits are b2."""
+    rng = np.random.default_rng(42)
+    d, C = 16, 11
+    x = rng.standard_normal((4 + 3, d)).astype(np.float32)
+    offsets = np.array([0, 3, 4, 7], np.int32)           # [CLS a b], [CLS], [CLS v v]
+    sizes = np.array([1, 1, 3, 2, 1, 4, 2], np.float32)
+    x[5] = x[6] = rng.standard_normal(d).astype(np.float32)
+    g, b = np.ones(d, np.float32), np.zeros(d, np.float32)
+    W2 = (rng.standard_normal((C, d)) * 0.7).astype(np.float32)
+    b2 = (0.3 * rng.standard_normal(C)).astype(np.float32)
+    eye = np.eye(d, dtype=np.float32)
+    head = MlpHead(POOL_SPATIAL, g, b, 1e-6, eye, np.full(d, 40.0, np.float32), W2, b2, 0.3)
+    e = oracle.exit_mlp("f32", offsets, x, sizes, head)
+    np.testing.assert_allclose(e["pool"][0], (x[1].astype(np.float64) + 3 * x[2].astype(np.float64)) / 4,
+                               rtol=1e-15, atol=1e-15)
+    np.testing.assert_array_equal(e["pool"][1], x[3].astype(np.float64))
+    np.testing.assert_array_equal(e["pool"][2], x[5].astype(np.float64))
+    # identity first layer: head == LayerNorm -> W2 with bias b2 + 40 W2 1, the linear head
+    # (samples 1 and 2, whose pools are float32 values the linear head can take as CLS rows)
+    shifted = (b2.astype(np.float64) + 40.0 * W2.astype(np.float64).sum(1))
+    cls_rows = np.stack([e["pool"][i] for i in (1, 2)]).astype(np.float32)
+    lin = oracle.exit_check("f32", np.arange(3, dtype=np.int32), cls_rows,
+                            Head(g, b, 1e-6, W2, shifted.astype(np.float32), 0.3))
+    lin_logits = lin["logits"].astype(np.float64) - (shifted - shifted.astype(np.float32).astype(np.float64))
+    np.testing.assert_allclose(e["logits"][1:], lin_logits, rtol=1e-6, atol=1e-5)
+    np.testing.assert_allclose(e["hidden"][1:], lin["u"] + 40.0, rtol=1e-15, atol=1e-13)
+    # saturated-negative hidden layer
+    head.b1 = np.full(d, -40.0, np.float32)
+    e = oracle.exit_mlp("f32", offsets, x, sizes, head)
+    assert not e["hidden"].any()
+    np.testing.assert_array_equal(e["logits"], np.tile(b2, (3, 1)))
+    # CLS-only head reads the CLS row only
+    head.pool = POOL_CLS
+    e = oracle.exit_mlp("f32", offsets, x, sizes, head)
+    np.testing.assert_array_equal(e["pool"], x[offsets[:-1]].astype(np.float64))
+
+
 ALL_PINS = [
     pin_bf16_rounding_table,
     pin_bf16_rounding_vs_torch,
@@ -647,4 +754,6 @@ ALL_PINS = [
     pin_scores_integer_brute_force,
     pin_scores_correctly_rounded,
     pin_scores_special_cases,
+    pin_exit_mlp_vs_torch,
+    pin_exit_mlp_special_cases,
 ]

@@ -48,6 +48,18 @@ MUTANTS = {
                                 "acc += load_elem(dtype, w, d - 1 - j) * load_elem(dtype, x, t * d + j);"),
     "scores_float_accumulator": ("acc += load_elem(dtype, w, j) * load_elem(dtype, x, t * d + j);",
                                  "acc = (float)(acc + load_elem(dtype, w, j) * load_elem(dtype, x, t * d + j));"),
+    "mlp_pool_unweighted": ("z[j] += (double)sizes[t] * load_elem(dtype, x, t * d + j);",
+                            "z[j] += load_elem(dtype, x, t * d + j);"),
+    "mlp_pool_weight_sum": ("wsum += (double)sizes[t];", "wsum += 1.0;"),
+    "mlp_pool_includes_cls": ("for (int64_t t = o + 1; t < o + n; ++t) {\n                wsum",
+                              "for (int64_t t = o; t < o + n; ++t) {\n                wsum"),
+    "mlp_gelu_relu": ("double g = 0.5 * a * (1.0 + erf(a / sqrt(2.0)));", "double g = a > 0.0 ? a : 0.0;"),
+    "mlp_gelu_tanh": ("double g = 0.5 * a * (1.0 + erf(a / sqrt(2.0)));",
+                      "double g = 0.5 * a * (1.0 + tanh(0.7978845608 * (a + 0.044715 * a * a * a)));"),
+    "mlp_no_hidden_rounding": ("g = bf16_to_double(double_to_bf16(g));", "g = g;"),
+    "mlp_dropped_b1": ("a += (double)b1[k];", ";"),
+    "mlp_w1_transposed": ("load_elem(dtype, W1, (int64_t)k * d + j)", "load_elem(dtype, W1, (int64_t)j * H + k)"),
+    "mlp_w2_transposed": ("load_elem(dtype, W2, (int64_t)c * H + k)", "load_elem(dtype, W2, (int64_t)k * C + c)"),
     "scores_skip_last_row": ("for (int64_t t = offsets[i]; t < offsets[i + 1]; ++t) {",
                              "for (int64_t t = offsets[i]; t < offsets[i + 1] - 1; ++t) {"),
 }

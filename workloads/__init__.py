@@ -7,13 +7,17 @@ both the CPU oracle and the CUDA path without coupling them.
 from .synth import (  # noqa: F401
     CONFIGS,
     Batch,
+    POOL_CLS,
+    POOL_SPATIAL,
     Head,
+    MlpHead,
     RouterSpec,
     ScoreHeadSpec,
     StageSpec,
     Workload,
     bf16_bits_to_f32,
     f32_to_bf16_bits,
+    make_mlp_head,
     make_router,
     make_score_head,
     make_workload,

@@ -264,6 +264,48 @@ def make_score_head(rng: np.random.Generator, dim: int, dtype: str) -> ScoreHead
     return ScoreHeadSpec(_round(w, dtype), float(np.float32(rng.normal(0.0, 0.25))))
 
 
+POOL_CLS = 0       # CLS-only exit head
+POOL_SPATIAL = 1   # SpatialPool exit head: size-weighted mean of the patch tokens
+
+
+@dataclass
+class MlpHead:
+    """An exit head as a 2-layer MLP (the paper's SpatialPool and CLS-only heads):
+    pool -> LayerNorm -> Linear(d -> H) -> GELU -> Linear(H -> C) -> softmax, threshold tau."""
+    pool: int
+    gamma: np.ndarray   # [d] f32 or bf16 bits
+    beta: np.ndarray    # [d]
+    eps: float
+    w1: np.ndarray      # [H, d] row-major
+    b1: np.ndarray      # [H] f32
+    w2: np.ndarray      # [C, H] row-major
+    b2: np.ndarray      # [C] f32
+    tau: float
+
+    @property
+    def hidden(self) -> int:
+        return int(self.w1.shape[0])
+
+    @property
+    def classes(self) -> int:
+        return int(self.w2.shape[0])
+
+
+def make_mlp_head(rng: np.random.Generator, pool: int, dim: int, hidden: int, classes: int, dtype: str,
+                  tau: float = 0.05, logit_scale: float = 3.0) -> MlpHead:
+    """Random MLP exit head (no trained head exists here): LayerNorm affine near identity,
+    W1 ~ N(0, 1/d), b1 ~ N(0, 0.1^2), W2 ~ N(0, s^2 / H) so that the logits have standard
+    deviation about s (softmax maxima spread over a useful range), b2 ~ N(0, 0.1^2)."""
+    gamma = (1.0 + 0.1 * rng.standard_normal(dim)).astype(np.float32)
+    beta = (0.1 * rng.standard_normal(dim)).astype(np.float32)
+    w1 = (rng.standard_normal((hidden, dim)) / np.sqrt(dim)).astype(np.float32)
+    b1 = (0.1 * rng.standard_normal(hidden)).astype(np.float32)
+    w2 = (rng.standard_normal((classes, hidden)) * logit_scale / np.sqrt(hidden)).astype(np.float32)
+    b2 = (0.1 * rng.standard_normal(classes)).astype(np.float32)
+    return MlpHead(int(pool), _round(gamma, dtype), _round(beta, dtype), 1e-6, _round(w1, dtype), b1,
+                   _round(w2, dtype), b2, float(tau))
+
+
 def ragged_counts_from_sizes(rng: np.random.Generator, batch: int, max_tokens: int):
     """Ragged variant of the non-uniform-size config: draw patch sizes uniform in {1..4}
     until the next one would push the image's total (CLS included) past max_tokens."""

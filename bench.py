@@ -91,11 +91,17 @@ def peaks():
         return 6800.0, "fallback"
 
 
+# The translation unit of the per-sample kernel k_image_tc: its source and every header it
+# includes.  The recorded DRAM traffic stays valid while none of these changes.
+IMAGE_TC_SOURCES = ("paper_2607_02612_gb300/csrc/image_tc.cu", "paper_2607_02612_gb300/csrc/sample.cuh",
+                    "paper_2607_02612_gb300/csrc/launch.h", "paper_2607_02612_gb300/csrc/plan.cuh",
+                    "paper_2607_02612_gb300/csrc/common.cuh", "include/fusion.h")
+
+
 def source_hash() -> str:
     h = hashlib.sha256()
-    csrc = os.path.join(ROOT, "paper_2607_02612_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
-        with open(os.path.join(csrc, f), "rb") as fh:
+    for f in IMAGE_TC_SOURCES:
+        with open(os.path.join(ROOT, f), "rb") as fh:
             h.update(f.encode() + fh.read())
     return h.hexdigest()[:16]
 
@@ -402,6 +408,7 @@ def main():
     solo = run_solo_full_stage(args, fz, runner, w, b, dev, flush, peak) if full else None
     router = run_router(args, fz, runner, b, dev, flush, peak)
     scores = run_token_scores(args, fz, runner, b, dev, flush, peak)
+    exit_mlp = run_exit_mlp(args, fz, runner, b, dev, flush, peak)
 
     # ---- end to end through the C ABI with host buffers -------------------------------
     e2e = run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world)
@@ -428,6 +435,7 @@ def main():
         "solo_full_stage": solo,
         "router": router,
         "pruning_router": scores,
+        "exit_mlp": exit_mlp,
         "stages": per_stage,
         "kernel_ms_per_step": {"first (exit check or plan)": float(first_ms.sum(axis=1).mean()),
                                "k_image": float(image_ms.sum(axis=1).mean())},
@@ -574,6 +582,61 @@ def run_token_scores(args, fz, runner, b, dev, flush, peak):
     return {"kernel": "k_token_scores", "rows": rows, "ms": t * 1e3, "ms_p10_p90": [float(np.percentile(ms, 10)),
             float(np.percentile(ms, 90))], "algorithmic_bytes": nbytes, "achieved_gbs": nbytes / t / 1e9,
             "frac": nbytes / t / 1e9 / peak, "tokens_per_s": rows / t}
+
+
+def run_exit_mlp(args, fz, runner, b, dev, flush, peak):
+    """The exit check with the paper's block-8 exit head (SpatialPool, 2-layer MLP, hidden
+    2d, 1000 classes) on the step's input batch, L2 flushed before each call; bytes = token
+    rows + sizes (the pool) + both weight matrices + logits and outputs; events split the
+    call into pool + first layer and second layer + softmax."""
+    import torch
+    from workloads import POOL_SPATIAL, make_mlp_head
+    head = make_mlp_head(np.random.default_rng(2609), POOL_SPATIAL, b.dim, 2 * b.dim, 1000, b.dtype)
+    ht = runner.mlp_head_tensors(head, b.dtype, dev)
+    fus = runner.Fusion(b.batch, 1, dev)
+    db = runner.device_batch(b.dtype, b.offsets, b.x, b.keys, b.sizes, b.scores, device=dev)
+    nbytes_ws = fz.fusion_exit_mlp_workspace_size(b.batch, b.dim, ht.hidden, ht.classes)
+    ws = torch.zeros(nbytes_ws, dtype=torch.uint8, device=dev)
+    out = dict(mask=torch.zeros(b.batch, dtype=torch.uint8, device=dev),
+               logits=torch.zeros((b.batch, ht.classes), device=dev), maxp=torch.zeros(b.batch, device=dev))
+    code = fz.FUSION_BF16 if b.dtype == "bf16" else fz.FUSION_F32
+    hs = ht.c_struct()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    for e in ev:
+        e.record()
+
+    def one():
+        flush.fill_(3)
+        fz.fusion_profile_next(ev[0], ev[1], ev[2])
+        fz.check(fz.fusion_exit_check_mlp(code, db.ragged(), db.x, b.dim, db.sizes, hs, out["mask"], out["logits"],
+                                          out["maxp"], ws, nbytes_ws, fus.status))
+
+    one()
+    torch.cuda.synchronize()
+    g = None
+    if not args.eager:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            one()
+    run = g.replay if g is not None else one
+    for _ in range(args.warmup):
+        run()
+    ms, ms1 = [], []
+    for _ in range(args.steps):
+        run()
+        torch.cuda.synchronize()
+        ms.append(ev[0].elapsed_time(ev[2]))
+        ms1.append(ev[0].elapsed_time(ev[1]))
+    eb = 2 if b.dtype == "bf16" else 4
+    rows = int(b.offsets[-1])
+    H, C = ht.hidden, ht.classes
+    nbytes = rows * (b.dim * eb + 4) + (H * b.dim + C * H) * eb + b.batch * (C * 4 + 5)
+    flops = 2.0 * b.batch * (b.dim * H + H * C)
+    t = float(np.median(ms)) / 1e3
+    return {"kernels": "k_head_pool, k_exit (first layer), k_exit (second layer)", "batch": b.batch, "hidden": H,
+            "classes": C, "ms": t * 1e3, "ms_pool_and_first_layer": float(np.median(ms1)),
+            "algorithmic_bytes": nbytes, "achieved_gbs": nbytes / t / 1e9, "frac": nbytes / t / 1e9 / peak,
+            "tflops": flops / t / 1e12, "images_per_s": b.batch / t}
 
 
 def run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world):

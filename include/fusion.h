@@ -93,6 +93,10 @@ extern "C" {
    inside the per-sample kernel; larger ones launch a plan kernel first */
 #define FUSION_FUSED_PLAN_MAX_BATCH 1024
 
+/* Pooling of an MLP exit head (fusion_mlp_head.pool). */
+#define FUSION_POOL_CLS 0     /* the CLS row (the paper's CLS-only head, block 10) */
+#define FUSION_POOL_SPATIAL 1 /* size-weighted mean of the patch rows (SpatialPool head, block 8) */
+
 /* A ragged batch as seen by the device.  All pointers are device memory. */
 typedef struct fusion_ragged {
     int32_t max_batch;      /* host upper bound on the number of samples (>= 0) */
@@ -114,6 +118,23 @@ typedef struct fusion_exit_head {
     int32_t classes;      /* C >= 1 */
     float tau;            /* exit threshold */
 } fusion_exit_head;
+
+/* Exit head as a 2-layer MLP (Sec. III-G; Sec. IV-I: the paper's SpatialPool head at
+ * block 8 and CLS-only head at block 10): head(z) = W2 GELU(W1 LN(pool(z)) + b1) + b2,
+ * then softmax; a sample exits iff its maximum class probability c >= tau (Eq. 7). */
+typedef struct fusion_mlp_head {
+    int32_t pool;         /* FUSION_POOL_CLS or FUSION_POOL_SPATIAL */
+    const void *ln_gamma; /* [dim], dtype */
+    const void *ln_beta;  /* [dim], dtype */
+    float ln_eps;         /* LayerNorm epsilon (biased variance) */
+    const void *w1;       /* [hidden, dim] row-major, dtype */
+    const float *b1;      /* [hidden] float32 */
+    int32_t hidden;       /* H: a multiple of 16 in [16, FUSION_MAX_DIM] */
+    const void *w2;       /* [classes, hidden] row-major, dtype */
+    const float *b2;      /* [classes] float32 */
+    int32_t classes;      /* C >= 1 */
+    float tau;            /* exit threshold */
+} fusion_mlp_head;
 
 /* Human-readable name of a return code or of a single FUSION_DEV_* bit. */
 const char *fusion_status_string(int code);
@@ -184,6 +205,33 @@ int fusion_merge(int dtype, fusion_ragged in, const void *x, int32_t dim, const 
 int fusion_exit_check(int dtype, fusion_ragged in, const void *x, int32_t dim,
                       fusion_exit_head head, uint8_t *exit_mask, float *logits, float *max_prob,
                       void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream);
+
+/*
+ * Scratch bytes of fusion_exit_check_mlp for max_batch samples, token width dim and
+ * the head's hidden width and classes; zero-filled before its first use, left
+ * zero-filled by every call (as fusion_workspace_size).
+ */
+size_t fusion_exit_mlp_workspace_size(int32_t max_batch, int32_t dim, int32_t hidden, int32_t classes);
+
+/*
+ * fusion_exit_check_mlp: the exit check (Sec. III-D, Eq. 6 and Eq. 7) with an MLP exit
+ * head.  For every sample: z = its CLS row (FUSION_POOL_CLS) or sum_t s_t x_t / sum_t s_t
+ * over its patch rows (FUSION_POOL_SPATIAL; the CLS row when it has no patch), in
+ * float32; u = LayerNorm(z) (gamma, beta, eps, biased variance); h = GELU(W1 u + b1)
+ * with GELU(a) = a (1 + erf(a / sqrt 2)) / 2; logits l = W2 h + b2; c = max_k
+ * softmax(l)_k; exit iff c >= tau.  For FUSION_BF16, u and h are rounded to bf16 (the
+ * operands of the two tensor-core products, float32 accumulation).
+ * sizes: [max_rows] float32 token sizes (needed for FUSION_POOL_SPATIAL, else may be
+ * NULL).  Outputs as fusion_exit_check: exit_mask [max_batch], logits [max_batch,
+ * classes] (may be NULL), max_prob [max_batch] (may be NULL).
+ * Errors: FUSION_ERR_INVALID_ARG for NULL or misaligned pointers or a bad pool;
+ * FUSION_ERR_SHAPE for a hidden width outside the dim rule or classes < 1;
+ * FUSION_ERR_WORKSPACE below fusion_exit_mlp_workspace_size; device bits BAD_BATCH,
+ * BAD_OFFSETS (that sample's head input is zero), NONFINITE.
+ */
+int fusion_exit_check_mlp(int dtype, fusion_ragged in, const void *x, int32_t dim, const float *sizes,
+                          fusion_mlp_head head, uint8_t *exit_mask, float *logits, float *max_prob,
+                          void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream);
 
 /*
  * fusion_exit_check_noalloc: fusion_exit_check for callers that cannot allocate

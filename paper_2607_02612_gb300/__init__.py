@@ -36,6 +36,11 @@ from ._binding import (  # noqa: F401
     fusion_merge,
     fusion_merge_router,
     fusion_token_scores,
+    fusion_exit_check_mlp,
+    fusion_exit_mlp_workspace_size,
+    mlp_head,
+    FUSION_POOL_CLS,
+    FUSION_POOL_SPATIAL,
     fusion_profile_next,
     fusion_prune,
     fusion_stage,

@@ -37,10 +37,13 @@ FUSION_STAGE_PRUNE = 4
 FUSION_MAX_TOKENS = 1024
 FUSION_FUSED_PLAN_MAX_BATCH = 1024
 FUSION_MAX_DIM = 1024
+FUSION_POOL_CLS = 0
+FUSION_POOL_SPATIAL = 1
 
 EXPORTED = ("fusion_status_string", "fusion_version", "fusion_profile_next", "fusion_workspace_size",
             "fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune", "fusion_compact",
-            "fusion_stage", "fusion_merge_router", "fusion_token_scores")
+            "fusion_stage", "fusion_merge_router", "fusion_token_scores", "fusion_exit_mlp_workspace_size",
+            "fusion_exit_check_mlp")
 
 
 class FusionError(RuntimeError):
@@ -51,6 +54,13 @@ class fusion_ragged(ctypes.Structure):
     _fields_ = [("max_batch", ctypes.c_int32), ("max_tokens", ctypes.c_int32),
                 ("max_rows", ctypes.c_int64), ("offsets", ctypes.c_void_p),
                 ("batch", ctypes.c_void_p), ("ids", ctypes.c_void_p)]
+
+
+class fusion_mlp_head(ctypes.Structure):
+    _fields_ = [("pool", ctypes.c_int32), ("ln_gamma", ctypes.c_void_p), ("ln_beta", ctypes.c_void_p),
+                ("ln_eps", ctypes.c_float), ("w1", ctypes.c_void_p), ("b1", ctypes.c_void_p),
+                ("hidden", ctypes.c_int32), ("w2", ctypes.c_void_p), ("b2", ctypes.c_void_p),
+                ("classes", ctypes.c_int32), ("tau", ctypes.c_float)]
 
 
 class fusion_exit_head(ctypes.Structure):
@@ -97,8 +107,12 @@ def load(path: Optional[str] = None):
     lib.fusion_merge_router.argtypes = [ctypes.c_int, R, V, I32, V, ctypes.c_float, ctypes.c_float, ctypes.c_float,
                                         V, V, V, V]
     lib.fusion_token_scores.argtypes = [ctypes.c_int, R, V, I32, V, ctypes.c_float, V, V, V]
+    lib.fusion_exit_mlp_workspace_size.argtypes = [I32, I32, I32, I32]
+    lib.fusion_exit_mlp_workspace_size.restype = SZ
+    lib.fusion_exit_check_mlp.argtypes = [ctypes.c_int, R, V, I32, V, fusion_mlp_head, V, V, V, V, SZ, V, V]
     for name in ("fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune",
-                 "fusion_compact", "fusion_stage", "fusion_merge_router", "fusion_token_scores"):
+                 "fusion_compact", "fusion_stage", "fusion_merge_router", "fusion_token_scores",
+                 "fusion_exit_check_mlp"):
         getattr(lib, name).restype = ctypes.c_int
     del I64, F
     if path is None:
@@ -135,6 +149,12 @@ def ragged(max_batch: int, max_tokens: int, max_rows: int, offsets, batch=None, 
 def exit_head(gamma, beta, eps: float, weight, bias, classes: int, tau: float) -> fusion_exit_head:
     return fusion_exit_head(_ptr(gamma), _ptr(beta), float(eps), _ptr(weight), _ptr(bias), int(classes),
                             float(tau))
+
+
+def mlp_head(pool: int, gamma, beta, eps: float, w1, b1, hidden: int, w2, b2, classes: int,
+             tau: float) -> fusion_mlp_head:
+    return fusion_mlp_head(int(pool), _ptr(gamma), _ptr(beta), float(eps), _ptr(w1), _ptr(b1), int(hidden),
+                           _ptr(w2), _ptr(b2), int(classes), float(tau))
 
 
 def check(rc: int) -> None:
@@ -206,6 +226,18 @@ def fusion_token_scores(dtype, in_, x, dim, w, b, scores_out, dev_status, stream
     """Prune scores from a linear pruning router, s = w . z + b per token row (Sec. III-E, Eq. 8)."""
     return load().fusion_token_scores(int(dtype), in_, _ptr(x), int(dim), _ptr(w), float(b), _ptr(scores_out),
                                       _ptr(dev_status), _stream(stream))
+
+
+def fusion_exit_mlp_workspace_size(max_batch: int, dim: int, hidden: int, classes: int) -> int:
+    return int(load().fusion_exit_mlp_workspace_size(int(max_batch), int(dim), int(hidden), int(classes)))
+
+
+def fusion_exit_check_mlp(dtype, in_, x, dim, sizes, head, exit_mask, logits, max_prob, workspace, workspace_bytes,
+                          dev_status, stream=None) -> int:
+    """Exit check with an MLP exit head (SpatialPool or CLS-only; Sec. III-D, Eq. 6-7)."""
+    return load().fusion_exit_check_mlp(int(dtype), in_, _ptr(x), int(dim), _ptr(sizes), head, _ptr(exit_mask),
+                                        _ptr(logits), _ptr(max_prob), _ptr(workspace), int(workspace_bytes),
+                                        _ptr(dev_status), _stream(stream))
 
 
 def fusion_prune(dtype, in_, x, dim, sizes, scores, rho, x_out, sizes_out, scores_out, offsets_out,

@@ -1,5 +1,8 @@
 // Exit check (Sec. III-D, Eq. 6-7): u = LayerNorm(CLS), logits = W u + b,
-// c = max_k softmax(logits)_k, exit iff c >= tau.
+// c = max_k softmax(logits)_k, exit iff c >= tau.  The general kernel also runs the two
+// layers of the MLP exit heads (Sec. III-G): the first reads the pooled float32 rows, the
+// LayerNorm and GELU(W1 u + b1) rounded to the dtype; the second reads those rows densely,
+// without LayerNorm, and ends in the softmax maximum and the exit rule.
 //
 // Two kernels.  The cluster kernel (heads of at most 8 class tiles) is described below.
 // The general one: grid (class tiles of kExitCT) x (sample tiles of kExitBT).  Every CTA computes
@@ -54,6 +57,12 @@ __device__ __forceinline__ uint16_t ln_out_bf16(float x, F2 mean, F2 rstd, float
 __device__ __forceinline__ float ln_out_f32(float x, F2 mean, F2 rstd, float g, float b) {
     const float d = __fsub_rn(__fsub_rn(x, mean.hi), mean.lo);
     return __fmaf_rn(__fmul_rn(d, rstd.hi), g, b);
+}
+
+template <typename T> __device__ __forceinline__ T from_float(float v);
+template <> __device__ __forceinline__ float from_float<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_float<__nv_bfloat16>(float v) {
+    return __float2bfloat16_rn(v);
 }
 
 template <typename T>
@@ -235,10 +244,10 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
             const int sl = it / nchunk, c = it - sl * nchunk;
             const int s = s0 + sl;
             T *dst = u_s + (size_t)sl * u_stride + c * CH;
-            long long row = -1;
-            if (sl < kExitBT && s < B) {
-                row = p.in.offsets[s];
-                if (row < 0 || row >= p.in.max_rows) row = -1;
+            long long row = -1;   // in_mode 2: the LayerNorm reads u_in and fills the tile
+            if (sl < kExitBT && s < B && p.in_mode != 2) {
+                row = p.in_mode == 0 ? (long long)p.in.offsets[s] : (long long)s;
+                if (p.in_mode == 0 && (row < 0 || row >= p.in.max_rows)) row = -1;
             }
             if (row >= 0)
                 cp_async16(dst, reinterpret_cast<const T *>(p.x) + row * dim + c * CH);
@@ -253,7 +262,7 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
         // ---- LayerNorm of one CLS row per warp (float-float statistics) ---------------
         const int s = s0 + warp;
         bool ok = s < B;
-        if (ok) {
+        if (ok && p.in_mode == 0) {
             const long long row = p.in.offsets[s];
             if (row < 0 || row >= p.in.max_rows) {
                 if (lane == 0) raise_status(p.status, FUSION_DEV_BAD_OFFSETS);
@@ -261,11 +270,27 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
             }
         }
         T *xr = u_s + (size_t)warp * u_stride;
-        if (ok) {
+        // the row's chunk c as floats: from the tile, or from the float32 input rows
+        const float *ur = p.in_mode == 2 && ok ? p.u_in + (size_t)s * dim : nullptr;
+        auto in_chunk = [&](int c, float (&f)[CH]) {
+            if (ur) {
+#pragma unroll
+                for (int e = 0; e < CH; e += 4) {
+                    const float4 v = *reinterpret_cast<const float4 *>(ur + c * CH + e);
+                    f[e] = v.x;
+                    f[e + 1] = v.y;
+                    f[e + 2] = v.z;
+                    f[e + 3] = v.w;
+                }
+            } else {
+                chunk_to_f(*reinterpret_cast<const uint4 *>(xr + c * CH), f);
+            }
+        };
+        if (ok && !p.skip_ln) {
             float ss = 0.0f, sc = 0.0f;
             for (int c = lane; c < nchunk; c += 32) {
                 float f[CH];
-                chunk_to_f(*reinterpret_cast<const uint4 *>(xr + c * CH), f);
+                in_chunk(c, f);
 #pragma unroll
                 for (int e = 0; e < CH; ++e) neu_add(ss, sc, f[e]);
             }
@@ -275,7 +300,7 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
             float lo = 0.0f;
             for (int c = lane; c < nchunk; c += 32) {
                 float f[CH];
-                chunk_to_f(*reinterpret_cast<const uint4 *>(xr + c * CH), f);
+                in_chunk(c, f);
 #pragma unroll
                 for (int e = 0; e < CH; ++e) {
                     F2 d = two_sum(f[e], -mean.hi);
@@ -292,7 +317,7 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
             const T *bb = reinterpret_cast<const T *>(p.head.beta);
             for (int c = lane; c < nchunk; c += 32) {
                 float f[CH], gf[CH], bf[CH];
-                chunk_to_f(*reinterpret_cast<const uint4 *>(xr + c * CH), f);
+                in_chunk(c, f);
                 chunk_to_f(ldg16(g + c * CH), gf);
                 chunk_to_f(ldg16(bb + c * CH), bf);
                 if constexpr (kBf16) {
@@ -311,7 +336,7 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
                     *reinterpret_cast<float4 *>(xr + c * CH) = o;
                 }
             }
-        } else {
+        } else if (!ok) {   // (skip_ln: the loaded rows stay as they are)
             for (int c = lane; c < nchunk; c += 32) *reinterpret_cast<uint4 *>(xr + c * CH) = make_uint4(0, 0, 0, 0);
         }
     }
@@ -323,8 +348,19 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
     if (active) {
         exit_gemm<T>(p, u_s, w_region, c0, dim, C, n_k, acc, acc2);
         exit_logits<T>(p, lg_s, bias_s, acc, acc2, s0, c0, B, C);
-        // ---- partial softmax of this class tile: warp -> sample ------------------------
-        {
+        if (p.out_mode == 1) {
+            // ---- hidden layer of an MLP head: GELU (erf form), rounded to the dtype -------
+            T *ho = reinterpret_cast<T *>(p.hidden_out);
+            for (int it = tid; it < kExitBT * kExitCT; it += kExitThreads) {
+                const int sl = it / kExitCT, col = it - sl * kExitCT;
+                if (s0 + sl < B && c0 + col < C) {
+                    const float a = lg_s[it];
+                    const float g = 0.5f * a * (1.0f + erff(a * 0.70710678118654752f));
+                    ho[(size_t)(s0 + sl) * C + c0 + col] = from_float<T>(g);
+                }
+            }
+        } else {
+            // ---- partial softmax of this class tile: warp -> sample ------------------------
             const int sl = warp, s = s0 + sl;
             float m = -INFINITY;
             for (int col = lane; col < kExitCT; col += 32) m = fmaxf(m, lg_s[sl * kExitCT + col]);
@@ -340,6 +376,7 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
             if (lane == 0 && s < B) p.partials[(size_t)s * p.n_ctile + ct] = make_float2(m, z);
         }
     }
+    if (p.out_mode == 1) return;   // no softmax across the tiles of a hidden layer
 
     // ---- the last class tile of this sample tile merges the partials ---------------
     __shared__ int s_last;
@@ -670,7 +707,7 @@ cudaError_t launch_exit_cluster(const ExitParams &p, cudaStream_t s) {
 cudaError_t launch_exit(int dtype, const ExitParams &p, cudaStream_t s) {
     // the class tiles of a sample tile as one cluster (portable size: at most 8 tiles,
     // 1024 classes); larger heads take the kernel with a global last-CTA merge
-    if (p.n_ctile <= 8 && p.n_btile > 0)
+    if (p.n_ctile <= 8 && p.n_btile > 0 && p.in_mode == 0 && !p.skip_ln && p.out_mode == 0)
         return dtype == FUSION_BF16 ? launch_exit_cluster<__nv_bfloat16>(p, s) : launch_exit_cluster<float>(p, s);
     const size_t smem = exit_smem_bytes(dtype, p.dim);
     const dim3 grid(p.n_ctile, p.n_btile);

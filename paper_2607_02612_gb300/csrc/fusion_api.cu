@@ -361,6 +361,100 @@ int fusion_merge_router(int dtype, fusion_ragged in, const void *x, int32_t dim,
     return rc;
 }
 
+namespace {
+// fusion_exit_check_mlp scratch: the linear exit workspace for `classes`, then the pooled
+// rows [max_batch, dim] float32 and the hidden rows [max_batch, hidden] (float32 size).
+struct MlpWs {
+    size_t u, hid, total;
+};
+MlpWs mlp_ws_layout(int32_t max_batch, int32_t dim, int32_t hidden, int32_t classes) {
+    const size_t mb = (size_t)(max_batch > 0 ? max_batch : 1);
+    MlpWs L;
+    L.u = (ws_layout(max_batch, classes).total + 255) / 256 * 256;
+    L.hid = (L.u + mb * (size_t)dim * sizeof(float) + 255) / 256 * 256;
+    L.total = (L.hid + mb * (size_t)hidden * sizeof(float) + 255) / 256 * 256;
+    return L;
+}
+}  // namespace
+
+size_t fusion_exit_mlp_workspace_size(int32_t max_batch, int32_t dim, int32_t hidden, int32_t classes) {
+    if (max_batch < 0) max_batch = 0;
+    return mlp_ws_layout(max_batch, dim < 16 ? 16 : dim, hidden < 16 ? 16 : hidden, classes < 1 ? 1 : classes).total;
+}
+
+int fusion_exit_check_mlp(int dtype, fusion_ragged in, const void *x, int32_t dim, const float *sizes,
+                          fusion_mlp_head head, uint8_t *exit_mask, float *logits, float *max_prob,
+                          void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream) {
+    FZ_TRY(check_dtype(dtype));
+    FZ_TRY(check_ragged(in));
+    FZ_TRY(check_dim(dim));
+    FZ_TRY(check_dim(head.hidden));
+    if (head.classes < 1) return FUSION_ERR_SHAPE;
+    if (head.pool != FUSION_POOL_CLS && head.pool != FUSION_POOL_SPATIAL) return FUSION_ERR_INVALID_ARG;
+    if (head.pool == FUSION_POOL_SPATIAL && !sizes) return FUSION_ERR_INVALID_ARG;
+    if (!x || !exit_mask || !aligned16(x)) return FUSION_ERR_INVALID_ARG;
+    if (!head.ln_gamma || !head.ln_beta || !head.w1 || !head.b1 || !head.w2 || !head.b2) return FUSION_ERR_INVALID_ARG;
+    if (!aligned16(head.ln_gamma) || !aligned16(head.ln_beta) || !aligned16(head.w1) || !aligned16(head.w2))
+        return FUSION_ERR_INVALID_ARG;
+    const MlpWs L = mlp_ws_layout(in.max_batch, dim, head.hidden, head.classes);
+    if (!workspace || !aligned16(workspace)) return FUSION_ERR_WORKSPACE;
+    if (workspace_bytes < L.total) return FUSION_ERR_WORKSPACE;
+    unsigned char *wb = static_cast<unsigned char *>(workspace);
+    float *u = reinterpret_cast<float *>(wb + L.u);
+    void *hid = wb + L.hid;
+    const Ws w = carve(workspace, in.max_batch, head.classes);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int n_btile = ceil_div(in.max_batch > 0 ? in.max_batch : 1, kExitBT);
+
+    PoolParams pp{};
+    pp.in = dev(in);
+    pp.x = x;
+    pp.dim = dim;
+    pp.sizes = sizes;
+    pp.pool = head.pool;
+    pp.u_out = u;
+    pp.status = dev_status;
+
+    ExitParams l1{};   // LayerNorm, first layer and GELU
+    l1.in = dev(in);
+    l1.dim = dim;
+    l1.head = Head{head.ln_gamma, head.ln_beta, head.ln_eps, head.w1, head.b1, head.hidden, 0.0f};
+    l1.counters = w.counters;
+    l1.partials = w.partials;
+    l1.n_ctile = ceil_div(head.hidden, kExitCT);
+    l1.n_btile = n_btile;
+    l1.status = dev_status;
+    l1.in_mode = 2;
+    l1.u_in = u;
+    l1.out_mode = 1;
+    l1.hidden_out = hid;
+
+    ExitParams l2{};   // second layer, softmax maximum and exit rule
+    l2.in = dev(in);
+    l2.x = hid;
+    l2.dim = head.hidden;
+    l2.head = Head{nullptr, nullptr, 0.0f, head.w2, head.b2, head.classes, head.tau};
+    l2.exit_mask = exit_mask;
+    l2.logits = logits;
+    l2.max_prob = max_prob;
+    l2.counters = w.counters;
+    l2.partials = w.partials;
+    l2.n_ctile = ceil_div(head.classes, kExitCT);
+    l2.n_btile = n_btile;
+    l2.status = dev_status;
+    l2.in_mode = 1;
+    l2.skip_ln = 1;
+
+    const ProfileEvents ev = take_profile();
+    record(ev.start, s);
+    int rc = cuda_rc(launch_head_pool(dtype, pp, s));
+    if (rc == FUSION_OK) rc = cuda_rc(launch_exit(dtype, l1, s));
+    record(ev.mid, s);
+    if (rc == FUSION_OK) rc = cuda_rc(launch_exit(dtype, l2, s));
+    record(ev.end, s);
+    return rc;
+}
+
 int fusion_token_scores(int dtype, fusion_ragged in, const void *x, int32_t dim, const void *w, float b,
                         float *scores_out, int32_t *dev_status, void *stream) {
     FZ_TRY(check_dtype(dtype));

@@ -24,6 +24,12 @@ struct ExitParams {
     int do_plan;     // run the compaction plan in the last CTA
     PlanArgs plan;
     int *status;
+    // the layers of an MLP exit head (zero for the linear head of the ragged CLS rows)
+    int in_mode;     // 0: CLS rows of the ragged batch x; 1: dense rows x[s] of [B, dim]; 2: dense float32 rows u_in[s]
+    int skip_ln;     // 1: the rows enter the product as they are (no LayerNorm)
+    int out_mode;    // 0: softmax maximum and exit rule; 1: GELU(W u + b) rounded to the dtype into hidden_out
+    const float *u_in;   // [max_batch, dim] for in_mode 2
+    void *hidden_out;    // [max_batch, classes] for out_mode 1
 };
 cudaError_t launch_exit(int dtype, const ExitParams &p, cudaStream_t s);
 size_t exit_smem_bytes(int dtype, int dim);
@@ -40,6 +46,18 @@ struct RouterParams {
     int *status;
 };
 cudaError_t launch_router(int dtype, const RouterParams &p, cudaStream_t s);
+
+// ---- exit-head pooling: the CLS row or the size-weighted mean of the patch rows ----------
+struct PoolParams {
+    Ragged in;
+    const void *x;
+    int dim;
+    const float *sizes;
+    int pool;        // FUSION_POOL_CLS or FUSION_POOL_SPATIAL
+    float *u_out;    // [max_batch, dim]
+    int *status;
+};
+cudaError_t launch_head_pool(int dtype, const PoolParams &p, cudaStream_t s);
 
 // ---- pruning router: linear token scores ------------------------------------------------
 struct ScoreParams {

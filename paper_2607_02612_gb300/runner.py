@@ -94,6 +94,40 @@ def head_tensors(head, dtype: str, device="cuda") -> HeadTensors:
                        torch.from_numpy(np.asarray(head.bias, np.float32)).to(device), float(head.tau))
 
 
+@dataclass
+class MlpHeadTensors:
+    """An MLP exit head on the device (fusion_mlp_head)."""
+    pool: int
+    gamma: torch.Tensor
+    beta: torch.Tensor
+    eps: float
+    w1: torch.Tensor
+    b1: torch.Tensor
+    w2: torch.Tensor
+    b2: torch.Tensor
+    tau: float
+
+    @property
+    def hidden(self) -> int:
+        return int(self.w1.shape[0])
+
+    @property
+    def classes(self) -> int:
+        return int(self.w2.shape[0])
+
+    def c_struct(self) -> fb.fusion_mlp_head:
+        return fb.mlp_head(self.pool, self.gamma, self.beta, self.eps, self.w1, self.b1, self.hidden, self.w2,
+                           self.b2, self.classes, self.tau)
+
+
+def mlp_head_tensors(head, dtype: str, device="cuda") -> MlpHeadTensors:
+    f32 = lambda a: torch.from_numpy(np.asarray(a, np.float32)).to(device)   # noqa: E731
+    return MlpHeadTensors(int(head.pool), tokens_to_torch(head.gamma, dtype, device),
+                          tokens_to_torch(head.beta, dtype, device), float(head.eps),
+                          tokens_to_torch(head.w1, dtype, device), f32(head.b1),
+                          tokens_to_torch(head.w2, dtype, device), f32(head.b2), float(head.tau))
+
+
 class Fusion:
     """Owns a zero-initialised workspace and a device status word; each method
     allocates its outputs and enqueues one C-ABI call on the current stream."""
@@ -103,6 +137,7 @@ class Fusion:
         self.ws_bytes = fb.fusion_workspace_size(max_batch, classes)
         self.workspace = torch.zeros(self.ws_bytes, dtype=torch.uint8, device=self.device)
         self.status = torch.zeros(1, dtype=torch.int32, device=self.device)
+        self._mlp_ws: Optional[torch.Tensor] = None   # scratch of exit_check_mlp, sized at first use
         self.max_batch = max_batch
         self.classes = classes
 
@@ -139,6 +174,20 @@ class Fusion:
         """Prune scores s = w . z + bias of every token row from a linear pruning router (Eq. 8)."""
         o = out if out is not None else torch.zeros(b.max_rows, dtype=torch.float32, device=self.device)
         fb.check(fb.fusion_token_scores(DTYPE_CODE[b.dtype], b.ragged(), b.x, b.dim, w, bias, o, self.status))
+        return o
+
+    def exit_check_mlp(self, b: DeviceBatch, head: "MlpHeadTensors") -> Dict[str, torch.Tensor]:
+        """Exit check with an MLP exit head (SpatialPool or CLS-only), its own scratch."""
+        dev = self.device
+        o = dict(exit_mask=torch.zeros(b.max_batch, dtype=torch.uint8, device=dev),
+                 logits=torch.zeros((b.max_batch, head.classes), dtype=torch.float32, device=dev),
+                 max_prob=torch.zeros(b.max_batch, dtype=torch.float32, device=dev))
+        nbytes = fb.fusion_exit_mlp_workspace_size(b.max_batch, b.dim, head.hidden, head.classes)
+        if self._mlp_ws is None or self._mlp_ws.numel() < nbytes:
+            self._mlp_ws = torch.zeros(nbytes, dtype=torch.uint8, device=dev)
+        fb.check(fb.fusion_exit_check_mlp(DTYPE_CODE[b.dtype], b.ragged(), b.x, b.dim, b.sizes, head.c_struct(),
+                                          o["exit_mask"], o["logits"], o["max_prob"], self._mlp_ws, nbytes,
+                                          self.status))
         return o
 
     def exit_check(self, b: DeviceBatch, head: HeadTensors) -> Dict[str, torch.Tensor]:

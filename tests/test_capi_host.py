@@ -152,7 +152,8 @@ def test_binding_constants_match_header():
         text = f.read()
     defs = dict(re.findall(r"#define\s+(FUSION_[A-Z0-9_]+)\s+(-?\d+)", text))
     for name in ("FUSION_MAX_TOKENS", "FUSION_MAX_DIM", "FUSION_FUSED_PLAN_MAX_BATCH", "FUSION_STAGE_MERGE",
-                 "FUSION_STAGE_EXIT", "FUSION_STAGE_PRUNE", "FUSION_DEV_TIMEOUT"):
+                 "FUSION_STAGE_EXIT", "FUSION_STAGE_PRUNE", "FUSION_DEV_TIMEOUT", "FUSION_POOL_CLS",
+                 "FUSION_POOL_SPATIAL"):
         assert int(defs[name]) == getattr(fb, name), name
 
 
@@ -183,3 +184,32 @@ def test_token_scores_rejects_bad_arguments(lib):
     for kw in (dict(x=None), dict(w=None), dict(scores_out=None), dict(x=FAKE + 4), dict(w=FAKE + 8),
                dict(b=float("nan")), dict(b=float("-inf"))):
         assert call(**kw) == fz.FUSION_ERR_INVALID_ARG, kw
+
+
+def test_exit_check_mlp_rejects_bad_arguments(lib):
+    ws = fz.fusion_exit_mlp_workspace_size(4, 384, 768, 1000)
+    assert ws > fz.fusion_workspace_size(4, 1000)
+    assert fz.fusion_exit_mlp_workspace_size(8, 384, 768, 1000) > ws
+    assert fz.fusion_exit_mlp_workspace_size(4, 384, 1024, 1000) > ws
+
+    def head(**kw):
+        h = dict(pool=fz.FUSION_POOL_SPATIAL, gamma=FAKE, beta=FAKE, eps=1e-6, w1=FAKE, b1=FAKE, hidden=768,
+                 w2=FAKE, b2=FAKE, classes=1000, tau=0.5)
+        h.update(kw)
+        return fz.mlp_head(*h.values())
+
+    def call(**kw):
+        args = dict(dtype=fz.FUSION_BF16, in_=_r(), x=FAKE, dim=384, sizes=FAKE, head=head(), exit_mask=FAKE,
+                    logits=None, max_prob=None, workspace=FAKE, workspace_bytes=ws, dev_status=FAKE, stream=0)
+        args.update(kw)
+        return fz.fusion_exit_check_mlp(*args.values())
+    assert call(dtype=4) == fz.FUSION_ERR_DTYPE
+    assert call(dim=100) == fz.FUSION_ERR_SHAPE
+    assert call(head=head(hidden=100)) == fz.FUSION_ERR_SHAPE
+    assert call(head=head(hidden=2048)) == fz.FUSION_ERR_SHAPE
+    assert call(head=head(classes=0)) == fz.FUSION_ERR_SHAPE
+    for kw in (dict(head=head(pool=2)), dict(sizes=None), dict(x=None), dict(exit_mask=None), dict(x=FAKE + 8),
+               dict(head=head(w1=None)), dict(head=head(b2=None)), dict(head=head(w2=FAKE + 4))):
+        assert call(**kw) == fz.FUSION_ERR_INVALID_ARG, kw
+    assert call(sizes=None, head=head(pool=fz.FUSION_POOL_CLS), workspace=None) == fz.FUSION_ERR_WORKSPACE
+    assert call(workspace_bytes=ws - 1) == fz.FUSION_ERR_WORKSPACE

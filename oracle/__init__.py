@@ -54,6 +54,8 @@ def configure(lib):
     lib.orc_exit_mlp.argtypes = [i32, i32, P, i32, P, P, i32, P, P, dbl, P, P, i32, P, P, i32, dbl,
                                  P, P, P, P, P, P]
     lib.orc_exit_mlp.restype = ctypes.c_int
+    lib.orc_attention.argtypes = [i32, i32, P, i32, i32, P, P, P]
+    lib.orc_attention.restype = ctypes.c_int
     lib.orc_token_scores.restype = ctypes.c_int
     lib.orc_double_to_bf16.argtypes = [dbl]
     lib.orc_double_to_bf16.restype = ctypes.c_uint16
@@ -184,6 +186,24 @@ def exit_mlp(dtype: str, offsets, x, sizes, head) -> Dict[str, np.ndarray]:
                           float(np.float32(head.tau)), _p(mask), _p(logits), _p(maxp), _p(gap), _p(z), _p(hid))
     _check(rc, "exit_mlp")
     return dict(exit_mask=mask, logits=logits, max_prob=maxp, exit_gap=gap, pool=z, hidden=hid)
+
+
+def attention(dtype: str, offsets, qkv, heads: int, sizes=None) -> np.ndarray:
+    """Size-aware (proportional) attention per sample and head over a ragged batch:
+    softmax(q k^T / sqrt(dh) + log s) v.  qkv [rows, 3 * heads * dh] (timm's packed q, k, v);
+    sizes [rows] or None (plain attention).  Returns [rows, heads * dh] float64 (rows outside
+    the samples are 0)."""
+    lib = _load()
+    et = _elem_dtype(dtype)
+    offsets = _c(offsets, np.int32)
+    qkv = _c(qkv, et)
+    rows = qkv.shape[0]
+    dh = qkv.shape[1] // (3 * heads)
+    out = np.zeros((rows, heads * dh), np.float64)
+    sz = None if sizes is None else _c(sizes, np.float32)
+    _check(lib.orc_attention(_DT[dtype], len(offsets) - 1, _p(offsets), heads, dh, _p(qkv),
+                             None if sz is None else _p(sz), _p(out)), "attention")
+    return out
 
 
 def merge_router(dtype: str, offsets, x, w, beta: float, tau_tgt: float, tau_ref: float, ids=None,

@@ -24,6 +24,10 @@
  *   exit (MLP heads)  Sec. III-D, Eq. 6 and Eq. 7 with the paper's two exit heads
  *           (Sec. III-G, Sec. IV-I: a SpatialPool head at block 8, a CLS-only head at block 10,
  *           each a 2-layer MLP): head(z) = W2 GELU(W1 LN(pool(z)) + b1) + b2.
+ *   attention  the block that consumes a compacted batch (Algorithm 1, Block_b): per
+ *           sample and head, softmax(q k^T / sqrt(d_h) + log s_j) v with the size-aware
+ *           (proportional) attention of ToMe, so that a merged token of size s weighs
+ *           like the s tokens it replaced.
  *   scores  Sec. III-E, Eq. 8 (the prune scores' source): s_i = h_b(z_i) with a
  *           linear scoring head, s = w . z + b for every token, rounded once to
  *           float32.
@@ -650,5 +654,58 @@ int orc_exit_mlp(int dtype, int B, const int32_t *offsets, int d, const void *x,
     free(u);
     free(h);
     free(l);
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------------------- */
+/* size-aware attention over a ragged batch (Algorithm 1, Block_b; ToMe)         */
+/* ------------------------------------------------------------------------- */
+/*
+ * qkv [rows, 3, H, dh] row-major (the q, k and v projections of every token, dtype);
+ * sizes [rows] float32, or NULL for plain attention (every size 1).  For every sample,
+ * head h and query row m of the sample:
+ *   l_j = (q_m . k_j) / sqrt(dh) + log(s_j),  p = softmax(l) over the sample's rows,
+ *   out[m, h, :] = sum_j p_j v_j   (double, [rows, H, dh]; rows outside the samples untouched).
+ */
+int orc_attention(int dtype, int B, const int32_t *offsets, int H, int dh, const void *qkv, const float *sizes,
+                  double *out)
+{
+    if (B < 0 || H <= 0 || dh <= 0)
+        return ORC_ERR_ARG;
+    const int64_t rs = (int64_t)3 * H * dh; /* row stride of qkv */
+    const double scale = 1.0 / sqrt((double)dh);
+    for (int i = 0; i < B; ++i) {
+        const int64_t o = offsets[i], n = offsets[i + 1] - offsets[i];
+        double *l = malloc(sizeof(double) * (size_t)(n > 0 ? n : 1));
+        if (!l)
+            return ORC_ERR_NOMEM;
+        for (int h = 0; h < H; ++h) {
+            const int64_t qo = (int64_t)h * dh, ko = (int64_t)(H + h) * dh, vo = (int64_t)(2 * H + h) * dh;
+            for (int64_t m = 0; m < n; ++m) {
+                double lmax = -INFINITY;
+                for (int64_t j = 0; j < n; ++j) {
+                    double dot = 0.0;
+                    for (int e = 0; e < dh; ++e)
+                        dot += load_elem(dtype, qkv, (o + m) * rs + qo + e) * load_elem(dtype, qkv, (o + j) * rs + ko + e);
+                    l[j] = dot * scale + (sizes ? log((double)sizes[o + j]) : 0.0);
+                    if (l[j] > lmax)
+                        lmax = l[j];
+                }
+                double S = 0.0;
+                for (int64_t j = 0; j < n; ++j) {
+                    l[j] = exp(l[j] - lmax);
+                    S += l[j];
+                }
+                double *dst = out + (o + m) * (int64_t)H * dh + (int64_t)h * dh;
+                for (int e = 0; e < dh; ++e) {
+                    double acc = 0.0;
+                    for (int64_t j = 0; j < n; ++j)
+                        acc += l[j] * load_elem(dtype, qkv, (o + j) * rs + vo + e);
+                    dst[e] = acc / S;
+                }
+            }
+        }
+        free(l);
+    }
     return ORC_OK;
 }

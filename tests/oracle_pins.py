@@ -732,6 +732,59 @@ def pin_exit_mlp_special_cases():
     np.testing.assert_array_equal(e["pool"], x[offsets[:-1]].astype(np.float64))
 
 
+def pin_attention_vs_torch():
+    """Size-aware attention against torch float64 scaled_dot_product_attention with log(sizes)
+    as the additive mask (the logit bias of ToMe's proportional attention), per sample and
+    head, both dtypes, with and without sizes."""
+    rng = np.random.default_rng(51)
+    F = torch.nn.functional
+    H, dh = 3, 16
+    Ns = [1, 5, 17, 2, 33]
+    offsets = np.concatenate([[0], np.cumsum(Ns)]).astype(np.int32)
+    T = int(offsets[-1])
+    q32 = (rng.standard_normal((T, 3 * H * dh)) * 1.5).astype(np.float32)
+    sizes = rng.integers(1, 6, T).astype(np.float32)
+    for dtype in ("f32", "bf16"):
+        qs = f32_to_bf16_bits(q32) if dtype == "bf16" else q32
+        qf = (bf16_bits_to_f32(qs) if dtype == "bf16" else q32).astype(np.float64)
+        for sz in (sizes, None):
+            got = oracle.attention(dtype, offsets, qs, H, sz)
+            for i in range(len(Ns)):
+                o, n = offsets[i], offsets[i + 1] - offsets[i]
+                blk = torch.from_numpy(qf[o:o + n].reshape(n, 3, H, dh)).permute(1, 2, 0, 3)   # [3, H, n, dh]
+                mask = torch.zeros(n, n, dtype=torch.float64) if sz is None else \
+                    torch.log(torch.from_numpy(sz[o:o + n].astype(np.float64)))[None, :].expand(n, n)
+                ref = F.scaled_dot_product_attention(blk[0], blk[1], blk[2], attn_mask=mask)   # [H, n, dh]
+                np.testing.assert_allclose(got[o:o + n], ref.permute(1, 0, 2).reshape(n, H * dh).numpy(),
+                                           rtol=1e-12, atol=1e-12)
+
+
+def pin_attention_closed_forms():
+    """A zero query sees equal logits, so proportional attention returns the size-weighted
+    mean of the values; a token present twice with size 1 attends and is attended exactly
+    like one token of size 2 (the property that makes merged tokens of size s stand for the
+    s tokens they replaced); a one-token sample returns its value; no sizes means sizes 1."""
+    rng = np.random.default_rng(52)
+    H, dh = 2, 8
+    x = rng.standard_normal((4, 3 * H * dh)).astype(np.float32)
+    sizes = np.array([1, 3, 2, 5], np.float32)
+    x0 = x.copy()
+    x0[:, :H * dh] = 0.0                                   # q = 0
+    got = oracle.attention("f32", np.array([0, 4], np.int32), x0, H, sizes)
+    v = x0[:, 2 * H * dh:].astype(np.float64)
+    mean = (sizes[:, None].astype(np.float64) * v).sum(0) / sizes.sum()
+    np.testing.assert_allclose(got, np.tile(mean, (4, 1)), rtol=1e-14, atol=1e-14)
+    dup = np.stack([x[0], x[1], x[1]])                     # [t0, t1, t1] sizes 1 vs [t0, t1] sizes (1, 2)
+    a = oracle.attention("f32", np.array([0, 3], np.int32), dup, H, np.ones(3, np.float32))
+    b = oracle.attention("f32", np.array([0, 2], np.int32), x[:2], H, np.array([1, 2], np.float32))
+    np.testing.assert_allclose(a[:2], b, rtol=1e-13, atol=1e-13)
+    np.testing.assert_allclose(a[2], b[1], rtol=1e-13, atol=1e-13)
+    one = oracle.attention("f32", np.array([0, 1], np.int32), x[:1], H, sizes[:1])
+    np.testing.assert_array_equal(one[0], x[0, 2 * H * dh:].astype(np.float64))
+    np.testing.assert_array_equal(oracle.attention("f32", np.array([0, 4], np.int32), x, H, None),
+                                  oracle.attention("f32", np.array([0, 4], np.int32), x, H, np.ones(4, np.float32)))
+
+
 ALL_PINS = [
     pin_bf16_rounding_table,
     pin_bf16_rounding_vs_torch,
@@ -756,4 +809,6 @@ ALL_PINS = [
     pin_scores_special_cases,
     pin_exit_mlp_vs_torch,
     pin_exit_mlp_special_cases,
+    pin_attention_vs_torch,
+    pin_attention_closed_forms,
 ]

@@ -60,6 +60,11 @@ MUTANTS = {
     "mlp_dropped_b1": ("a += (double)b1[k];", ";"),
     "mlp_w1_transposed": ("load_elem(dtype, W1, (int64_t)k * d + j)", "load_elem(dtype, W1, (int64_t)j * H + k)"),
     "mlp_w2_transposed": ("load_elem(dtype, W2, (int64_t)c * H + k)", "load_elem(dtype, W2, (int64_t)k * C + c)"),
+    "attn_no_scale": ("l[j] = dot * scale + ", "l[j] = dot + "),
+    "attn_size_not_log": ("(sizes ? log((double)sizes[o + j]) : 0.0)", "(sizes ? (double)sizes[o + j] : 0.0)"),
+    "attn_k_from_q": ("ko = (int64_t)(H + h) * dh", "ko = (int64_t)h * dh"),
+    "attn_v_from_k": ("vo = (int64_t)(2 * H + h) * dh", "vo = (int64_t)(H + h) * dh"),
+    "attn_not_normalised": ("dst[e] = acc / S;", "dst[e] = acc;"),
     "scores_skip_last_row": ("for (int64_t t = offsets[i]; t < offsets[i + 1]; ++t) {",
                              "for (int64_t t = offsets[i]; t < offsets[i + 1] - 1; ++t) {"),
 }

@@ -409,6 +409,7 @@ def main():
     router = run_router(args, fz, runner, b, dev, flush, peak)
     scores = run_token_scores(args, fz, runner, b, dev, flush, peak)
     exit_mlp = run_exit_mlp(args, fz, runner, b, dev, flush, peak)
+    attention = run_attention(args, fz, runner, b, dev, flush, peak)
 
     # ---- end to end through the C ABI with host buffers -------------------------------
     e2e = run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world)
@@ -436,6 +437,7 @@ def main():
         "router": router,
         "pruning_router": scores,
         "exit_mlp": exit_mlp,
+        "attention": attention,
         "stages": per_stage,
         "kernel_ms_per_step": {"first (exit check or plan)": float(first_ms.sum(axis=1).mean()),
                                "k_image": float(image_ms.sum(axis=1).mean())},
@@ -637,6 +639,60 @@ def run_exit_mlp(args, fz, runner, b, dev, flush, peak):
             "classes": C, "ms": t * 1e3, "ms_pool_and_first_layer": float(np.median(ms1)),
             "algorithmic_bytes": nbytes, "achieved_gbs": nbytes / t / 1e9, "frac": nbytes / t / 1e9 / peak,
             "tflops": flops / t / 1e12, "images_per_s": b.batch / t}
+
+
+def run_attention(args, fz, runner, b, dev, flush, peak):
+    """Size-aware attention (the block consuming a compacted batch) over the step's input batch:
+    DeiT-S heads (6 x 64), random bf16 q, k, v rows, the batch's token sizes, L2 flushed before
+    each launch; bytes = qkv read + output written + sizes; FLOPs = 4 N^2 64 per head and sample
+    (q k^T and p v).  Reported against both the HBM and the tensor roofline."""
+    import torch
+    heads = 6
+    rng = np.random.default_rng(2610)
+    rows = int(b.offsets[-1])
+    qkv = torch.from_numpy(rng.standard_normal((rows, 3 * heads * 64), dtype=np.float32)).to(dev).to(torch.bfloat16)
+    db = runner.device_batch(b.dtype, b.offsets, b.x, b.keys, b.sizes, b.scores, device=dev)
+    fus = runner.Fusion(b.batch, 1, dev)
+    out = torch.empty((rows, heads * 64), dtype=torch.bfloat16, device=dev)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    for e in ev:
+        e.record()
+
+    def one():
+        flush.fill_(3)
+        fz.fusion_profile_next(ev[0], None, ev[1])
+        fus.attention(db, qkv, heads, db.sizes, out=out)
+
+    one()
+    torch.cuda.synchronize()
+    g = None
+    if not args.eager:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            one()
+    run = g.replay if g is not None else one
+    for _ in range(args.warmup):
+        run()
+    ms = []
+    for _ in range(args.steps):
+        run()
+        torch.cuda.synchronize()
+        ms.append(ev[0].elapsed_time(ev[1]))
+    n = np.diff(b.offsets).astype(np.float64)
+    nbytes = rows * (3 * heads * 64 * 2 + heads * 64 * 2 + 4)
+    flops = float(4.0 * 64 * heads * np.sum(n * n))
+    t = float(np.median(ms)) / 1e3
+    tpeak, tsrc = None, None
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            tpeak, tsrc = float(json.load(f)["bf16_tflops"]), "measured (cuBLAS bf16 burst)"
+    except (OSError, ValueError, KeyError):
+        tpeak, tsrc = 1900.0, "fallback"
+    return {"kernel": "k_attn_tc", "batch": b.batch, "heads": heads, "tokens": rows, "ms": t * 1e3,
+            "ms_p10_p90": [float(np.percentile(ms, 10)), float(np.percentile(ms, 90))],
+            "algorithmic_bytes": nbytes, "achieved_gbs": nbytes / t / 1e9, "frac_hbm": nbytes / t / 1e9 / peak,
+            "tflops": flops / t / 1e12, "frac_tensor": flops / t / 1e12 / tpeak, "tensor_peak_tflops": tpeak,
+            "tensor_peak_source": tsrc, "images_per_s": b.batch / t}
 
 
 def run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world):

@@ -93,6 +93,10 @@ extern "C" {
    inside the per-sample kernel; larger ones launch a plan kernel first */
 #define FUSION_FUSED_PLAN_MAX_BATCH 1024
 
+/* Size-aware attention (fusion_attention): head width and the longest sample. */
+#define FUSION_ATTN_HEAD_DIM 64
+#define FUSION_ATTN_MAX_TOKENS 256
+
 /* Pooling of an MLP exit head (fusion_mlp_head.pool). */
 #define FUSION_POOL_CLS 0     /* the CLS row (the paper's CLS-only head, block 10) */
 #define FUSION_POOL_SPATIAL 1 /* size-weighted mean of the patch rows (SpatialPool head, block 8) */
@@ -305,6 +309,27 @@ int fusion_compact(int dtype, fusion_ragged in, const void *x, int32_t dim, cons
 int fusion_merge_router(int dtype, fusion_ragged in, const void *x, int32_t dim, const void *w,
                         float beta, float tau_tgt, float tau_ref, int32_t *r_out, float *m_out,
                         int32_t *dev_status, void *stream);
+
+/*
+ * fusion_attention: the attention of the transformer block that consumes a compacted
+ * batch (Algorithm 1, Block_b), with the size-aware (proportional) attention of ToMe, so
+ * that a merged token of size s weighs like the s tokens it replaced.  For every sample
+ * (rows offsets[i] .. offsets[i+1]-1), head h and query row m of the sample:
+ *   out[m, h, :] = sum_j p_j v_j,  p = softmax_j(q_m . k_j / sqrt(64) + log s_j)
+ * over the sample's rows j (plain attention when sizes is NULL).  tcgen05 tensor cores:
+ * q k^T and p v in bf16 with float32 accumulation, p rounded to bf16 for the second
+ * product, the row sum taken in float32 before that rounding.
+ * dtype: FUSION_BF16 only.  qkv: [max_rows, 3, heads, 64] bf16 row-major (timm's packed
+ * projection output: q, then k, then v, each heads x 64), 16-byte aligned; sizes:
+ * [max_rows] float32 token sizes (> 0) or NULL; out: [max_rows, heads, 64] bf16,
+ * 16-byte aligned; rows outside the samples are not written.
+ * Errors: FUSION_ERR_DTYPE unless bf16; FUSION_ERR_SHAPE for head_dim != 64, heads < 1 or
+ * in.max_tokens > FUSION_ATTN_MAX_TOKENS; FUSION_ERR_INVALID_ARG for NULL or misaligned
+ * pointers; device bits BAD_BATCH, BAD_OFFSETS (that sample is not written), TIMEOUT.
+ * No workspace.
+ */
+int fusion_attention(int dtype, fusion_ragged in, const void *qkv, int32_t heads, int32_t head_dim,
+                     const float *sizes, void *out, int32_t *dev_status, void *stream);
 
 /*
  * fusion_token_scores: the prune scores from a pruning router with a linear

@@ -37,13 +37,15 @@ FUSION_STAGE_PRUNE = 4
 FUSION_MAX_TOKENS = 1024
 FUSION_FUSED_PLAN_MAX_BATCH = 1024
 FUSION_MAX_DIM = 1024
+FUSION_ATTN_HEAD_DIM = 64
+FUSION_ATTN_MAX_TOKENS = 256
 FUSION_POOL_CLS = 0
 FUSION_POOL_SPATIAL = 1
 
 EXPORTED = ("fusion_status_string", "fusion_version", "fusion_profile_next", "fusion_workspace_size",
             "fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune", "fusion_compact",
             "fusion_stage", "fusion_merge_router", "fusion_token_scores", "fusion_exit_mlp_workspace_size",
-            "fusion_exit_check_mlp")
+            "fusion_exit_check_mlp", "fusion_attention")
 
 
 class FusionError(RuntimeError):
@@ -110,9 +112,10 @@ def load(path: Optional[str] = None):
     lib.fusion_exit_mlp_workspace_size.argtypes = [I32, I32, I32, I32]
     lib.fusion_exit_mlp_workspace_size.restype = SZ
     lib.fusion_exit_check_mlp.argtypes = [ctypes.c_int, R, V, I32, V, fusion_mlp_head, V, V, V, V, SZ, V, V]
+    lib.fusion_attention.argtypes = [ctypes.c_int, R, V, I32, I32, V, V, V, V]
     for name in ("fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune",
                  "fusion_compact", "fusion_stage", "fusion_merge_router", "fusion_token_scores",
-                 "fusion_exit_check_mlp"):
+                 "fusion_exit_check_mlp", "fusion_attention"):
         getattr(lib, name).restype = ctypes.c_int
     del I64, F
     if path is None:
@@ -238,6 +241,12 @@ def fusion_exit_check_mlp(dtype, in_, x, dim, sizes, head, exit_mask, logits, ma
     return load().fusion_exit_check_mlp(int(dtype), in_, _ptr(x), int(dim), _ptr(sizes), head, _ptr(exit_mask),
                                         _ptr(logits), _ptr(max_prob), _ptr(workspace), int(workspace_bytes),
                                         _ptr(dev_status), _stream(stream))
+
+
+def fusion_attention(dtype, in_, qkv, heads, head_dim, sizes, out, dev_status, stream=None) -> int:
+    """Size-aware attention per sample and head over a ragged batch (ToMe proportional attention)."""
+    return load().fusion_attention(int(dtype), in_, _ptr(qkv), int(heads), int(head_dim), _ptr(sizes), _ptr(out),
+                                   _ptr(dev_status), _stream(stream))
 
 
 def fusion_prune(dtype, in_, x, dim, sizes, scores, rho, x_out, sizes_out, scores_out, offsets_out,

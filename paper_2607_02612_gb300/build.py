@@ -19,7 +19,7 @@ INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(OUT_DIR, "libfusion.so")
 
-SOURCES = ["fusion_api.cu", "exit.cu", "image.cu", "image_tc.cu", "router.cu", "scores.cu", "pool.cu", "noalloc.cu"]
+SOURCES = ["fusion_api.cu", "exit.cu", "image.cu", "image_tc.cu", "router.cu", "scores.cu", "pool.cu", "attn.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "--expt-relaxed-constexpr", f"-I{INCLUDE}", f"-I{CSRC}"]

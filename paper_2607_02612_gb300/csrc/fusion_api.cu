@@ -455,6 +455,30 @@ int fusion_exit_check_mlp(int dtype, fusion_ragged in, const void *x, int32_t di
     return rc;
 }
 
+int fusion_attention(int dtype, fusion_ragged in, const void *qkv, int32_t heads, int32_t head_dim,
+                     const float *sizes, void *out, int32_t *dev_status, void *stream) {
+    FZ_TRY(check_dtype(dtype));
+    if (dtype != FUSION_BF16) return FUSION_ERR_DTYPE;
+    FZ_TRY(check_ragged(in));
+    if (head_dim != FUSION_ATTN_HEAD_DIM || heads < 1 || heads > 64 || in.max_tokens > FUSION_ATTN_MAX_TOKENS)
+        return FUSION_ERR_SHAPE;
+    if (!qkv || !out || !aligned16(qkv) || !aligned16(out)) return FUSION_ERR_INVALID_ARG;
+    AttnParams p{};
+    p.in = dev(in);
+    p.qkv = qkv;
+    p.heads = heads;
+    p.sizes = sizes;
+    p.out = out;
+    p.status = dev_status;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const ProfileEvents ev = take_profile();
+    record(ev.start, s);
+    record(ev.mid, s);
+    const int rc = cuda_rc(launch_attention(p, s));
+    record(ev.end, s);
+    return rc;
+}
+
 int fusion_token_scores(int dtype, fusion_ragged in, const void *x, int32_t dim, const void *w, float b,
                         float *scores_out, int32_t *dev_status, void *stream) {
     FZ_TRY(check_dtype(dtype));

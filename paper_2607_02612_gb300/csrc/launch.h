@@ -59,6 +59,23 @@ struct PoolParams {
 };
 cudaError_t launch_head_pool(int dtype, const PoolParams &p, cudaStream_t s);
 
+// ---- size-aware attention over a ragged batch ---------------------------------------------------
+struct AttnParams {
+    Ragged in;
+    const void *qkv;       // [max_rows, 3, heads, 64] bf16
+    int heads;
+    const float *sizes;    // [max_rows] or NULL (plain attention)
+    void *out;             // [max_rows, heads, 64] bf16
+    int *status;
+    uint32_t u_bytes;      // set by the launcher (shared-memory geometry)
+    uint32_t tmem_cols;
+};
+struct AttnGeometry {
+    uint32_t u_bytes, smem, tmem_cols;
+};
+AttnGeometry attn_geometry(int max_tokens);
+cudaError_t launch_attention(const AttnParams &p, cudaStream_t s);
+
 // ---- pruning router: linear token scores ------------------------------------------------
 struct ScoreParams {
     Ragged in;

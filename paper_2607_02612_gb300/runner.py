@@ -190,6 +190,16 @@ class Fusion:
                                           self.status))
         return o
 
+    def attention(self, b: DeviceBatch, qkv: torch.Tensor, heads: int, sizes: Optional[torch.Tensor] = None,
+                  out: Optional[torch.Tensor] = None) -> torch.Tensor:
+        """Size-aware attention of the batch's samples: qkv [max_rows, 3 * heads * 64] bf16, sizes
+        [max_rows] (None: plain attention); returns [max_rows, heads * 64] bf16."""
+        o = out if out is not None else torch.zeros((b.max_rows, heads * fb.FUSION_ATTN_HEAD_DIM),
+                                                    dtype=torch.bfloat16, device=self.device)
+        fb.check(fb.fusion_attention(DTYPE_CODE["bf16"], b.ragged(), qkv, heads, fb.FUSION_ATTN_HEAD_DIM, sizes, o,
+                                     self.status))
+        return o
+
     def exit_check(self, b: DeviceBatch, head: HeadTensors) -> Dict[str, torch.Tensor]:
         dev = self.device
         o = dict(exit_mask=torch.zeros(b.max_batch, dtype=torch.uint8, device=dev),

@@ -153,7 +153,7 @@ def test_binding_constants_match_header():
     defs = dict(re.findall(r"#define\s+(FUSION_[A-Z0-9_]+)\s+(-?\d+)", text))
     for name in ("FUSION_MAX_TOKENS", "FUSION_MAX_DIM", "FUSION_FUSED_PLAN_MAX_BATCH", "FUSION_STAGE_MERGE",
                  "FUSION_STAGE_EXIT", "FUSION_STAGE_PRUNE", "FUSION_DEV_TIMEOUT", "FUSION_POOL_CLS",
-                 "FUSION_POOL_SPATIAL"):
+                 "FUSION_POOL_SPATIAL", "FUSION_ATTN_HEAD_DIM", "FUSION_ATTN_MAX_TOKENS"):
         assert int(defs[name]) == getattr(fb, name), name
 
 
@@ -213,3 +213,19 @@ def test_exit_check_mlp_rejects_bad_arguments(lib):
         assert call(**kw) == fz.FUSION_ERR_INVALID_ARG, kw
     assert call(sizes=None, head=head(pool=fz.FUSION_POOL_CLS), workspace=None) == fz.FUSION_ERR_WORKSPACE
     assert call(workspace_bytes=ws - 1) == fz.FUSION_ERR_WORKSPACE
+
+
+def test_attention_rejects_bad_arguments(lib):
+    def call(**kw):
+        args = dict(dtype=fz.FUSION_BF16, in_=_r(max_tokens=197), qkv=FAKE, heads=6, head_dim=64, sizes=None,
+                    out=FAKE, dev_status=FAKE, stream=0)
+        args.update(kw)
+        return fz.fusion_attention(*args.values())
+    assert call(dtype=fz.FUSION_F32) == fz.FUSION_ERR_DTYPE
+    assert call(dtype=9) == fz.FUSION_ERR_DTYPE
+    assert call(head_dim=32) == fz.FUSION_ERR_SHAPE
+    assert call(heads=0) == fz.FUSION_ERR_SHAPE
+    assert call(in_=_r(max_tokens=257)) == fz.FUSION_ERR_SHAPE
+    assert call(in_=_r(offsets=None)) == fz.FUSION_ERR_INVALID_ARG
+    for kw in (dict(qkv=None), dict(out=None), dict(qkv=FAKE + 2), dict(out=FAKE + 8)):
+        assert call(**kw) == fz.FUSION_ERR_INVALID_ARG, kw

@@ -10,13 +10,16 @@
 // operands; V, rows of keys with the dims contiguous, is the MN-major B operand of the second
 // product as it lies (8-key swizzle atoms 1024 bytes apart); its rows past the sample are
 // zeroed once it has landed.  Per query tile t: S_t = Q_t K^T (M = 128, N = tokens
-// rounded up to 16, K = 64) accumulates in tensor-memory columns [256 t, 256 t + N); warps
-// 4t..4t+3 then take one row each per thread: logits scaled by log2(e) / sqrt(dh) plus
-// log2(s_j), masked past the sample, the row maximum, exp2 (ex2.approx), the row sum, and the unnormalised
-// probabilities P_t as bf16 into shared memory (swizzled K-major again, over the dead Q and K
-// tiles).  O_t = P_t V (M = 128, N = 64, K = tokens rounded up to 16) accumulates over the first
-// 64 columns of S_t's region; the epilogue divides each row by its sum and stores bf16.  P is
-// rounded to bf16 (the operand type of the second product); the sum is taken before that.
+// rounded up to 16, K = 64) accumulates in tensor-memory columns [0, N);
+// warp w and warp w + 4 share the rows of lane quadrant w, each taking half of the columns
+// (maxima and sums meet in shared memory): logits scaled by log2(e) / sqrt(dh) plus
+// log2(s_j), masked past the sample, the row maximum, exp2 (ex2.approx), the row sum, and the
+// unnormalised probabilities P_t as bf16 pairs written back over S's first columns; O_t = P_t V
+// (M = 128, N = 64, K = tokens rounded up to 16, A = P from tensor memory) accumulates in
+// columns [128, 192); the epilogue divides each row by its sum and stores bf16.  P is rounded to
+// bf16 (the operand type of the second product); the sum is taken before that.  Without a P
+// buffer a CTA needs Q, K and V only (84 KB for 197 tokens) and 256 tensor-memory columns, so
+// two CTAs share an SM; the query tiles of a sample run one after the other.
 //
 // Every wait on an mbarrier is bounded; on a timeout the CTA raises FUSION_DEV_TIMEOUT, skips
 // its outputs, waits (bounded) for the operations it started and frees its tensor memory.
@@ -30,6 +33,7 @@ constexpr int kAttnThreads = 256;
 constexpr int kAttnDh = 64;
 constexpr int kAttnMaxN = 256;
 constexpr uint32_t kQTileBytes = 128 * 128;   // 128 rows x one K-block of 64 bf16
+constexpr uint32_t kAttnTmemCols = 256;       // S (<= 256 columns); P over its first half; O at 128
 
 __device__ __forceinline__ float ex2(float x) {   // 2^x, one MUFU instruction (2^-inf = 0)
     float y;
@@ -41,14 +45,29 @@ struct AttnMaps {
     CUtensorMap b32, b8;   // qkv rows, boxes of 64 dims x 32 / 8 rows, 128-byte swizzle
 };
 
-__global__ void __launch_bounds__(kAttnThreads, 1)
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8]) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(r[0]),
+                 "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+                 : "memory");
+}
+// D (tensor memory) += A (tensor memory, 128 lanes x 16 bf16 packed in 8 columns) x B (shared memory).
+__device__ __forceinline__ void umma_bf16_ts(uint32_t tmem_d, uint32_t tmem_a, uint64_t bdesc, uint32_t idesc,
+                                             uint32_t accumulate) {
+    asm volatile(
+        "{ .reg .pred p; setp.ne.b32 p, %4, 0; tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p; }" ::"r"(tmem_d),
+        "r"(tmem_a), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+__global__ void __launch_bounds__(kAttnThreads, 2)
     k_attn_tc(const __grid_constant__ AttnMaps maps, AttnParams p) {
     extern __shared__ unsigned char sm_raw[];
     unsigned char *sm = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~uintptr_t(1023));
     __shared__ __align__(8) unsigned long long bar_ld, bar_s, bar_o;
     __shared__ uint32_t tmem_base;
-    __shared__ int s_fail, s_issued;   // s_issued: 1 = the products S were issued, 2 = also O
+    __shared__ int s_fail, s_issued;   // s_issued: operations started (for the drain on a timeout)
     __shared__ float lsz[kAttnMaxN];   // log2 of the key sizes
+    __shared__ float red[2][128];      // the two column halves' row maxima, then row sums
 
     const int tid = threadIdx.x, warp = tid >> 5;
     const int h = blockIdx.x, i = blockIdx.y;
@@ -66,14 +85,13 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     const int H = p.heads;
     const int npad = (n + 15) & ~15;              // keys rounded up to the MMA granularity
     const int T = (n + 127) >> 7;                 // query tiles
-    const int nkb = (npad + 63) >> 6;             // K-blocks of 64 keys in P and V^T
-    unsigned char *U = sm;                        // Q tiles and K, later the P tiles
-    unsigned char *Kr = U + (size_t)T * kQTileBytes;
-    unsigned char *Vr = sm + p.u_bytes;           // V rows (MN-major B operand)
+    unsigned char *Q = sm;                        // T tiles of 128 rows
+    unsigned char *Kr = sm + (size_t)T * kQTileBytes;
+    unsigned char *Vr = Kr + (size_t)npad * 128;  // V rows (MN-major B operand)
 
     if (warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(&tmem_base)),
-                     "r"(p.tmem_cols)
+                     "r"(kAttnTmemCols)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
@@ -88,7 +106,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     }
     __syncthreads();
 
-    // ---- loads: K rows and the query tiles by TMA (rows rounded up to 8) --------------------
+    // ---- loads: the query tiles, K and V by TMA (rows rounded up to 8) --------------------------
     if (tid == 0) {
         const int rk = (n + 7) & ~7;
         uint32_t bytes = 2u * (uint32_t)rk * 128u;
@@ -99,167 +117,172 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             for (; r + 32 <= cnt; r += 32) tma_load_2d(smem_addr(dst + r * 128), &maps.b32, x, y0 + r, smem_addr(&bar_ld));
             for (; r < cnt; r += 8) tma_load_2d(smem_addr(dst + r * 128), &maps.b8, x, y0 + r, smem_addr(&bar_ld));
         };
+        for (int t = 0; t < T; ++t) rows(Q + (size_t)t * kQTileBytes, h * kAttnDh, o0 + 128 * t, (min(128, n - 128 * t) + 7) & ~7);
         rows(Kr, (H + h) * kAttnDh, o0, rk);
         rows(Vr, (2 * H + h) * kAttnDh, o0, rk);
-        for (int t = 0; t < T; ++t) rows(U + (size_t)t * kQTileBytes, h * kAttnDh, o0 + 128 * t, (min(128, n - 128 * t) + 7) & ~7);
+        s_issued = 1;
     }
-    // ---- key log-sizes; once V has landed, its rows past the sample are zeroed ----------------
     for (int j = tid; j < npad; j += kAttnThreads)
         lsz[j] = j < n ? (p.sizes ? log2f(p.sizes[o0 + j]) : 0.0f) : 0.0f;
-    __syncthreads();
-    const uint32_t tmem = tmem_base;
-
-    // ---- S_t = Q_t K^T ----------------------------------------------------------------------
-    if (tid == 0) {
-        if (mbar_wait(smem_addr(&bar_ld), 0)) {
-            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(npad >> 3) << 17) | (8u << 24);
-            for (int t = 0; t < T; ++t)
-#pragma unroll
-                for (int k = 0; k < 4; ++k)
-                    umma_bf16(tmem + 256u * t, sw128_desc(smem_addr(U + (size_t)t * kQTileBytes) + k * 32),
-                              sw128_desc(smem_addr(Kr) + k * 32), idesc, k ? 1u : 0u);
-            umma_commit(smem_addr(&bar_s));
-            s_issued = 1;
-        } else {
-            s_fail = 1;
-        }
-    }
+    if (tid == 0 && !mbar_wait(smem_addr(&bar_ld), 0)) s_fail = 1;
     __syncthreads();
     // V rows n .. npad-1 (another sample's rows or stale memory) read as zero in P V
-    if (s_fail == 0 && npad > n) {
+    if (s_fail == 0)
         for (int c = tid; c < (npad - n) * 8; c += kAttnThreads)
             reinterpret_cast<uint4 *>(Vr + (size_t)n * 128)[c] = make_uint4(0u, 0u, 0u, 0u);
-    }
-    if (s_fail == 0 && !mbar_wait(smem_addr(&bar_s), 0)) atomicOr(&s_fail, 2);
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // visible to the tensor core
     __syncthreads();
 
-    // ---- softmax rows: warps 4t .. 4t + 3 take tile t, one row per thread --------------------
-    const int t = warp >> 2;
-    const int r = tid & 127;   // row of the tile = tensor-memory lane
-    const int m = 128 * t + r; // query row of the sample
-    const uint32_t lane_addr = tmem + 256u * t + ((uint32_t)((warp & 3) * 32) << 16);
+    const uint32_t tmem = tmem_base;
+    const int half = warp >> 2;                 // column half of the row
+    const int r = tid & 127;                    // row of the tile = tensor-memory lane
+    const uint32_t lane_addr = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+    const int nch = npad >> 4;                  // 16-column chunks of S
+    const int cA = (nch + 1) >> 1;              // chunks [0, cA) to half 0, [cA, nch) to half 1
+    const int c_lo = half ? cA : 0, c_hi = half ? nch : cA;
     constexpr float kScale2 = 0.18033688011112042f;   // log2(e) / sqrt(64)
-    float lsum = 0.0f;
-    if (s_fail == 0 && t < T) {   // warp-uniform: every lane takes part in the tensor-memory loads
-        float mx = -INFINITY;
-        for (int c0 = 0; c0 < npad; c0 += 16) {
-            uint32_t v[16];
-            tmem_ld16(lane_addr + (uint32_t)c0, v);
-            if (c0 + 16 <= n) {
-#pragma unroll
-                for (int e = 0; e < 16; ++e) mx = fmaxf(mx, fmaf(__uint_as_float(v[e]), kScale2, lsz[c0 + e]));
-            } else {
-#pragma unroll
-                for (int e = 0; e < 16; ++e)
-                    if (c0 + e < n) mx = fmaxf(mx, fmaf(__uint_as_float(v[e]), kScale2, lsz[c0 + e]));
-            }
-        }
-        unsigned char *P = U + (size_t)t * nkb * kQTileBytes;
-        for (int c0 = 0; c0 < npad; c0 += 16) {
-            uint32_t v[16];
-            tmem_ld16(lane_addr + (uint32_t)c0, v);
-            float pr[16];
-#pragma unroll
-            for (int e = 0; e < 16; ++e) pr[e] = ex2(fmaf(__uint_as_float(v[e]), kScale2, lsz[c0 + e]) - mx);
-            if (c0 + 16 > n) {
-#pragma unroll
-                for (int e = 0; e < 16; ++e)
-                    if (c0 + e >= n) pr[e] = 0.0f;
-            }
-            uint32_t pk[8];
-#pragma unroll
-            for (int e = 0; e < 16; e += 2) {
-                lsum += pr[e] + pr[e + 1];
-                const __nv_bfloat162 b2 = __floats2bfloat162_rn(pr[e], pr[e + 1]);
-                pk[e >> 1] = *reinterpret_cast<const uint32_t *>(&b2);
-            }
-            unsigned char *blk = P + (size_t)(c0 >> 6) * kQTileBytes + r * 128;
-            const int cc = (c0 & 63) >> 3;
-            *reinterpret_cast<uint4 *>(blk + ((cc ^ (r & 7)) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-            *reinterpret_cast<uint4 *>(blk + (((cc + 1) ^ (r & 7)) << 4)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-        }
-    }
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // P visible to the tensor core
-    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-    __syncthreads();
+    const uint32_t idesc_s = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(npad >> 3) << 17) | (8u << 24);
+    // B = V as it lies: MN-major (bit 16), 8-key swizzle atoms 1024 bytes apart
+    const uint32_t idesc_o =
+        (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) | ((uint32_t)(kAttnDh >> 3) << 17) | (8u << 24);
 
-    // ---- O_t = P_t V over the first 64 columns of S_t ------------------------------------------
-    if (tid == 0 && s_fail == 0) {
+    bool stop = s_fail != 0;   // read between two barriers: the same in every thread
+    for (int t = 0; t < T && !stop; ++t) {
+        // ---- S = Q_t K^T into columns [0, npad) ---------------------------------------------
+        if (tid == 0) {
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+                umma_bf16(tmem, sw128_desc(smem_addr(Q + (size_t)t * kQTileBytes) + k * 32), sw128_desc(smem_addr(Kr) + k * 32),
+                          idesc_s, k ? 1u : 0u);
+            umma_commit(smem_addr(&bar_s));
+            s_issued = 2 + 2 * t;
+        }
+        if (!mbar_wait(smem_addr(&bar_s), (uint32_t)t & 1u)) atomicOr(&s_fail, 2);
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        // B = V as it lies: MN-major (bit 16), 8-key swizzle atoms 1024 bytes apart
-        const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) | ((uint32_t)(kAttnDh >> 3) << 17) |
-                               (8u << 24);
-        for (int tt = 0; tt < T; ++tt) {
-            const uint32_t pa = smem_addr(U + (size_t)tt * nkb * kQTileBytes);
-            for (int kk = 0; kk < npad / 16; ++kk)
-                umma_bf16(tmem + 256u * tt, sw128_desc(pa + (kk >> 2) * kQTileBytes + (kk & 3) * 32),
-                          sw128_desc(smem_addr(Vr) + kk * 2048u), idesc, kk ? 1u : 0u);
-        }
-        umma_commit(smem_addr(&bar_o));
-        s_issued = 2;
-    }
-    __syncthreads();
-    if (s_fail == 0 && !mbar_wait(smem_addr(&bar_o), 0)) atomicOr(&s_fail, 4);
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    __syncthreads();
-
-    // ---- epilogue: O / row sum -> bf16 --------------------------------------------------------
-    if (s_fail == 0 && t < T) {
-        uint32_t o[64];
+        const bool rows_here = 128 * t + 32 * (warp & 3) < n;   // warp-uniform: a warp of rows past the sample idles
+        // ---- row maximum over this half's columns ----------------------------------------------
+        float mx = -INFINITY;
+        if (rows_here) {
+            for (int c = c_lo; c < c_hi; ++c) {
+                uint32_t v[16];
+                tmem_ld16(lane_addr + (uint32_t)(16 * c), v);
+                if (16 * c + 16 <= n) {
 #pragma unroll
-        for (int c0 = 0; c0 < 64; c0 += 16) tmem_ld16(lane_addr + (uint32_t)c0, *reinterpret_cast<uint32_t(*)[16]>(o + c0));
-        if (m < n) {
-            const float inv = 1.0f / lsum;
-            uint4 *dst = reinterpret_cast<uint4 *>(reinterpret_cast<__nv_bfloat16 *>(p.out) +
-                                                   (size_t)(o0 + m) * H * kAttnDh + (size_t)h * kAttnDh);
+                    for (int e = 0; e < 16; ++e) mx = fmaxf(mx, fmaf(__uint_as_float(v[e]), kScale2, lsz[16 * c + e]));
+                } else {
 #pragma unroll
-            for (int c = 0; c < 8; ++c) {
-                uint32_t w[4];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const __nv_bfloat162 b2 = __floats2bfloat162_rn(__uint_as_float(o[8 * c + 2 * e]) * inv,
-                                                                    __uint_as_float(o[8 * c + 2 * e + 1]) * inv);
-                    w[e] = *reinterpret_cast<const uint32_t *>(&b2);
+                    for (int e = 0; e < 16; ++e)
+                        if (16 * c + e < n) mx = fmaxf(mx, fmaf(__uint_as_float(v[e]), kScale2, lsz[16 * c + e]));
                 }
-                dst[c] = make_uint4(w[0], w[1], w[2], w[3]);
             }
         }
+        red[half][r] = mx;
+        __syncthreads();
+        mx = fmaxf(red[0][r], red[1][r]);
+        // ---- P = 2^(logit - max) as bf16 pairs, and the row sum; P goes over S's first columns once
+        // ---- every S column of the row has been read (the other half reads some of them) ----------
+        float lsum = 0.0f;
+        uint32_t pk[8][8];   // this half's chunks, at most 8
+        if (rows_here) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const int c = c_lo + q;
+                if (c < c_hi) {
+                    uint32_t v[16];
+                    tmem_ld16(lane_addr + (uint32_t)(16 * c), v);
+                    float pr[16];
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) pr[e] = ex2(fmaf(__uint_as_float(v[e]), kScale2, lsz[16 * c + e]) - mx);
+                    if (16 * c + 16 > n) {
+#pragma unroll
+                        for (int e = 0; e < 16; ++e)
+                            if (16 * c + e >= n) pr[e] = 0.0f;
+                    }
+#pragma unroll
+                    for (int e = 0; e < 16; e += 2) {
+                        lsum += pr[e] + pr[e + 1];
+                        const __nv_bfloat162 b2 = __floats2bfloat162_rn(pr[e], pr[e + 1]);
+                        pk[q][e >> 1] = *reinterpret_cast<const uint32_t *>(&b2);
+                    }
+                }
+            }
+        }
+        __syncthreads();   // every S column read; both halves' maxima read
+        if (rows_here) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                if (c_lo + q < c_hi) tmem_st8(lane_addr + (uint32_t)(8 * (c_lo + q)), pk[q]);
+            asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+        }
+        red[half][r] = lsum;
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncthreads();
+        lsum = red[0][r] + red[1][r];
+        // ---- O = P V into columns [128, 192) ---------------------------------------------------
+        const bool ok_s = s_fail == 0;   // the S waits' outcome, after the barrier above
+        if (tid == 0 && ok_s) {
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            for (int kk = 0; kk < npad / 16; ++kk)
+                umma_bf16_ts(tmem + 128u, tmem + 8u * kk, sw128_desc(smem_addr(Vr) + kk * 2048u), idesc_o, kk ? 1u : 0u);
+            umma_commit(smem_addr(&bar_o));
+            s_issued = 3 + 2 * t;
+        }
+        if (ok_s && !mbar_wait(smem_addr(&bar_o), (uint32_t)t & 1u)) atomicOr(&s_fail, 4);
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        // ---- epilogue: this half's 32 dims of O / row sum -> bf16 -------------------------------
+        if (rows_here) {
+            uint32_t o[32];
+            tmem_ld16(lane_addr + 128u + 32u * half, *reinterpret_cast<uint32_t(*)[16]>(o));
+            tmem_ld16(lane_addr + 144u + 32u * half, *reinterpret_cast<uint32_t(*)[16]>(o + 16));
+            const int m = 128 * t + r;
+            if (m < n && s_fail == 0) {
+                const float inv = 1.0f / lsum;
+                uint4 *dst = reinterpret_cast<uint4 *>(reinterpret_cast<__nv_bfloat16 *>(p.out) +
+                                                       (size_t)(o0 + m) * H * kAttnDh + (size_t)h * kAttnDh + 32 * half);
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    uint32_t w[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const __nv_bfloat162 b2 = __floats2bfloat162_rn(__uint_as_float(o[8 * c + 2 * e]) * inv,
+                                                                        __uint_as_float(o[8 * c + 2 * e + 1]) * inv);
+                        w[e] = *reinterpret_cast<const uint32_t *>(&b2);
+                    }
+                    dst[c] = make_uint4(w[0], w[1], w[2], w[3]);
+                }
+            }
+        }
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncthreads();   // O read and the sums consumed before the next tile's S overwrites them
+        stop = s_fail != 0;
+        __syncthreads();   // nobody writes s_fail again before every thread has read it
     }
     if (tid == 0 && s_fail != 0) {   // let everything this CTA started finish before it leaves
         raise_status(p.status, FUSION_DEV_TIMEOUT);
         mbar_wait(smem_addr(&bar_ld), 0);
-        if (s_issued >= 1) mbar_wait(smem_addr(&bar_s), 0);
-        if (s_issued >= 2) mbar_wait(smem_addr(&bar_o), 0);
+        const int k = s_issued;   // 2 + 2t: S of tile t issued; 3 + 2t: also its O
+        if (k >= 2) mbar_wait(smem_addr(&bar_s), (uint32_t)((k - 2) >> 1) & 1u);
+        if (k >= 3 && (k & 1)) mbar_wait(smem_addr(&bar_o), (uint32_t)((k - 3) >> 1) & 1u);
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
     if (warp == 0)
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(p.tmem_cols) : "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kAttnTmemCols) : "memory");
 }
 
 }  // namespace
 
-AttnGeometry attn_geometry(int max_tokens) {
-    AttnGeometry g{};
-    const int npad = (max_tokens + 15) & ~15, T = (max_tokens + 127) >> 7, nkb = (npad + 63) >> 6;
-    const uint32_t qk = (uint32_t)T * kQTileBytes + (uint32_t)npad * 128u;
-    const uint32_t pt = (uint32_t)T * (uint32_t)nkb * kQTileBytes;
-    g.u_bytes = ((qk > pt ? qk : pt) + 1023u) & ~1023u;
-    g.smem = 1024u + g.u_bytes + (uint32_t)npad * 128u;
-    g.tmem_cols = 256u * (uint32_t)T;
-    return g;
+size_t attn_smem_bytes(int max_tokens) {
+    const int npad = (max_tokens + 15) & ~15, T = (max_tokens + 127) >> 7;
+    return 1024u + (size_t)T * kQTileBytes + 2u * (size_t)npad * 128u;   // alignment, Q tiles, K, V
 }
 
 cudaError_t launch_attention(const AttnParams &p, cudaStream_t s) {
     if (p.in.max_batch == 0 || p.heads == 0) return cudaSuccess;
     EncodeTiledFn enc = encode_fn();
     if (!enc) return cudaErrorNotSupported;
-    const AttnGeometry g = attn_geometry(p.in.max_tokens);
-    AttnParams q = p;
-    q.u_bytes = g.u_bytes;
-    q.tmem_cols = g.tmem_cols;
+    const size_t smem = attn_smem_bytes(p.in.max_tokens);
     AttnMaps maps;
     for (int b = 0; b < 2; ++b) {
         cuuint64_t dims[2] = {(cuuint64_t)3 * p.heads * kAttnDh, (cuuint64_t)p.in.max_rows};
@@ -271,9 +294,9 @@ cudaError_t launch_attention(const AttnParams &p, cudaStream_t s) {
                 CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
     }
-    cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)g.smem);
+    cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    k_attn_tc<<<dim3((unsigned)p.heads, (unsigned)p.in.max_batch), kAttnThreads, g.smem, s>>>(maps, q);
+    k_attn_tc<<<dim3((unsigned)p.heads, (unsigned)p.in.max_batch), kAttnThreads, smem, s>>>(maps, p);
     return cudaGetLastError();
 }
 

@@ -67,13 +67,8 @@ struct AttnParams {
     const float *sizes;    // [max_rows] or NULL (plain attention)
     void *out;             // [max_rows, heads, 64] bf16
     int *status;
-    uint32_t u_bytes;      // set by the launcher (shared-memory geometry)
-    uint32_t tmem_cols;
 };
-struct AttnGeometry {
-    uint32_t u_bytes, smem, tmem_cols;
-};
-AttnGeometry attn_geometry(int max_tokens);
+size_t attn_smem_bytes(int max_tokens);
 cudaError_t launch_attention(const AttnParams &p, cudaStream_t s);
 
 // ---- pruning router: linear token scores ------------------------------------------------

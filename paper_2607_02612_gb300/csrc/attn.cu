@@ -13,7 +13,9 @@
 // rounded up to 16, K = 64) accumulates in tensor-memory columns [0, N);
 // warp w and warp w + 4 share the rows of lane quadrant w, each taking half of the columns
 // (maxima and sums meet in shared memory): logits scaled by log2(e) / sqrt(dh) plus
-// log2(s_j), masked past the sample, the row maximum, exp2 (ex2.approx), the row sum, and the
+// log2(s_j), masked past the sample, shifted by max_j S scale + max_j log2 s_j (an upper bound of
+// the row maximum within log2(max s / min s), so sizes within a factor 2^100 of each other keep
+// every probability a normal float), exp2 (ex2.approx), the row sum, and the
 // unnormalised probabilities P_t as bf16 pairs written back over S's first columns; O_t = P_t V
 // (M = 128, N = 64, K = tokens rounded up to 16, A = P from tensor memory) accumulates in
 // columns [128, 192); the epilogue divides each row by its sum and stores bf16.  P is rounded to
@@ -45,6 +47,15 @@ struct AttnMaps {
     CUtensorMap b32, b8;   // qkv rows, boxes of 64 dims x 32 / 8 rows, 128-byte swizzle
 };
 
+// The two warps that share lane quadrant w (warps w and w + 4) meet at named barrier 1 + w.
+__device__ __forceinline__ void pair_sync(int warp) {
+    switch (warp & 3) {   // literal ids: the kernel reserves barriers 0..4 only
+    case 0: asm volatile("bar.sync 1, 64;" ::: "memory"); break;
+    case 1: asm volatile("bar.sync 2, 64;" ::: "memory"); break;
+    case 2: asm volatile("bar.sync 3, 64;" ::: "memory"); break;
+    default: asm volatile("bar.sync 4, 64;" ::: "memory"); break;
+    }
+}
 __device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8]) {
     asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(r[0]),
                  "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
@@ -68,6 +79,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     __shared__ int s_fail, s_issued;   // s_issued: operations started (for the drain on a timeout)
     __shared__ float lsz[kAttnMaxN];   // log2 of the key sizes
     __shared__ float red[2][128];      // the two column halves' row maxima, then row sums
+    __shared__ float s_lszmax;         // max_j log2 s_j
 
     const int tid = threadIdx.x, warp = tid >> 5;
     const int h = blockIdx.x, i = blockIdx.y;
@@ -126,6 +138,13 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         lsz[j] = j < n ? (p.sizes ? log2f(p.sizes[o0 + j]) : 0.0f) : 0.0f;
     if (tid == 0 && !mbar_wait(smem_addr(&bar_ld), 0)) s_fail = 1;
     __syncthreads();
+    if (warp == 0) {   // max_j log2 s_j over the sample
+        float lm = -INFINITY;
+        for (int j = threadIdx.x; j < n; j += 32) lm = fmaxf(lm, lsz[j]);
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) lm = fmaxf(lm, __shfl_xor_sync(0xFFFFFFFFu, lm, o));
+        if (threadIdx.x == 0) s_lszmax = lm;
+    }
     // V rows n .. npad-1 (another sample's rows or stale memory) read as zero in P V
     if (s_fail == 0)
         for (int c = tid; c < (npad - n) * 8; c += kAttnThreads)
@@ -161,7 +180,8 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         if (!mbar_wait(smem_addr(&bar_s), (uint32_t)t & 1u)) atomicOr(&s_fail, 2);
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         const bool rows_here = 128 * t + 32 * (warp & 3) < n;   // warp-uniform: a warp of rows past the sample idles
-        // ---- row maximum over this half's columns ----------------------------------------------
+        // ---- the softmax shift: max_j S * scale + max_j log2 s_j, an upper bound of the row's largest
+        // ---- logit by at most log2(max s / min s) (the result does not depend on the shift) -------
         float mx = -INFINITY;
         if (rows_here) {
             for (int c = c_lo; c < c_hi; ++c) {
@@ -169,17 +189,17 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
                 tmem_ld16(lane_addr + (uint32_t)(16 * c), v);
                 if (16 * c + 16 <= n) {
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) mx = fmaxf(mx, fmaf(__uint_as_float(v[e]), kScale2, lsz[16 * c + e]));
+                    for (int e = 0; e < 16; ++e) mx = fmaxf(mx, __uint_as_float(v[e]));
                 } else {
 #pragma unroll
                     for (int e = 0; e < 16; ++e)
-                        if (16 * c + e < n) mx = fmaxf(mx, fmaf(__uint_as_float(v[e]), kScale2, lsz[16 * c + e]));
+                        if (16 * c + e < n) mx = fmaxf(mx, __uint_as_float(v[e]));
                 }
             }
         }
         red[half][r] = mx;
-        __syncthreads();
-        mx = fmaxf(red[0][r], red[1][r]);
+        pair_sync(warp);
+        mx = fmaf(fmaxf(red[0][r], red[1][r]), kScale2, s_lszmax);
         // ---- P = 2^(logit - max) as bf16 pairs, and the row sum; P goes over S's first columns once
         // ---- every S column of the row has been read (the other half reads some of them) ----------
         float lsum = 0.0f;
@@ -208,7 +228,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
                 }
             }
         }
-        __syncthreads();   // every S column read; both halves' maxima read
+        pair_sync(warp);   // every S column of these rows read; both halves' maxima read
         if (rows_here) {
 #pragma unroll
             for (int q = 0; q < 8; ++q)
@@ -217,7 +237,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         }
         red[half][r] = lsum;
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-        __syncthreads();
+        __syncthreads();   // all of P stored before the second product
         lsum = red[0][r] + red[1][r];
         // ---- O = P V into columns [128, 192) ---------------------------------------------------
         const bool ok_s = s_fail == 0;   // the S waits' outcome, after the barrier above

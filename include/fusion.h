@@ -95,7 +95,7 @@ extern "C" {
 
 /* Size-aware attention (fusion_attention): head width and the longest sample. */
 #define FUSION_ATTN_HEAD_DIM 64
-#define FUSION_ATTN_MAX_TOKENS 256
+#define FUSION_ATTN_MAX_TOKENS 1024
 
 /* Pooling of an MLP exit head (fusion_mlp_head.pool). */
 #define FUSION_POOL_CLS 0     /* the CLS row (the paper's CLS-only head, block 10) */
@@ -323,6 +323,8 @@ int fusion_merge_router(int dtype, fusion_ragged in, const void *x, int32_t dim,
  * projection output: q, then k, then v, each heads x 64), 16-byte aligned; sizes:
  * [max_rows] float32 token sizes (> 0) or NULL; out: [max_rows, heads, 64] bf16,
  * 16-byte aligned; rows outside the samples are not written.
+ * Calls with in.max_tokens <= 256 hold each sample in shared memory; longer ones (up to
+ * FUSION_ATTN_MAX_TOKENS) stream blocks of 128 keys, two passes per query tile.
  * Errors: FUSION_ERR_DTYPE unless bf16; FUSION_ERR_SHAPE for head_dim != 64, heads < 1 or
  * in.max_tokens > FUSION_ATTN_MAX_TOKENS; FUSION_ERR_INVALID_ARG for NULL or misaligned
  * pointers; device bits BAD_BATCH, BAD_OFFSETS (that sample is not written), TIMEOUT.

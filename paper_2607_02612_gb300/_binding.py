@@ -38,7 +38,7 @@ FUSION_MAX_TOKENS = 1024
 FUSION_FUSED_PLAN_MAX_BATCH = 1024
 FUSION_MAX_DIM = 1024
 FUSION_ATTN_HEAD_DIM = 64
-FUSION_ATTN_MAX_TOKENS = 256
+FUSION_ATTN_MAX_TOKENS = 1024
 FUSION_POOL_CLS = 0
 FUSION_POOL_SPATIAL = 1
 

@@ -4,7 +4,9 @@
 // row m of the sample:
 //   out[m, h] = sum_j softmax_j(q_m . k_j / sqrt(dh) + log s_j) v_j.
 //
-// One CTA of 256 threads per (head, sample); samples of at most 256 tokens, dh = 64, bf16.
+// One CTA of 256 threads per (head, sample), dh = 64, bf16.  Samples of at most 256 tokens
+// (calls whose max_tokens is at most 256) keep the whole sample in shared memory (k_attn_tc);
+// longer samples, up to 1024 tokens, stream key blocks (k_attn_tc_long, below).
 // TMA brings the sample's query tiles of 128 rows, its K rows and its V rows (one 128-byte
 // row of 64 dims each, 128-byte swizzle) from the packed qkv matrix.  Q and K are K-major
 // operands; V, rows of keys with the dims contiguous, is the MN-major B operand of the second
@@ -291,9 +293,261 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kAttnTmemCols) : "memory");
 }
 
+// ---------------------------------------------------------------------------
+// Samples of 257 .. 1024 tokens.  The keys come in blocks of 128 (K, and V for the second
+// pass), double-buffered by TMA one step ahead; per query tile a first pass over the key blocks
+// takes the softmax shift (max_j S scale + max_j log2 s_j, as above) and a second pass forms P
+// over S's first columns and accumulates O = P V over the key blocks in columns [128, 192).
+// Q tiles are double-buffered too; every step waits for the previous step's products, so a
+// buffer is refilled only once nothing reads it.
+// ---------------------------------------------------------------------------
+constexpr int kLongMaxN = 1024;
+constexpr uint32_t kKvBytes = 128 * 128;   // a block of 128 key rows (K or V)
+
+__global__ void __launch_bounds__(kAttnThreads, 2)
+    k_attn_tc_long(const __grid_constant__ AttnMaps maps, AttnParams p) {
+    extern __shared__ unsigned char sm_raw[];
+    unsigned char *sm = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~uintptr_t(1023));
+    __shared__ __align__(8) unsigned long long bar_ld[2], bar_s, bar_o;
+    __shared__ uint32_t tmem_base;
+    __shared__ int s_fail, s_ld, s_ns, s_no;   // steps whose loads were issued; products S and O issued
+    __shared__ float lsz[kLongMaxN];
+    __shared__ float red[2][128];
+    __shared__ float s_lszmax;
+
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int h = blockIdx.x, i = blockIdx.y;
+    const int B = device_batch(p.in);
+    if (B < 0) {
+        if (h == 0 && i == 0 && tid == 0) raise_status(p.status, FUSION_DEV_BAD_BATCH);
+        return;
+    }
+    if (i >= B) return;
+    const int o0 = p.in.offsets[i], n = p.in.offsets[i + 1] - o0;
+    if (o0 < 0 || n < 1 || n > p.in.max_tokens || n > kLongMaxN || (long long)o0 + n > p.in.max_rows) {
+        if (h == 0 && tid == 0) raise_status(p.status, FUSION_DEV_BAD_OFFSETS);
+        return;
+    }
+    const int H = p.heads;
+    const int T = (n + 127) >> 7;          // query tiles
+    const int nkv = (n + 127) >> 7;        // key blocks
+    const int steps = T * 2 * nkv;         // (tile, pass, block) in that order
+    unsigned char *Qb = sm;                                 // [2] query tiles
+    unsigned char *Kb = sm + 2 * kQTileBytes;               // [2] key blocks
+    unsigned char *Vb = Kb + 2 * kKvBytes;                  // [2] value blocks
+
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(&tmem_base)),
+                     "r"(kAttnTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    // the loads of step k into buffer k & 1: the key block, the value block in the second pass,
+    // the query tile at a tile's first step
+    auto issue = [&](int k) {
+        const int t = k / (2 * nkv), pass = (k / nkv) & 1, kb = k % nkv;
+        const int buf = k & 1;
+        const int rows_k = min(128, n - 128 * kb), rk = (rows_k + 7) & ~7;
+        const bool q = pass == 0 && kb == 0;
+        const int rq = (min(128, n - 128 * t) + 7) & ~7;
+        uint32_t bytes = (uint32_t)rk * 128u * (pass ? 2u : 1u) + (q ? (uint32_t)rq * 128u : 0u);
+        const uint32_t bar = smem_addr(&bar_ld[buf]);
+        mbar_expect_tx(bar, bytes);
+        auto rows = [&](unsigned char *dst, int x, int y0, int cnt) {
+            int r = 0;
+            for (; r + 32 <= cnt; r += 32) tma_load_2d(smem_addr(dst + r * 128), &maps.b32, x, y0 + r, bar);
+            for (; r < cnt; r += 8) tma_load_2d(smem_addr(dst + r * 128), &maps.b8, x, y0 + r, bar);
+        };
+        rows(Kb + buf * kKvBytes, (H + h) * kAttnDh, o0 + 128 * kb, rk);
+        if (pass) rows(Vb + buf * kKvBytes, (2 * H + h) * kAttnDh, o0 + 128 * kb, rk);
+        if (q) rows(Qb + (t & 1) * kQTileBytes, h * kAttnDh, o0 + 128 * t, rq);
+    };
+    if (tid == 0) {
+        s_fail = 0;
+        s_ns = s_no = 0;
+        mbar_init(smem_addr(&bar_ld[0]), 1);
+        mbar_init(smem_addr(&bar_ld[1]), 1);
+        mbar_init(smem_addr(&bar_s), 1);
+        mbar_init(smem_addr(&bar_o), 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        issue(0);
+        s_ld = 1;
+    }
+    for (int j = tid; j < n; j += kAttnThreads) lsz[j] = p.sizes ? log2f(p.sizes[o0 + j]) : 0.0f;
+    __syncthreads();
+    if (warp == 0) {
+        float lm = -INFINITY;
+        for (int j = threadIdx.x; j < n; j += 32) lm = fmaxf(lm, lsz[j]);
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) lm = fmaxf(lm, __shfl_xor_sync(0xFFFFFFFFu, lm, o));
+        if (threadIdx.x == 0) s_lszmax = lm;
+    }
+    __syncthreads();
+
+    const uint32_t tmem = tmem_base;
+    const int half = warp >> 2;
+    const int r = tid & 127;
+    const uint32_t lane_addr = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+    constexpr float kScale2 = 0.18033688011112042f;   // log2(e) / sqrt(64)
+    const uint32_t idesc_o =
+        (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) | ((uint32_t)(kAttnDh >> 3) << 17) | (8u << 24);
+    float mraw = -INFINITY, mx = 0.0f, lsum = 0.0f;
+    bool stop = false;
+    for (int k = 0; k < steps && !stop; ++k) {
+        const int t = k / (2 * nkv), pass = (k / nkv) & 1, kb = k % nkv;
+        const int buf = k & 1;
+        const int rows_k = min(128, n - 128 * kb), npadb = (rows_k + 15) & ~15;
+        const bool rows_here = 128 * t + 32 * (warp & 3) < n;   // warp-uniform
+        const int nch = npadb >> 4, cA = (nch + 1) >> 1;
+        const int c_lo = half ? cA : 0, c_hi = half ? nch : cA;
+        // ---- this step's blocks landed; the next step's loads go out -------------------------
+        if (tid == 0) {
+            if (!mbar_wait(smem_addr(&bar_ld[buf]), (uint32_t)(k >> 1) & 1u)) {
+                s_fail = 1;
+            } else if (k + 1 < steps) {
+                issue(k + 1);
+                s_ld = k + 2;
+            }
+        }
+        __syncthreads();
+        if (s_fail & 1) break;   // uniform: bit 1 is written only before the barrier above
+        if (pass == 1 && rows_k < npadb)   // value rows past the sample read as zero in P V
+            for (int c = tid; c < (npadb - rows_k) * 8; c += kAttnThreads)
+                reinterpret_cast<uint4 *>(Vb + buf * kKvBytes + (size_t)rows_k * 128)[c] = make_uint4(0u, 0u, 0u, 0u);
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncthreads();
+        // ---- S = Q_t K_kb^T --------------------------------------------------------------------
+        if (tid == 0) {
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const uint32_t idesc_s = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(npadb >> 3) << 17) | (8u << 24);
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+                umma_bf16(tmem, sw128_desc(smem_addr(Qb + (t & 1) * kQTileBytes) + kk * 32),
+                          sw128_desc(smem_addr(Kb + buf * kKvBytes) + kk * 32), idesc_s, kk ? 1u : 0u);
+            umma_commit(smem_addr(&bar_s));
+            s_ns = s_ns + 1;
+        }
+        if (!mbar_wait(smem_addr(&bar_s), (uint32_t)k & 1u)) atomicOr(&s_fail, 2);
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        if (pass == 0) {
+            // ---- first pass: running maximum of S over this half's columns ---------------------
+            if (rows_here) {
+                for (int c = c_lo; c < c_hi; ++c) {
+                    uint32_t v[16];
+                    tmem_ld16(lane_addr + (uint32_t)(16 * c), v);
+#pragma unroll
+                    for (int e = 0; e < 16; ++e)
+                        if (16 * c + e < rows_k) mraw = fmaxf(mraw, __uint_as_float(v[e]));
+                }
+            }
+            if (kb == nkv - 1) {   // the tile's shift from both halves
+                red[half][r] = mraw;
+                pair_sync(warp);
+                mx = fmaf(fmaxf(red[0][r], red[1][r]), kScale2, s_lszmax);
+                pair_sync(warp);
+            }
+        } else {
+            // ---- second pass: P over S's first columns, then O += P V_kb ----------------------
+            uint32_t pk[4][8];   // this half's chunks, at most 4
+            if (rows_here) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const int c = c_lo + q;
+                    if (c < c_hi) {
+                        uint32_t v[16];
+                        tmem_ld16(lane_addr + (uint32_t)(16 * c), v);
+                        float pr[16];
+#pragma unroll
+                        for (int e = 0; e < 16; ++e)
+                            pr[e] = 16 * c + e < rows_k
+                                        ? ex2(fmaf(__uint_as_float(v[e]), kScale2, lsz[128 * kb + 16 * c + e]) - mx)
+                                        : 0.0f;
+#pragma unroll
+                        for (int e = 0; e < 16; e += 2) {
+                            lsum += pr[e] + pr[e + 1];
+                            const __nv_bfloat162 b2 = __floats2bfloat162_rn(pr[e], pr[e + 1]);
+                            pk[q][e >> 1] = *reinterpret_cast<const uint32_t *>(&b2);
+                        }
+                    }
+                }
+            }
+            pair_sync(warp);   // every S column of these rows read
+            if (rows_here) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    if (c_lo + q < c_hi) tmem_st8(lane_addr + (uint32_t)(8 * (c_lo + q)), pk[q]);
+                asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncthreads();
+            const bool ok_s = s_fail == 0;
+            if (tid == 0 && ok_s) {
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                for (int kk = 0; kk < npadb / 16; ++kk)
+                    umma_bf16_ts(tmem + 128u, tmem + 8u * kk, sw128_desc(smem_addr(Vb + buf * kKvBytes) + kk * 2048u),
+                                 idesc_o, (kb | kk) ? 1u : 0u);
+                umma_commit(smem_addr(&bar_o));
+                s_no = s_no + 1;
+            }
+            if (ok_s && !mbar_wait(smem_addr(&bar_o), (uint32_t)(t * nkv + kb) & 1u)) atomicOr(&s_fail, 4);
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            if (kb == nkv - 1) {
+                // ---- the tile's epilogue: O / row sum -> bf16 --------------------------------------
+                red[half][r] = lsum;
+                __syncthreads();
+                const float l = red[0][r] + red[1][r];
+                if (rows_here && s_fail == 0) {
+                    uint32_t o[32];
+                    tmem_ld16(lane_addr + 128u + 32u * half, *reinterpret_cast<uint32_t(*)[16]>(o));
+                    tmem_ld16(lane_addr + 144u + 32u * half, *reinterpret_cast<uint32_t(*)[16]>(o + 16));
+                    const int m = 128 * t + r;
+                    if (m < n) {
+                        const float inv = 1.0f / l;
+                        uint4 *dst = reinterpret_cast<uint4 *>(reinterpret_cast<__nv_bfloat16 *>(p.out) +
+                                                               (size_t)(o0 + m) * H * kAttnDh + (size_t)h * kAttnDh +
+                                                               32 * half);
+#pragma unroll
+                        for (int c = 0; c < 4; ++c) {
+                            uint32_t w[4];
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                const __nv_bfloat162 b2 = __floats2bfloat162_rn(
+                                    __uint_as_float(o[8 * c + 2 * e]) * inv, __uint_as_float(o[8 * c + 2 * e + 1]) * inv);
+                                w[e] = *reinterpret_cast<const uint32_t *>(&b2);
+                            }
+                            dst[c] = make_uint4(w[0], w[1], w[2], w[3]);
+                        }
+                    }
+                }
+                mraw = -INFINITY;
+                lsum = 0.0f;
+            }
+        }
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncthreads();   // S, P and O read before the next step's products overwrite them
+        stop = s_fail != 0;
+        __syncthreads();
+    }
+    if (tid == 0 && s_fail != 0) {   // let everything this CTA started finish before it leaves
+        raise_status(p.status, FUSION_DEV_TIMEOUT);
+        for (int b = 0; b < 2; ++b) {
+            const int last = s_ld - 1 - ((s_ld - 1 - b) & 1);   // the last step issued into buffer b
+            if (last >= 0) mbar_wait(smem_addr(&bar_ld[b]), (uint32_t)(last >> 1) & 1u);
+        }
+        if (s_ns > 0) mbar_wait(smem_addr(&bar_s), (uint32_t)(s_ns - 1) & 1u);
+        if (s_no > 0) mbar_wait(smem_addr(&bar_o), (uint32_t)(s_no - 1) & 1u);
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kAttnTmemCols) : "memory");
+}
+
 }  // namespace
 
 size_t attn_smem_bytes(int max_tokens) {
+    if (max_tokens > kAttnMaxN) return 1024u + 2u * kQTileBytes + 4u * kKvBytes;   // two Q tiles, two K and V blocks
     const int npad = (max_tokens + 15) & ~15, T = (max_tokens + 127) >> 7;
     return 1024u + (size_t)T * kQTileBytes + 2u * (size_t)npad * 128u;   // alignment, Q tiles, K, V
 }
@@ -314,9 +568,10 @@ cudaError_t launch_attention(const AttnParams &p, cudaStream_t s) {
                 CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
     }
-    cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    auto kern = p.in.max_tokens > kAttnMaxN ? k_attn_tc_long : k_attn_tc;   // whole samples resident, or key blocks
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    k_attn_tc<<<dim3((unsigned)p.heads, (unsigned)p.in.max_batch), kAttnThreads, smem, s>>>(maps, p);
+    kern<<<dim3((unsigned)p.heads, (unsigned)p.in.max_batch), kAttnThreads, smem, s>>>(maps, p);
     return cudaGetLastError();
 }
 

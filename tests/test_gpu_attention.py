@@ -75,8 +75,8 @@ def _check(offsets, qkv, H, sizes, label, nb=None, **kw):
 
 @pytest.mark.parametrize("sizes", [True, False])
 def test_attention_tile_boundaries(sizes):
-    """Sample lengths on both sides of every boundary of the kernel: 8-row TMA boxes, 16-key MMA
-    granularity, 64-key K-blocks, the 128-row query tile, the 256-token bound."""
+    """Sample lengths on both sides of every boundary of the resident-sample kernel: 8-row TMA boxes,
+    16-key MMA granularity, 64-key K-blocks, the 128-row query tile, the 256-token bound."""
     Ns = [1, 2, 7, 8, 9, 15, 16, 17, 63, 64, 65, 127, 128, 129, 130, 191, 192, 200, 255, 256]
     offsets, qkv, sz = _case(Ns, 3, 61, lead=3, tail=5)
     st = _check(offsets, qkv, 3, sz if sizes else None, f"boundaries sizes={sizes}")
@@ -101,14 +101,34 @@ def test_attention_large_logits_and_count():
     assert st == 0
 
 
+@pytest.mark.parametrize("sizes", [True, False])
+def test_attention_long_samples(sizes):
+    """Samples past 256 tokens stream key blocks of 128 (the ViT-L/16@384 length, 577, and the
+    1024-token bound), mixed with short ones in the same call and around the block edges."""
+    Ns = [577, 1, 300, 129, 1024, 256, 257, 385, 640]
+    offsets, qkv, sz = _case(Ns, 2, 65, lead=2, tail=3)
+    st = _check(offsets, qkv, 2, sz if sizes else None, f"long samples sizes={sizes}")
+    assert st == 0
+
+
+def test_attention_vit_l_shapes():
+    """ViT-L/16@384: 16 heads of 64, 577 tokens, a few images."""
+    offsets, qkv, sz = _case([577, 577, 400], 16, 66)
+    st = _check(offsets, qkv, 16, sz, "ViT-L 16 heads")
+    assert st == 0
+
+
 def test_attention_malformed():
     offsets, qkv, sz = _case([10, 20, 30], 2, 64)
     bad = offsets.copy()
     bad[2] = bad[1] - 1                    # a decreasing pair: that sample is not written
     g, st = _run(bad, qkv, 2, sz, max_tokens=64)
     assert st & fz.FUSION_DEV_BAD_OFFSETS
-    long = np.array([0, 10, 300, 310], np.int32)   # longer than max_tokens (and the 256 bound)
+    long = np.array([0, 10, 300, 310], np.int32)   # longer than max_tokens
     qkv2 = np.zeros((310, qkv.shape[1]), np.uint16)
     g, st = _run(long, qkv2, 2, None, max_tokens=256)
+    assert st & fz.FUSION_DEV_BAD_OFFSETS
+    assert (g[10:300] == SENTINEL).all()
+    g, st = _run(long, qkv2, 2, None, max_tokens=280)   # the key-block kernel checks the same
     assert st & fz.FUSION_DEV_BAD_OFFSETS
     assert (g[10:300] == SENTINEL).all()

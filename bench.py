@@ -253,6 +253,46 @@ def cpu_baseline(workload_name: str):
                       f"({dt:.1f} s, single thread)"}
 
 
+def oracle_side_legs(b):
+    """The oracle beside each side measurement (router, pruning-router scores, MLP exit head,
+    attention): bounded samples of the same inputs, single thread, timed before any GPU work."""
+    import oracle
+    from workloads import POOL_SPATIAL, f32_to_bf16_bits, make_mlp_head, make_router, make_score_head
+
+    def timed(fn, min_s=0.25):   # seconds per call, repeated until at least min_s in total
+        reps, t0 = 0, time.perf_counter()
+        while True:
+            fn()
+            reps += 1
+            dt = time.perf_counter() - t0
+            if dt >= min_s:
+                return dt / reps
+
+    def entry(value, unit, sample):
+        return {"value": value, "unit": unit, "cores": 1, "kind": "oracle", "sample": sample}
+
+    out = {}
+    rs = make_router(np.random.default_rng(2607), b.dim, b.dtype)
+    dt = timed(lambda: oracle.merge_router(b.dtype, b.offsets, b.x, rs.w, rs.beta, rs.tau_tgt, rs.tau_ref))
+    out["router"] = entry(b.batch / dt, "images/s", f"all {b.batch} images")
+    n = min(64, b.batch)
+    rows = int(b.offsets[n])
+    sh = make_score_head(np.random.default_rng(2608), b.dim, b.dtype)
+    dt = timed(lambda: oracle.token_scores(b.dtype, b.offsets[:n + 1], b.x[:rows], sh.w, sh.b))
+    out["pruning_router"] = entry(rows / dt, "tokens/s", f"{n} images, {rows} token rows")
+    n = min(32, b.batch)
+    rows = int(b.offsets[n])
+    mh = make_mlp_head(np.random.default_rng(2609), POOL_SPATIAL, b.dim, 2 * b.dim, 1000, b.dtype)
+    dt = timed(lambda: oracle.exit_mlp(b.dtype, b.offsets[:n + 1], b.x[:rows], b.sizes[:rows], mh))
+    out["exit_mlp"] = entry(n / dt, "images/s", f"{n} images, SpatialPool head, hidden {2 * b.dim}, 1000 classes")
+    n = min(2, b.batch)
+    rows = int(b.offsets[n])
+    qkv = f32_to_bf16_bits(np.random.default_rng(2610).standard_normal((rows, 3 * 6 * 64), dtype=np.float32))
+    dt = timed(lambda: oracle.attention("bf16", b.offsets[:n + 1], qkv, 6, b.sizes[:rows]))
+    out["attention"] = entry(n / dt, "images/s", f"{n} images x 6 heads")
+    return out
+
+
 # ---------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------
@@ -284,6 +324,7 @@ def main():
 
     w = make_workload(args.workload, seed_offset=rank)
     b = w.batch
+    side_cpu = oracle_side_legs(b) if cpu is not None else {}
     specs = w.stages
     classes = max([s.head.classes for s in specs if s.head is not None] + [1])
     fus = runner.Fusion(b.batch, classes, dev)
@@ -410,6 +451,9 @@ def main():
     scores = run_token_scores(args, fz, runner, b, dev, flush, peak)
     exit_mlp = run_exit_mlp(args, fz, runner, b, dev, flush, peak)
     attention = run_attention(args, fz, runner, b, dev, flush, peak)
+    for name, leg in (("router", router), ("pruning_router", scores), ("exit_mlp", exit_mlp), ("attention", attention)):
+        if name in side_cpu:
+            leg["cpu_oracle"] = side_cpu[name]
 
     # ---- end to end through the C ABI with host buffers -------------------------------
     e2e = run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world)

@@ -321,7 +321,9 @@ int fusion_merge_router(int dtype, fusion_ragged in, const void *x, int32_t dim,
  * product, the row sum taken in float32 before that rounding.
  * dtype: FUSION_BF16 only.  qkv: [max_rows, 3, heads, 64] bf16 row-major (timm's packed
  * projection output: q, then k, then v, each heads x 64), 16-byte aligned; sizes:
- * [max_rows] float32 token sizes (> 0) or NULL; out: [max_rows, heads, 64] bf16,
+ * [max_rows] float32 token sizes (> 0, within a factor 2^100 of each other inside a sample:
+ * the softmax is shifted by max_j q.k / sqrt(64) + max_j log s_j, which exceeds the row's
+ * largest logit by at most log(max s / min s)) or NULL; out: [max_rows, heads, 64] bf16,
  * 16-byte aligned; rows outside the samples are not written.
  * Calls with in.max_tokens <= 256 hold each sample in shared memory; longer ones (up to
  * FUSION_ATTN_MAX_TOKENS) stream blocks of 128 keys, two passes per query tile.

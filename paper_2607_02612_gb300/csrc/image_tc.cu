@@ -136,7 +136,10 @@ __global__ void __launch_bounds__(kTcThreads, 2)
         for (int b = 0; b < per_kb; ++b) issue_box(kb, b);
     };
 
-    // the first stages' loads go out before anything else, spread over warp 0
+    // the sample's token sizes and scores first (a few KB that would otherwise queue behind
+    // the bulk loads), then the first stages' loads, spread over warp 0
+    MetaPtrs m(sm, meta_layout(p.in.max_tokens, g.meta_base));
+    meta_prefetch<kTcThreads>(p, s, m);
     if (warp == 0) {
         if (lane == 0) s_fail = 0;
         if (dec) {
@@ -153,8 +156,7 @@ __global__ void __launch_bounds__(kTcThreads, 2)
             for (int t = lane; t < S0 * per_kb; t += 32) issue_box(t / per_kb, t % per_kb);
         }
     }
-    MetaPtrs m(sm, meta_layout(p.in.max_tokens, g.meta_base));
-    meta_init<kTcThreads>(p, s, m);
+    meta_init_rest<kTcThreads>(p, s, m);
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");

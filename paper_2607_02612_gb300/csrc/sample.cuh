@@ -261,6 +261,33 @@ __device__ __forceinline__ void meta_init(const ImageParams &p, const SampleInfo
     }
 }
 
+// meta_init in two parts, for a kernel whose own bulk loads would otherwise sit ahead of the
+// token sizes and scores in the memory queues: the copies of the sizes and scores go out first
+// (cp.async, no registers held), the rest of the metadata after, and the copies are waited for
+// at its end (before the caller's barrier).
+template <int NT>
+__device__ __forceinline__ void meta_prefetch(const ImageParams &p, const SampleInfo &s, MetaPtrs &m) {
+    for (int pos = threadIdx.x; pos < s.N; pos += NT) {
+        cp_async4(&m.tsize[pos], p.sizes + s.start + pos);
+        if (p.scores) cp_async4(&m.tscore[pos], p.scores + s.start + pos);
+    }
+    cp_async_commit();
+}
+template <int NT>
+__device__ __forceinline__ void meta_init_rest(const ImageParams &p, const SampleInfo &s, MetaPtrs &m) {
+    const int tid = threadIdx.x;
+    for (int a = tid; a < s.nA; a += NT) {
+        m.best[a] = 0ull;
+        m.sel[a] = 0;
+        m.match[a] = 0;
+    }
+    for (int n = tid; n <= s.nB; n += NT) m.scnt[n] = 0;
+    if (tid == 0) m.tmp[kMergedCount] = 0;
+    if (!p.scores)
+        for (int pos = tid; pos < s.N; pos += NT) m.tscore[pos] = 0.0f;
+    cp_async_wait_all();
+}
+
 // best[a] holds the packed (similarity, lowest B index) maximum of every A row.  Writes
 // match[a] and, when tokens merge, sel[a] for the r_eff A tokens of largest similarity
 // (lowest position on ties) and mkey[rank] = (match[a] << kKeyShift) | a for each of them.

@@ -161,12 +161,9 @@ template <typename T, int K>
 cudaError_t launch_k(const ScoreParams &p, int sms, cudaStream_t s) {
     auto kern = k_token_scores<T, K>;
     constexpr size_t smem = ScoreRing<K>::smem;
-    static bool opted = false;
-    if (!opted) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        opted = true;
-    }
+    // set on every launch: the attribute belongs to the current device
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
     const long long R = 32 / p.group;
     const long long tasks = ((p.in.max_rows + R - 1) / R + ScoreRing<K>::U - 1) / ScoreRing<K>::U;
     long long blocks = (tasks + kScoreThreads / 32 - 1) / (kScoreThreads / 32);

@@ -753,21 +753,21 @@ def run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world):
     dst = {"x": db.x.view(torch.int16) if b.dtype == "bf16" else db.x, "sizes": db.sizes, "scores": db.scores,
            "offsets": db.offsets}
     h2d = sum(t.numel() * t.element_size() for t in host.values())
-    last = chain.outs[-1]
-    exit_outs = [o for o in chain.outs if o["exit_mask"] is not None]
+    out = chain.host_results()
+    graph = None
+    if not args.eager:
+        chain.run()
+        torch.cuda.synchronize()
+        graph = chain.capture()
+    launch = graph.replay if graph is not None else chain.run
     d2h_bytes = []
 
     def one():
         for k in host:
             dst[k].copy_(host[k], non_blocking=True)
-        chain.run()
-        nb = int(last["batch"].item())                       # the result's size, then the result
-        rows = int(last["offsets"][nb].item())
-        res = [last["offsets"][:nb + 1].cpu(), last["ids"][:nb].cpu(), last["sizes"][:rows].cpu(),
-               last["x"][:rows].cpu()]
-        for o in exit_outs:
-            res += [o["exit_mask"].cpu(), o["max_prob"].cpu()]
-        d2h_bytes.append(sum(t.numel() * t.element_size() for t in res))
+        launch()
+        res, n = out.fetch()                                 # the result's size, then the result
+        d2h_bytes.append(n)
         return res
 
     for _ in range(2):
@@ -783,7 +783,9 @@ def run_e2e(args, fz, runner, chain, b, dev, S, units_step, barrier, world):
     dt, units = reduce_over_ranks(dt, units_step * steps, world, dev)
     return {"value": units / dt, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h_bytes[-1]), "steps": steps,
-            "note": "pinned host inputs, C-ABI chain (no L2 flush), host reads the survivor count then the results"}
+            "note": ("pinned host inputs and outputs, C-ABI chain " +
+                     ("launched eagerly" if graph is None else "as a replayed CUDA graph") +
+                     " (no L2 flush); the host reads the survivor count, then the results")}
 
 
 if __name__ == "__main__":

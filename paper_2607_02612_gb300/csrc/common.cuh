@@ -219,6 +219,13 @@ __device__ __forceinline__ F2 f2_div(F2 a, F2 b) {
     const float q2 = __fdiv_rn(r.hi, b.hi);
     return quick_two_sum(q1, q2);
 }
+// 1 / n in float-float for a positive float n: the correctly rounded reciprocal r plus the
+// remainder 1 - r n (exact in one fma for a correctly rounded r) times r, about 46 correct
+// bits.  It needs no data, so a caller computes it before a reduction rather than after.
+__device__ __forceinline__ F2 f2_recip(float n) {
+    const float r = __frcp_rn(n);
+    return quick_two_sum(r, __fmul_rn(__fmaf_rn(-r, n, 1.0f), r));
+}
 // 1 / sqrt(v) for a positive float-float v: one Newton step in float-float on the
 // float32 estimate, about 44 correct bits.
 __device__ __forceinline__ F2 f2_rsqrt(F2 v) {

@@ -294,8 +294,8 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
 #pragma unroll
                 for (int e = 0; e < CH; ++e) neu_add(ss, sc, f[e]);
             }
-            const F2 fdim = {(float)dim, 0.0f};
-            const F2 mean = f2_div(warp_sum_f2(two_sum(ss, sc)), fdim);
+            const F2 rdim = f2_recip((float)dim);
+            const F2 mean = f2_mul(warp_sum_f2(two_sum(ss, sc)), rdim);
             ss = sc = 0.0f;
             float lo = 0.0f;
             for (int c = lane; c < nchunk; c += 32) {
@@ -310,7 +310,7 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
                     lo = __fmaf_rn(2.0f * d.hi, d.lo, __fadd_rn(lo, sq.lo));
                 }
             }
-            const F2 var = f2_div(warp_sum_f2(f2_add_f(two_sum(ss, sc), lo)), fdim);
+            const F2 var = f2_mul(warp_sum_f2(f2_add_f(two_sum(ss, sc), lo)), rdim);
             const F2 rstd = f2_rsqrt(f2_add_f(var, p.head.eps));
             if (lane == 0 && !(isfinite(mean.hi) && isfinite(var.hi))) raise_status(p.status, FUSION_DEV_NONFINITE);
             const T *g = reinterpret_cast<const T *>(p.head.gamma);
@@ -450,8 +450,9 @@ struct ExitClSmem {
     static __host__ __device__ size_t bias_off(int dim) { return w_off(dim) + 2 * B::w_stage; }
     static __host__ __device__ size_t part_off(int dim) { return bias_off(dim) + kExitCT * sizeof(float); }
     static __host__ __device__ size_t red_off(int dim) { return part_off(dim) + (size_t)kExitBT * 8 * sizeof(float2); }
+    static __host__ __device__ size_t flag_off(int dim) { return red_off(dim) + (size_t)(kExitThreads / 32) * 8 * sizeof(float); }
     static __host__ __device__ size_t total(int dim) {
-        const size_t t = red_off(dim) + (size_t)(kExitThreads / 32) * 8 * sizeof(float);
+        const size_t t = flag_off(dim) + (size_t)kExitBT * sizeof(int);
         const size_t plan = w_off(dim) + (4 * kExitThreads + 40) * sizeof(int);   // run_plan reuses the W stages
         return t > plan ? t : plan;
     }
@@ -479,6 +480,7 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(ExitParams p) {
     float *bias_s = reinterpret_cast<float *>(sm + L::bias_off(dim));
     float2 *part_s = reinterpret_cast<float2 *>(sm + L::part_off(dim));
     float *red = reinterpret_cast<float *>(sm + L::red_off(dim));
+    int *rowflag_s = reinterpret_cast<int *>(sm + L::flag_off(dim));   // [kExitBT]: 1 row, 0 none, -1 bad
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int ct = blockIdx.x, bt = blockIdx.y;
@@ -504,10 +506,12 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(ExitParams p) {
             const int sli = rank + jj * ncl, si = s0 + sli;
             T *dst = x_s + (size_t)jj * u_stride + c * CH;
             long long row = -1;
-            if (sli < kExitBT && si < B) {
+            const bool want = sli < kExitBT && si < B;
+            if (want) {
                 row = p.in.offsets[si];
                 if (row < 0 || row >= p.in.max_rows) row = -1;
             }
+            if (c == 0) rowflag_s[jj] = want ? (row >= 0 ? 1 : -1) : 0;
             if (row >= 0)
                 cp_async16(dst, reinterpret_cast<const T *>(p.x) + row * dim + c * CH);
             else
@@ -537,14 +541,10 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(ExitParams p) {
         if (n_k > 1) issue_w_chunk<T>(p, w_region + S::w_stage, c0, KC, dim, C, tid);
 
         // ---- LayerNorm, G warps per row: one pass of sum and sum of squares -----------
-        bool ok = has_row && s < B;
-        if (ok) {
-            const long long row = p.in.offsets[s];
-            if (row < 0 || row >= p.in.max_rows) {
-                if (gt == 0) raise_status(p.status, FUSION_DEV_BAD_OFFSETS);
-                ok = false;
-            }
-        }
+        const int rflag = has_row ? rowflag_s[j] : 0;   // checked by the load loop above
+        if (rflag < 0 && gt == 0) raise_status(p.status, FUSION_DEV_BAD_OFFSETS);
+        const bool ok = rflag > 0;
+        const F2 rdim = f2_recip((float)dim);
         const T *xr = x_s + (size_t)j * u_stride;
         float s1 = 0.0f, c1 = 0.0f, s2 = 0.0f, c2 = 0.0f, l2 = 0.0f;
         if (ok) {
@@ -566,14 +566,16 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(ExitParams p) {
         }
         __syncthreads();
         if (ok) {
-            F2 t1 = {0.0f, 0.0f}, t2 = {0.0f, 0.0f};
-            for (int w = j * G; w < j * G + G; ++w) {   // the group's warps, in order
-                t1 = f2_add(t1, {red[w * 8 + 0], red[w * 8 + 1]});
-                t2 = f2_add(t2, {red[w * 8 + 2], red[w * 8 + 3]});
+            // the group's G (a power of two) warp sums: every aligned run of G lanes adds them
+            // as a butterfly, so all lanes hold the same bits (f2_add is symmetric)
+            const int wq = j * G + (lane & (G - 1));
+            F2 t1 = {red[wq * 8 + 0], red[wq * 8 + 1]}, t2 = {red[wq * 8 + 2], red[wq * 8 + 3]};
+            for (int m = G >> 1; m >= 1; m >>= 1) {
+                t1 = f2_add(t1, f2_shfl_xor(t1, m));
+                t2 = f2_add(t2, f2_shfl_xor(t2, m));
             }
-            const F2 fdim = {(float)dim, 0.0f};
-            const F2 mean = f2_div(t1, fdim);
-            const F2 ex2 = f2_div(t2, fdim);
+            const F2 mean = f2_mul(t1, rdim);
+            const F2 ex2 = f2_mul(t2, rdim);
             const F2 m2 = f2_mul(mean, mean);
             F2 var = f2_add(ex2, {-m2.hi, -m2.lo});
             if (var.hi < 0.0f) var = {0.0f, 0.0f};

@@ -301,3 +301,51 @@ class Chain:
         with torch.cuda.graph(g):
             self.run()
         return g
+
+    def host_results(self) -> "HostResults":
+        """Pinned host buffers sized for this chain's results (see HostResults)."""
+        return HostResults(self)
+
+
+class HostResults:
+    """Pinned host copies of a chain's results: the survivors of the last stage (count,
+    offsets, ids, sizes, token rows) and every exit check's mask and max probability.
+
+    fetch() runs on the current stream after the chain was enqueued: one asynchronous copy
+    of the fixed-size parts (the count, the offsets bound, the exit outputs), one host wait,
+    then copies of the survivors' exact extent and a second wait.  Returns host views
+    (valid until the next fetch) and the number of bytes copied."""
+
+    def __init__(self, chain: Chain):
+        last = chain.outs[-1]
+        self._last = last
+        self._exits = [(o["exit_mask"], o["max_prob"]) for o in chain.outs if o["exit_mask"] is not None]
+        pin = lambda t: torch.empty(t.shape, dtype=t.dtype).pin_memory()   # noqa: E731
+        self.batch = pin(last["batch"])
+        self.offsets = pin(last["offsets"])
+        self.ids = pin(last["ids"])
+        self.sizes = pin(last["sizes"])
+        self.x = pin(last["x"])
+        self.exits = [(pin(m), pin(p)) for m, p in self._exits]
+
+    def fetch(self):
+        last = self._last
+        self.batch.copy_(last["batch"], non_blocking=True)
+        self.offsets.copy_(last["offsets"], non_blocking=True)
+        n = self.batch.numel() * 4 + self.offsets.numel() * 4
+        for (hm, hp), (m, p) in zip(self.exits, self._exits):
+            hm.copy_(m, non_blocking=True)
+            hp.copy_(p, non_blocking=True)
+            n += hm.numel() * hm.element_size() + hp.numel() * hp.element_size()
+        torch.cuda.current_stream().synchronize()
+        nb = int(self.batch[0])
+        rows = int(self.offsets[nb])
+        parts = (("ids", nb), ("sizes", rows), ("x", rows))
+        for name, k in parts:
+            h = getattr(self, name)
+            h[:k].copy_(last[name][:k], non_blocking=True)
+            n += h[:k].numel() * h.element_size()
+        torch.cuda.current_stream().synchronize()
+        res = {"batch": nb, "offsets": self.offsets[:nb + 1], "ids": self.ids[:nb], "sizes": self.sizes[:rows],
+               "x": self.x[:rows], "exits": [(hm, hp) for hm, hp in self.exits]}
+        return res, n

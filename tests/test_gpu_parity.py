@@ -157,6 +157,49 @@ def test_chain_parity(name, B, graph):
     _report(rep, f"chain {name}")
 
 
+def test_chain_host_results():
+    """The serving loop of the end-to-end measurement: pinned host inputs copied in, the chain
+    replayed as a CUDA graph, the results fetched into pinned host buffers (survivor count
+    first, then the survivors' exact extent).  On two consecutive replays the device outputs
+    match the oracle's chain and the fetched host copies equal the device outputs."""
+    w = make_workload("deit_s_chain12_bf16_b256", batch=64)
+    b = w.batch
+    fzr = runner.Fusion(b.batch, max(s.head.classes for s in w.stages if s.head is not None))
+    db = P.device_batch(b)
+    stages = [runner.ChainStage(P.flags_of(s), *P.stage_tensors(s, b.dtype)) for s in w.stages]
+    ch = runner.Chain(fzr, db, stages)
+    hr = ch.host_results()
+    xh = torch.from_numpy(np.ascontiguousarray(b.x).view(np.int16)).pin_memory()
+    ch.run()
+    torch.cuda.synchronize()
+    g = ch.capture()
+    o_outs = oracle.chain(w)
+    for rep_i in range(2):
+        db.x.view(torch.int16).copy_(xh, non_blocking=True)
+        g.replay()
+        res, nbytes = hr.fetch()
+        assert int(fzr.status.item()) == 0
+        d_outs = [P.to_host(o, b.dtype) for o in ch.outs]
+        rep = P.Report()
+        P.compare_chain(rep, w, d_outs, o_outs)
+        assert rep.compared_samples > 0
+        _report(rep, f"host results, replay {rep_i}")
+        last = d_outs[-1]
+        nb = int(last["batch"][0])
+        rows = int(last["offsets"][nb])
+        assert res["batch"] == nb
+        np.testing.assert_array_equal(res["offsets"].numpy(), last["offsets"][:nb + 1])
+        np.testing.assert_array_equal(res["ids"].numpy(), last["ids"][:nb])
+        np.testing.assert_array_equal(res["sizes"].numpy(), last["sizes"][:rows])
+        np.testing.assert_array_equal(res["x"].view(torch.int16).numpy().view(np.uint16), last["x"][:rows])
+        exits = [o for o in d_outs if o["exit_mask"] is not None]
+        assert len(res["exits"]) == len(exits) == sum(1 for s in w.stages if s.exit)
+        for (hm, hp), o in zip(res["exits"], exits):
+            np.testing.assert_array_equal(hm.numpy(), o["exit_mask"])
+            np.testing.assert_array_equal(hp.numpy(), o["max_prob"])
+        assert nbytes >= res["x"].numel() * 2
+
+
 def _subset(batch: Batch, idx: np.ndarray) -> Batch:
     """The images idx of a batch, repacked (ids keep the original image numbers)."""
     counts = np.diff(batch.offsets)[idx]

@@ -306,10 +306,24 @@ class Chain:
         """Pinned host buffers sized for this chain's results (see HostResults)."""
         return HostResults(self)
 
+    def clone(self) -> "Chain":
+        """The same schedule over its own input, output and scratch buffers (the stage
+        parameters, read only, are shared); the inputs start as a copy of this chain's."""
+        b = self.inp
+        x = b.x.clone()
+        keys = x if b.keys is b.x else b.keys.clone()
+        cp = lambda t: None if t is None else t.clone()   # noqa: E731
+        inp = DeviceBatch(dtype=b.dtype, dim=b.dim, max_batch=b.max_batch, max_tokens=b.max_tokens,
+                          max_rows=b.max_rows, x=x, keys=keys, sizes=b.sizes.clone(), scores=cp(b.scores),
+                          offsets=b.offsets.clone(), batch=cp(b.batch), ids=cp(b.ids))
+        fus = Fusion(self.fusion.max_batch, self.fusion.classes, self.fusion.device)
+        return Chain(fus, inp, list(self.stages))
+
 
 class HostResults:
     """Pinned host copies of a chain's results: the survivors of the last stage (count,
-    offsets, ids, sizes, token rows) and every exit check's mask and max probability.
+    offsets, ids, sizes, token rows), every exit check's mask and max probability over the
+    images entering it, and the device status word.
 
     fetch() runs on the current stream after the chain was enqueued: one asynchronous copy
     of the fixed-size parts (the count, the offsets bound, the exit outputs), one host wait,
@@ -320,6 +334,9 @@ class HostResults:
         last = chain.outs[-1]
         self._last = last
         self._exits = [(o["exit_mask"], o["max_prob"]) for o in chain.outs if o["exit_mask"] is not None]
+        # images entering each exit check (None: the whole input batch)
+        self._exit_in = [b.batch for b, o in zip(chain.batches, chain.outs) if o["exit_mask"] is not None]
+        self._exit_max = [b.max_batch for b, o in zip(chain.batches, chain.outs) if o["exit_mask"] is not None]
         pin = lambda t: torch.empty(t.shape, dtype=t.dtype).pin_memory()   # noqa: E731
         self.batch = pin(last["batch"])
         self.offsets = pin(last["offsets"])
@@ -327,25 +344,127 @@ class HostResults:
         self.sizes = pin(last["sizes"])
         self.x = pin(last["x"])
         self.exits = [(pin(m), pin(p)) for m, p in self._exits]
+        self.exit_in = [None if t is None else pin(t) for t in self._exit_in]
+        self._status = chain.fusion.status
+        self.status = pin(self._status)
 
     def fetch(self):
+        self.fetch_fixed()
+        torch.cuda.current_stream().synchronize()
+        self.fetch_exact()
+        torch.cuda.current_stream().synchronize()
+        return self.result()
+
+    def fetch_fixed(self):
+        """Enqueue (current stream) the copies whose size the host knows: the survivor count,
+        the offsets bound and the exit outputs."""
         last = self._last
         self.batch.copy_(last["batch"], non_blocking=True)
         self.offsets.copy_(last["offsets"], non_blocking=True)
-        n = self.batch.numel() * 4 + self.offsets.numel() * 4
-        for (hm, hp), (m, p) in zip(self.exits, self._exits):
+        self.status.copy_(self._status, non_blocking=True)
+        self._n = self.batch.numel() * 4 + self.offsets.numel() * 4 + 4
+        for (hm, hp), (m, p), hc, c in zip(self.exits, self._exits, self.exit_in, self._exit_in):
             hm.copy_(m, non_blocking=True)
             hp.copy_(p, non_blocking=True)
-            n += hm.numel() * hm.element_size() + hp.numel() * hp.element_size()
-        torch.cuda.current_stream().synchronize()
-        nb = int(self.batch[0])
-        rows = int(self.offsets[nb])
-        parts = (("ids", nb), ("sizes", rows), ("x", rows))
-        for name, k in parts:
+            self._n += hm.numel() * hm.element_size() + hp.numel() * hp.element_size()
+            if hc is not None:
+                hc.copy_(c, non_blocking=True)
+                self._n += 4
+
+    def fetch_exact(self):
+        """Enqueue (current stream) the survivors' rows; the fixed copies must have landed."""
+        last = self._last
+        self._nb = int(self.batch[0])
+        self._rows = int(self.offsets[self._nb])
+        for name, k in (("ids", self._nb), ("sizes", self._rows), ("x", self._rows)):
             h = getattr(self, name)
             h[:k].copy_(last[name][:k], non_blocking=True)
-            n += h[:k].numel() * h.element_size()
-        torch.cuda.current_stream().synchronize()
+            self._n += h[:k].numel() * h.element_size()
+
+    def result(self):
+        nb, rows = self._nb, self._rows
         res = {"batch": nb, "offsets": self.offsets[:nb + 1], "ids": self.ids[:nb], "sizes": self.sizes[:rows],
-               "x": self.x[:rows], "exits": [(hm, hp) for hm, hp in self.exits]}
-        return res, n
+               "x": self.x[:rows], "status": int(self.status[0]), "exits": []}
+        for (hm, hp), hc, mx in zip(self.exits, self.exit_in, self._exit_max):
+            n = mx if hc is None else int(hc[0])
+            res["exits"].append((hm[:n], hp[:n]))
+        return res, self._n
+
+
+class Pipeline:
+    """Back-to-back steps of one schedule with host inputs and host results, the copies
+    overlapped with the computation: step k runs on slot k % 2 (a chain with its own
+    buffers, replayed as a CUDA graph), its inputs are copied on one copy stream while step
+    k - 1 computes, and its results come back on another.  The survivors' exact extent is
+    known only once the host has read their count, so submit() of step k returns the results
+    of step k - 1 (None for the first) and finish() those of the last step; host results stay
+    valid until the next call.  Slots are not reused before their results are on the host."""
+
+    def __init__(self, chain: Chain):
+        self.chains = [chain, chain.clone()]
+        self.graphs = []
+        for ch in self.chains:
+            ch.run()
+            torch.cuda.synchronize()
+            self.graphs.append(ch.capture())
+        self.hr = [ch.host_results() for ch in self.chains]
+        self.s_h2d, self.s_cmp, self.s_d2h = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+        ev = lambda: [torch.cuda.Event(), torch.cuda.Event()]   # noqa: E731
+        self.ev_h2d, self.ev_cmp, self.ev_cnt, self.ev_res = ev(), ev(), ev(), ev()
+        self.k = 0
+        self.pending: Optional[int] = None
+
+    def _inputs(self, slot: int) -> Dict[str, torch.Tensor]:
+        b = self.chains[slot].inp
+        d = {"x": b.x.view(torch.int16) if b.dtype == "bf16" else b.x, "sizes": b.sizes, "offsets": b.offsets}
+        if b.keys is not b.x:
+            d["keys"] = b.keys.view(torch.int16) if b.dtype == "bf16" else b.keys
+        if b.scores is not None:
+            d["scores"] = b.scores
+        return d
+
+    def submit(self, host: Dict[str, torch.Tensor]):
+        """host: pinned tensors named after the input fields (x as int16 bits for bf16)."""
+        c = self.k % 2
+        dst = self._inputs(c)
+        with torch.cuda.stream(self.s_h2d):
+            if self.k >= 2:
+                self.s_h2d.wait_event(self.ev_cmp[c])   # the slot's previous replay read its inputs
+            for name, t in host.items():
+                dst[name].copy_(t, non_blocking=True)
+            self.ev_h2d[c].record(self.s_h2d)
+        with torch.cuda.stream(self.s_cmp):
+            self.s_cmp.wait_event(self.ev_h2d[c])
+            if self.k >= 2:
+                self.s_cmp.wait_event(self.ev_res[c])   # the slot's previous results are on the host
+            self.graphs[c].replay()
+            self.ev_cmp[c].record(self.s_cmp)
+        prev = self._complete()
+        with torch.cuda.stream(self.s_d2h):
+            self.s_d2h.wait_event(self.ev_cmp[c])
+            self.hr[c].fetch_fixed()
+            self.ev_cnt[c].record(self.s_d2h)
+        self.pending = c
+        self.k += 1
+        return prev
+
+    def _complete(self):
+        p = self.pending
+        if p is None:
+            return None
+        self.pending = None
+        self.ev_cnt[p].synchronize()
+        with torch.cuda.stream(self.s_d2h):
+            self.hr[p].fetch_exact()
+            self.ev_res[p].record(self.s_d2h)
+        self.ev_res[p].synchronize()
+        return self.hr[p].result()
+
+    def finish(self):
+        """Results of the last submitted step (None if there is none)."""
+        return self._complete()
+
+    def status(self) -> int:
+        """OR of the slots' device status words (synchronises)."""
+        torch.cuda.synchronize()
+        return int(self.chains[0].fusion.status.item()) | int(self.chains[1].fusion.status.item())

@@ -192,12 +192,80 @@ def test_chain_host_results():
         np.testing.assert_array_equal(res["ids"].numpy(), last["ids"][:nb])
         np.testing.assert_array_equal(res["sizes"].numpy(), last["sizes"][:rows])
         np.testing.assert_array_equal(res["x"].view(torch.int16).numpy().view(np.uint16), last["x"][:rows])
-        exits = [o for o in d_outs if o["exit_mask"] is not None]
+        entering = [b.batch] + [int(o["batch"][0]) for o in d_outs[:-1]]
+        exits = [(o, n) for o, n in zip(d_outs, entering) if o["exit_mask"] is not None]
         assert len(res["exits"]) == len(exits) == sum(1 for s in w.stages if s.exit)
-        for (hm, hp), o in zip(res["exits"], exits):
-            np.testing.assert_array_equal(hm.numpy(), o["exit_mask"])
-            np.testing.assert_array_equal(hp.numpy(), o["max_prob"])
+        for (hm, hp), (o, n) in zip(res["exits"], exits):
+            assert len(hm) == len(hp) == n
+            np.testing.assert_array_equal(hm.numpy(), o["exit_mask"][:n])
+            np.testing.assert_array_equal(hp.numpy(), o["max_prob"][:n])
         assert nbytes >= res["x"].numel() * 2
+
+
+def _np(t: torch.Tensor) -> np.ndarray:
+    return (t.view(torch.int16) if t.dtype == torch.bfloat16 else t).numpy().copy()
+
+
+def _host_copy(res):
+    r = {k: (_np(v) if isinstance(v, torch.Tensor) else v) for k, v in res.items() if k != "exits"}
+    r["exits"] = [(_np(m), _np(p)) for m, p in res["exits"]]
+    return r
+
+
+def test_pipeline_overlapped_steps():
+    """Steps submitted back to back through the two-slot pipeline (input copies overlapping the
+    previous step's kernels, results one step late) give, step by step, the results of the same
+    inputs run one at a time; those match the oracle's chain for both inputs."""
+    wa = make_workload("deit_s_chain12_bf16_b256", batch=64)
+    wb = type(wa)(wa.spec, make_workload("deit_s_chain12_bf16_b256", batch=64, seed_offset=1).batch, wa.stages)
+    b = wa.batch
+    assert np.array_equal(b.offsets, wb.batch.offsets)
+    fzr = runner.Fusion(b.batch, max(s.head.classes for s in wa.stages if s.head is not None))
+    stages = [runner.ChainStage(P.flags_of(s), *P.stage_tensors(s, b.dtype)) for s in wa.stages]
+    ch = runner.Chain(fzr, P.device_batch(b), stages)
+
+    def pinned(bb):
+        return {"x": torch.from_numpy(np.ascontiguousarray(bb.x).view(np.int16)).pin_memory(),
+                "sizes": torch.from_numpy(bb.sizes).pin_memory(),
+                "scores": torch.from_numpy(bb.scores).pin_memory(),
+                "offsets": torch.from_numpy(bb.offsets).pin_memory()}
+    hosts = [pinned(wa.batch), pinned(wb.batch)]
+    # one at a time, on a separate chain
+    solo = ch.clone()
+    hr = solo.host_results()
+    want = []
+    for i, w in enumerate((wa, wb)):
+        db = solo.inp
+        db.x.view(torch.int16).copy_(hosts[i]["x"])
+        db.sizes.copy_(hosts[i]["sizes"])
+        db.scores.copy_(hosts[i]["scores"])
+        solo.run()
+        want.append(_host_copy(hr.fetch()[0]))
+        assert want[-1]["status"] == 0
+        rep = P.Report()
+        P.compare_chain(rep, w, [P.to_host(o, b.dtype) for o in solo.outs], oracle.chain(w))
+        assert rep.compared_samples > 0
+        _report(rep, f"pipeline reference input {i}")
+    pipe = runner.Pipeline(ch)
+    seq = [0, 1, 1, 0, 1, 0, 0]
+    got = []
+    for i in seq:
+        r = pipe.submit(hosts[i])
+        if r is not None:
+            got.append(_host_copy(r[0]))
+    got.append(_host_copy(pipe.finish()[0]))
+    assert pipe.status() == 0
+    assert len(got) == len(seq)
+    for k, (i, g) in enumerate(zip(seq, got)):
+        e = want[i]
+        assert g["batch"] == e["batch"] and g["status"] == 0, (k, i)
+        for name in ("offsets", "ids", "sizes", "x"):
+            np.testing.assert_array_equal(g[name], e[name], err_msg=f"step {k} input {i} {name}")
+        assert len(g["exits"]) == len(e["exits"]) == 4
+        for (gm, gp), (em, ep) in zip(g["exits"], e["exits"]):
+            np.testing.assert_array_equal(gm, em)
+            np.testing.assert_array_equal(gp, ep)
+    assert want[0]["batch"] != want[1]["batch"] or not np.array_equal(want[0]["ids"], want[1]["ids"])
 
 
 def _subset(batch: Batch, idx: np.ndarray) -> Batch:

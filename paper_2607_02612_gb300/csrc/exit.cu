@@ -14,6 +14,7 @@
 #include <cooperative_groups.h>
 
 #include "launch.h"
+#include "tc.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -437,6 +438,73 @@ __device__ __forceinline__ float to_float(__nv_bfloat16 v) { return __bfloat162f
 // them.  The head's weight chunks load while the LayerNorm runs; no global atomics
 // unless the plan kernel's work runs here (batches above the fused-plan bound).
 // ---------------------------------------------------------------------------
+constexpr int kExitWStages = 4;                      // TMA stages of the bf16 head weights
+constexpr uint32_t kExitWStage = kExitCT * 128u;     // one stage: kExitCT rows x 64 bf16 dims
+
+// The logits tile of the cluster kernel for bf16: as exit_gemm, with the weights' K chunks
+// of 64 dims arriving by TMA (chunks 0..kExitWStages-1 already issued by thread 0).  Stage
+// st holds rows c0.. of the tile, 128 bytes each, 16-byte chunk j of row n at j ^ (n % 8);
+// classes past C and dims past dim read as zeros.  Thread 0 waits on each stage (bounded) and
+// refills it once every warp is done with it.  The MMA sequence and the partial-sum flushes
+// are those of exit_gemm.  Returns false (uniform) when a wait gave up; the copies still in
+// flight are waited for (bounded) before returning.
+__device__ __forceinline__ bool exit_gemm_tma(const CUtensorMap *wmap, const __nv_bfloat16 *u_s, unsigned char *w_tma,
+                                              unsigned long long *wbar, int *s_wfail, int c0, int dim,
+                                              float (&acc)[4], float (&acc2)[4]) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int u_stride = ExitSmem<__nv_bfloat16>::u_stride(dim);
+    const int nk = (dim + 63) / 64;
+    const uint32_t ubase = smem_addr(u_s);
+    const int arow = (lane & 7) + ((lane >> 3) & 1) * 8;
+    const int brow = warp * 16 + (lane >> 4) * 8 + (lane & 7);
+    const uint32_t bsw = (uint32_t)(brow & 7);
+    int kc = 0;
+    for (; kc < nk; ++kc) {
+        const int st = kc % kExitWStages;
+        if (tid == 0 && !mbar_wait(smem_addr(&wbar[st]), (uint32_t)(kc / kExitWStages) & 1u)) *s_wfail = 1;
+        __syncthreads();
+        if (*s_wfail) break;
+        const int kw = min(64, dim - kc * 64);
+        const uint32_t wrow = smem_addr(w_tma + (size_t)st * kExitWStage) + (uint32_t)brow * 128u;
+        float t0[4] = {0.0f, 0.0f, 0.0f, 0.0f}, t1[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        for (int kk = 0; kk < kw; kk += 16) {
+            uint32_t af[4], b0, b1, b2, b3;
+            ldsm_x4(ubase + (uint32_t)((arow * u_stride + kc * 64 + kk + (lane >> 4) * 8) * 2), af[0], af[1], af[2],
+                    af[3]);
+            const uint32_t j = (uint32_t)(kk >> 3) + (uint32_t)((lane >> 3) & 1);
+            ldsm_x4(wrow + ((j ^ bsw) << 4), b0, b1, b2, b3);
+            mma_bf16_16816(t0, af, b0, b1);
+            mma_bf16_16816(t1, af, b2, b3);
+            if (kk == 48) {   // flush the partial sums every 64 dims
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    acc[e] += t0[e];
+                    acc2[e] += t1[e];
+                    t0[e] = t1[e] = 0.0f;
+                }
+            }
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            acc[e] += t0[e];
+            acc2[e] += t1[e];
+        }
+        __syncthreads();   // every warp is done with stage st
+        if (tid == 0 && kc + kExitWStages < nk) {
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            mbar_expect_tx(smem_addr(&wbar[st]), kExitWStage);
+            tma_load_2d(smem_addr(w_tma + (size_t)st * kExitWStage), wmap, (kc + kExitWStages) * 64, c0,
+                        smem_addr(&wbar[st]));
+        }
+    }
+    if (kc == nk) return true;
+    if (tid == 0)   // chunks kc.. issued and not consumed: let them land before the CTA moves on
+        for (int q = kc; q < nk && q < kc + kExitWStages; ++q)
+            (void)mbar_wait(smem_addr(&wbar[q % kExitWStages]), (uint32_t)(q / kExitWStages) & 1u);
+    __syncthreads();
+    return false;
+}
+
 template <typename T>
 struct ExitClSmem {
     static constexpr int EB = Elem<T>::kBytes;
@@ -447,7 +515,12 @@ struct ExitClSmem {
     static __host__ __device__ size_t g_off(int dim) { return x_off(dim) + (size_t)kExitBT * B::u_stride(dim) * EB; }
     static __host__ __device__ size_t be_off(int dim) { return g_off(dim) + ((size_t)dim * EB + 15) / 16 * 16; }
     static __host__ __device__ size_t w_off(int dim) { return be_off(dim) + ((size_t)dim * EB + 15) / 16 * 16; }
-    static __host__ __device__ size_t bias_off(int dim) { return w_off(dim) + 2 * B::w_stage; }
+    // bf16: kExitWStages TMA stages of [kExitCT rows][64 dims] (128-byte rows, 128-byte swizzle,
+    // 1024-byte aligned inside the region); float32: two cp.async stages
+    static __host__ __device__ size_t w_bytes() {
+        return EB == 2 ? (size_t)kExitWStages * kExitWStage + 1024 : 2 * B::w_stage;
+    }
+    static __host__ __device__ size_t bias_off(int dim) { return w_off(dim) + w_bytes(); }
     static __host__ __device__ size_t part_off(int dim) { return bias_off(dim) + kExitCT * sizeof(float); }
     static __host__ __device__ size_t red_off(int dim) { return part_off(dim) + (size_t)kExitBT * 8 * sizeof(float2); }
     static __host__ __device__ size_t flag_off(int dim) { return red_off(dim) + (size_t)(kExitThreads / 32) * 8 * sizeof(float); }
@@ -459,8 +532,10 @@ struct ExitClSmem {
 };
 
 template <typename T>
-__global__ void __launch_bounds__(kExitThreads) k_exit_cl(ExitParams p) {
+__global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant__ CUtensorMap wmap, ExitParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
+    __shared__ __align__(8) unsigned long long wbar[kExitWStages];
+    __shared__ int s_wfail;
     using S = ExitSmem<T>;
     using L = ExitClSmem<T>;
     constexpr int CH = Elem<T>::kPerChunk;
@@ -476,6 +551,8 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(ExitParams p) {
     T *g_s = reinterpret_cast<T *>(sm + L::g_off(dim));
     T *be_s = reinterpret_cast<T *>(sm + L::be_off(dim));
     unsigned char *w_region = sm + L::w_off(dim);
+    unsigned char *w_tma = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(w_region) + 1023) &
+                                                             ~uintptr_t(1023));   // bf16 TMA stages
     float *lg_s = reinterpret_cast<float *>(w_region);   // [kExitBT][kExitCT], reused after the GEMM
     float *bias_s = reinterpret_cast<float *>(sm + L::bias_off(dim));
     float2 *part_s = reinterpret_cast<float2 *>(sm + L::part_off(dim));
@@ -497,10 +574,9 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(ExitParams p) {
     const int j = warp / G, gt = tid - j * G * 32;   // row slot of this warp, thread index in its group
     const int sl = rank + j * ncl;
     const bool has_row = sl < kExitBT;
-    const int s = s0 + sl;
 
     if (active) {
-        // own CLS rows, gamma and beta first (group 0), then weight chunks 0 and 1
+        // own CLS rows, gamma and beta first (group 0), then the head's weight chunks
         for (int it = tid; it < kExitBT * nchunk; it += kExitThreads) {
             const int jj = it / nchunk, c = it - jj * nchunk;
             const int sli = rank + jj * ncl, si = s0 + sli;
@@ -530,15 +606,31 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(ExitParams p) {
             const int r = 8 + it / nchunk, c = it % nchunk;
             *reinterpret_cast<uint4 *>(u_s + (size_t)r * u_stride + c * CH) = make_uint4(0, 0, 0, 0);
         }
+        if (kBf16 && tid == 0) {
+            for (int q = 0; q < kExitWStages; ++q) mbar_init(smem_addr(&wbar[q]), 1);
+            s_wfail = 0;
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&wmap)) : "memory");
+        }
     }
     cl.sync();   // every CTA of the cluster runs before any remote shared-memory store
     if (active) {
         cp_async_wait_all();
         __syncthreads();
-        // the head's first two weight chunks load while the LayerNorm runs (issued only now:
-        // every CTA's 64 KB at once would hold up the CLS rows above)
-        issue_w_chunk<T>(p, w_region, c0, 0, dim, C, tid);
-        if (n_k > 1) issue_w_chunk<T>(p, w_region + S::w_stage, c0, KC, dim, C, tid);
+        // the head's first weight chunks load while the LayerNorm runs (issued only now: every
+        // CTA's 64 KB at once would hold up the CLS rows above)
+        if constexpr (kBf16) {
+            if (tid == 0) {
+                const int nk64 = (dim + 63) / 64;
+                for (int q = 0; q < kExitWStages && q < nk64; ++q) {
+                    mbar_expect_tx(smem_addr(&wbar[q]), kExitWStage);
+                    tma_load_2d(smem_addr(w_tma + (size_t)q * kExitWStage), &wmap, q * 64, c0, smem_addr(&wbar[q]));
+                }
+            }
+        } else {
+            issue_w_chunk<T>(p, w_region, c0, 0, dim, C, tid);
+            if (n_k > 1) issue_w_chunk<T>(p, w_region + S::w_stage, c0, KC, dim, C, tid);
+        }
 
         // ---- LayerNorm, G warps per row: one pass of sum and sum of squares -----------
         const int rflag = has_row ? rowflag_s[j] : 0;   // checked by the load loop above
@@ -616,7 +708,12 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(ExitParams p) {
     float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
     float acc2[4] = {0.0f, 0.0f, 0.0f, 0.0f};
     if (active) {
-        exit_gemm<T>(p, u_s, w_region, c0, dim, C, n_k, acc, acc2);
+        if constexpr (kBf16) {
+            if (!exit_gemm_tma(&wmap, u_s, w_tma, wbar, &s_wfail, c0, dim, acc, acc2) && tid == 0)
+                raise_status(p.status, FUSION_DEV_TIMEOUT);
+        } else {
+            exit_gemm<T>(p, u_s, w_region, c0, dim, C, n_k, acc, acc2);
+        }
         exit_logits<T>(p, lg_s, bias_s, acc, acc2, s0, c0, B, C);
         // partial softmax of this class tile, warp -> sample slot; to the sample's owner
         {
@@ -688,6 +785,19 @@ size_t exit_smem_bytes(int dtype, int dim) {
 
 template <typename T>
 cudaError_t launch_exit_cluster(const ExitParams &p, cudaStream_t s) {
+    CUtensorMap wmap{};
+    if (sizeof(T) == 2) {   // the head weights [C][dim] as boxes of 128 classes x 64 dims
+        EncodeTiledFn enc = encode_fn();
+        if (!enc) return cudaErrorNotSupported;
+        cuuint64_t dims[2] = {(cuuint64_t)p.dim, (cuuint64_t)p.head.classes};
+        cuuint64_t strides[1] = {(cuuint64_t)p.dim * 2};
+        cuuint32_t box[2] = {64, (cuuint32_t)kExitCT};
+        cuuint32_t estr[2] = {1, 1};
+        if (enc(&wmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(p.head.weight), dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
     const size_t smem = ExitClSmem<T>::total(p.dim);
     cudaError_t e = cudaFuncSetAttribute(k_exit_cl<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
@@ -703,7 +813,7 @@ cudaError_t launch_exit_cluster(const ExitParams &p, cudaStream_t s) {
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, k_exit_cl<T>, p);
+    return cudaLaunchKernelEx(&cfg, k_exit_cl<T>, wmap, p);
 }
 
 cudaError_t launch_exit(int dtype, const ExitParams &p, cudaStream_t s) {

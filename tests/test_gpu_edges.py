@@ -93,6 +93,25 @@ def test_degenerate_and_ragged_samples(dtype, keys):
     assert B == len(r)
 
 
+@pytest.mark.parametrize("dim,classes", [(16, 1), (80, 127), (208, 129), (384, 1000), (1024, 1000), (48, 640)])
+def test_exit_head_widths(dim, classes):
+    """The linear exit head over widths that end inside a 64-dim weight chunk (16, 80, 208),
+    class counts below, at and past a 128-class tile, and heads of one to eight tiles; tau in
+    the widest gap between the oracle's max_prob values around the median, so that about half
+    the samples exit and none sits at the threshold."""
+    rng = np.random.default_rng(dim + classes)
+    counts = rng.integers(1, 24, 41)
+    b = make_batch(counts, dim, "bf16", seed=dim, sizes="u1to4")
+    head = make_head(dim, classes, "bf16", 0.5, seed=classes, scale=2.0 / np.sqrt(dim))
+    spec = StageSpec(False, True, False, head=head)
+    o = oracle.stage(b, spec)
+    mp = np.sort(o["max_prob"])
+    lo = len(mp) // 2 - 5
+    k = lo + int(np.argmax(np.diff(mp[lo:lo + 11])))
+    head.tau = float(np.float32(0.5 * (mp[k] + mp[k + 1]))) if mp[k + 1] > mp[k] else float(mp[k])
+    run_stage_and_compare(b, StageSpec(False, True, False, head=head), f"exit head dim {dim} classes {classes}")
+
+
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 def test_identical_keys_zero_norm_and_signed_zero(dtype):
     b = make_batch([33, 20, 9], 32, dtype, same_keys=True, signed_zero_scores=True)

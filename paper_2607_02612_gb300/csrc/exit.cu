@@ -430,112 +430,76 @@ __device__ __forceinline__ float to_float(__nv_bfloat16 v) { return __bfloat162f
 
 // ---------------------------------------------------------------------------
 // The exit check as thread-block clusters: the n_ctile (<= 8) class tiles of one sample
-// tile form a cluster.  Cluster rank r computes the LayerNorm of the tile's samples
-// r, r + n_ctile, ... with several warps per row (one pass: sum and sum of squares in
-// float-float, var = E[x^2] - mean^2) and stores the normalised row into the shared
-// memory of every CTA of the cluster; each CTA then computes its logits tile and partial
-// softmax, sends (max, sum of exponentials) to the sample's owner, and the owner merges
-// them.  The head's weight chunks load while the LayerNorm runs; no global atomics
-// unless the plan kernel's work runs here (batches above the fused-plan bound).
+// tile (8 samples) form a cluster.  Cluster rank r computes the
+// LayerNorm of the tile's samples r, r + n_ctile, ... with several warps per row (one pass:
+// sum and sum of squares in float-float, var = E[x^2] - mean^2) and stores the normalised
+// row into the shared memory of every CTA of the cluster; each CTA then computes its logits
+// tile and partial softmax, sends (max, sum of exponentials) to the sample's owner, and the
+// owner merges them.  bf16: the head's weight tile arrives by TMA from the kernel's start
+// (all of it when it fits, else a ring), and the logits tile is one tcgen05 product
+// D[128 classes][16 samples] in tensor memory; float32: cp.async stages and FFMA.  No global
+// atomics unless the plan kernel's work runs here (batches above the fused-plan bound).
 // ---------------------------------------------------------------------------
-constexpr int kExitWStages = 4;                      // TMA stages of the bf16 head weights
 constexpr uint32_t kExitWStage = kExitCT * 128u;     // one stage: kExitCT rows x 64 bf16 dims
 
-// The logits tile of the cluster kernel for bf16: as exit_gemm, with the weights' K chunks
-// of 64 dims arriving by TMA (chunks 0..kExitWStages-1 already issued by thread 0).  Stage
-// st holds rows c0.. of the tile, 128 bytes each, 16-byte chunk j of row n at j ^ (n % 8);
-// classes past C and dims past dim read as zeros.  Thread 0 waits on each stage (bounded) and
-// refills it once every warp is done with it.  The MMA sequence and the partial-sum flushes
-// are those of exit_gemm.  Returns false (uniform) when a wait gave up; the copies still in
-// flight are waited for (bounded) before returning.
-__device__ __forceinline__ bool exit_gemm_tma(const CUtensorMap *wmap, const __nv_bfloat16 *u_s, unsigned char *w_tma,
-                                              unsigned long long *wbar, int *s_wfail, int c0, int dim,
-                                              float (&acc)[4], float (&acc2)[4]) {
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int u_stride = ExitSmem<__nv_bfloat16>::u_stride(dim);
-    const int nk = (dim + 63) / 64;
-    const uint32_t ubase = smem_addr(u_s);
-    const int arow = (lane & 7) + ((lane >> 3) & 1) * 8;
-    const int brow = warp * 16 + (lane >> 4) * 8 + (lane & 7);
-    const uint32_t bsw = (uint32_t)(brow & 7);
-    int kc = 0;
-    for (; kc < nk; ++kc) {
-        const int st = kc % kExitWStages;
-        if (tid == 0 && !mbar_wait(smem_addr(&wbar[st]), (uint32_t)(kc / kExitWStages) & 1u)) *s_wfail = 1;
-        __syncthreads();
-        if (*s_wfail) break;
-        const int kw = min(64, dim - kc * 64);
-        const uint32_t wrow = smem_addr(w_tma + (size_t)st * kExitWStage) + (uint32_t)brow * 128u;
-        float t0[4] = {0.0f, 0.0f, 0.0f, 0.0f}, t1[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-        for (int kk = 0; kk < kw; kk += 16) {
-            uint32_t af[4], b0, b1, b2, b3;
-            ldsm_x4(ubase + (uint32_t)((arow * u_stride + kc * 64 + kk + (lane >> 4) * 8) * 2), af[0], af[1], af[2],
-                    af[3]);
-            const uint32_t j = (uint32_t)(kk >> 3) + (uint32_t)((lane >> 3) & 1);
-            ldsm_x4(wrow + ((j ^ bsw) << 4), b0, b1, b2, b3);
-            mma_bf16_16816(t0, af, b0, b1);
-            mma_bf16_16816(t1, af, b2, b3);
-            if (kk == 48) {   // flush the partial sums every 64 dims
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    acc[e] += t0[e];
-                    acc2[e] += t1[e];
-                    t0[e] = t1[e] = 0.0f;
-                }
-            }
-        }
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            acc[e] += t0[e];
-            acc2[e] += t1[e];
-        }
-        __syncthreads();   // every warp is done with stage st
-        if (tid == 0 && kc + kExitWStages < nk) {
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            mbar_expect_tx(smem_addr(&wbar[st]), kExitWStage);
-            tma_load_2d(smem_addr(w_tma + (size_t)st * kExitWStage), wmap, (kc + kExitWStages) * 64, c0,
-                        smem_addr(&wbar[st]));
-        }
-    }
-    if (kc == nk) return true;
-    if (tid == 0)   // chunks kc.. issued and not consumed: let them land before the CTA moves on
-        for (int q = kc; q < nk && q < kc + kExitWStages; ++q)
-            (void)mbar_wait(smem_addr(&wbar[q % kExitWStages]), (uint32_t)(q / kExitWStages) & 1u);
-    __syncthreads();
-    return false;
+// Byte offset of 16-byte chunk c (8 bf16 dims) of row r in the bf16 cluster kernel's u tile:
+// K-blocks of 64 dims, each [16 rows][128 bytes] with chunk j of row r at j ^ (r % 8), the
+// K-major, 128-byte-swizzled layout of a tcgen05 operand (8-row groups 1024 bytes apart).
+__device__ __forceinline__ uint32_t u_tc_off(int r, int c) {
+    return (uint32_t)(c >> 3) * 2048u + (uint32_t)r * 128u + ((uint32_t)((c & 7) ^ (r & 7)) << 4);
 }
+constexpr uint32_t kExitTmemCols = 32;   // D: 128 classes (lanes) x 16 samples (columns)
+constexpr int kExitClMaxW = 16;          // most weight stages of the bf16 cluster kernel
+constexpr size_t kExitClBudget = 112 * 1024;   // its dynamic shared memory bound (two CTAs per SM)
 
 template <typename T>
 struct ExitClSmem {
     static constexpr int EB = Elem<T>::kBytes;
+    static constexpr bool kTc = EB == 2;
+    // samples per cluster (the tensor-memory product's N = 16 carries 8 of them: with 16,
+    // a CTA needs the SM for itself and the clusters no longer fit in one wave)
+    static constexpr int BT = kExitBT;
     using B = ExitSmem<T>;
-    // u rows (16, the GEMM's A tile) | own raw CLS rows (kExitBT) | gamma | beta | W stages (2)
-    // | bias | partials [kExitBT][8] | reduction scratch
-    static __host__ __device__ size_t x_off(int dim) { return B::u_bytes(dim); }
-    static __host__ __device__ size_t g_off(int dim) { return x_off(dim) + (size_t)kExitBT * B::u_stride(dim) * EB; }
-    static __host__ __device__ size_t be_off(int dim) { return g_off(dim) + ((size_t)dim * EB + 15) / 16 * 16; }
-    static __host__ __device__ size_t w_off(int dim) { return be_off(dim) + ((size_t)dim * EB + 15) / 16 * 16; }
-    // bf16: kExitWStages TMA stages of [kExitCT rows][64 dims] (128-byte rows, 128-byte swizzle,
-    // 1024-byte aligned inside the region); float32: two cp.async stages
-    static __host__ __device__ size_t w_bytes() {
-        return EB == 2 ? (size_t)kExitWStages * kExitWStage + 1024 : 2 * B::w_stage;
+    // u tile (16 GEMM rows; bf16: swizzled K-blocks) | W stages (bf16: w_stages(dim) TMA stages,
+    // the whole tile when it fits; float32: two cp.async stages) | own raw CLS rows (BT) | gamma |
+    // beta | bias | partials [BT][8] | reduction scratch | row flags.  bf16 offsets count from a
+    // 1024-byte aligned base (the total includes the slack).
+    static __host__ __device__ size_t u_bytes(int dim) { return kTc ? (size_t)((dim + 63) / 64) * 2048 : B::u_bytes(dim); }
+    static __host__ __device__ size_t rest_bytes(int dim) {   // everything but the W stages
+        return u_bytes(dim) + (size_t)BT * B::u_stride(dim) * EB + 2 * (((size_t)dim * EB + 15) / 16 * 16) +
+               kExitCT * sizeof(float) + (size_t)BT * 8 * sizeof(float2) + (kExitThreads / 32) * 8 * sizeof(float) +
+               (size_t)BT * sizeof(int);
     }
-    static __host__ __device__ size_t bias_off(int dim) { return w_off(dim) + w_bytes(); }
+    static __host__ __device__ int w_stages(int dim) {
+        if (!kTc) return 2;
+        const int nk = (dim + 63) / 64;
+        const size_t rest = rest_bytes(dim) + 1024;
+        int st = rest + 2 * kExitWStage <= kExitClBudget ? (int)((kExitClBudget - rest) / kExitWStage) : 2;
+        st = st < kExitClMaxW ? st : kExitClMaxW;
+        return nk < st ? nk : st;
+    }
+    static __host__ __device__ size_t w_bytes(int dim) { return kTc ? (size_t)w_stages(dim) * kExitWStage : 2 * B::w_stage; }
+    static __host__ __device__ size_t w_off(int dim) { return u_bytes(dim); }
+    static __host__ __device__ size_t x_off(int dim) { return w_off(dim) + w_bytes(dim); }
+    static __host__ __device__ size_t g_off(int dim) { return x_off(dim) + (size_t)BT * B::u_stride(dim) * EB; }
+    static __host__ __device__ size_t be_off(int dim) { return g_off(dim) + ((size_t)dim * EB + 15) / 16 * 16; }
+    static __host__ __device__ size_t bias_off(int dim) { return be_off(dim) + ((size_t)dim * EB + 15) / 16 * 16; }
     static __host__ __device__ size_t part_off(int dim) { return bias_off(dim) + kExitCT * sizeof(float); }
-    static __host__ __device__ size_t red_off(int dim) { return part_off(dim) + (size_t)kExitBT * 8 * sizeof(float2); }
+    static __host__ __device__ size_t red_off(int dim) { return part_off(dim) + (size_t)BT * 8 * sizeof(float2); }
     static __host__ __device__ size_t flag_off(int dim) { return red_off(dim) + (size_t)(kExitThreads / 32) * 8 * sizeof(float); }
     static __host__ __device__ size_t total(int dim) {
-        const size_t t = flag_off(dim) + (size_t)kExitBT * sizeof(int);
+        const size_t t = flag_off(dim) + (size_t)BT * sizeof(int);
         const size_t plan = w_off(dim) + (4 * kExitThreads + 40) * sizeof(int);   // run_plan reuses the W stages
-        return t > plan ? t : plan;
+        return (t > plan ? t : plan) + (kTc ? 1024 : 0);
     }
 };
 
 template <typename T>
 __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant__ CUtensorMap wmap, ExitParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
-    __shared__ __align__(8) unsigned long long wbar[kExitWStages];
+    __shared__ __align__(8) unsigned long long wbar[kExitClMaxW], wempty[kExitClMaxW], wdone;
     __shared__ int s_wfail;
+    __shared__ uint32_t tmem_base;
     using S = ExitSmem<T>;
     using L = ExitClSmem<T>;
     constexpr int CH = Elem<T>::kPerChunk;
@@ -543,46 +507,69 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
     constexpr int KC = S::KC;
     constexpr bool kBf16 = (EB == 2);
     constexpr int kWarps = kExitThreads / 32;
+    constexpr int BT = L::BT;
     cg::cluster_group cl = cg::this_cluster();
     const int ncl = (int)cl.num_blocks(), rank = (int)cl.block_rank();
     const int dim = p.dim, nchunk = dim / CH, u_stride = S::u_stride(dim);
-    T *u_s = reinterpret_cast<T *>(sm);
-    T *x_s = reinterpret_cast<T *>(sm + L::x_off(dim));
-    T *g_s = reinterpret_cast<T *>(sm + L::g_off(dim));
-    T *be_s = reinterpret_cast<T *>(sm + L::be_off(dim));
-    unsigned char *w_region = sm + L::w_off(dim);
-    unsigned char *w_tma = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(w_region) + 1023) &
-                                                             ~uintptr_t(1023));   // bf16 TMA stages
-    float *lg_s = reinterpret_cast<float *>(w_region);   // [kExitBT][kExitCT], reused after the GEMM
-    float *bias_s = reinterpret_cast<float *>(sm + L::bias_off(dim));
-    float2 *part_s = reinterpret_cast<float2 *>(sm + L::part_off(dim));
-    float *red = reinterpret_cast<float *>(sm + L::red_off(dim));
-    int *rowflag_s = reinterpret_cast<int *>(sm + L::flag_off(dim));   // [kExitBT]: 1 row, 0 none, -1 bad
+    unsigned char *base = kBf16 ? reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(sm) + 1023) &
+                                                                    ~uintptr_t(1023))
+                                : sm;
+    T *u_s = reinterpret_cast<T *>(base);   // float32: [16][u_stride]; bf16: see u_tc_off
+    T *x_s = reinterpret_cast<T *>(base + L::x_off(dim));
+    T *g_s = reinterpret_cast<T *>(base + L::g_off(dim));
+    T *be_s = reinterpret_cast<T *>(base + L::be_off(dim));
+    unsigned char *w_region = base + L::w_off(dim);   // bf16: 1024-byte aligned TMA stages
+    float *lg_s = reinterpret_cast<float *>(w_region);   // [BT][kExitCT], reused after the GEMM
+    float *bias_s = reinterpret_cast<float *>(base + L::bias_off(dim));
+    float2 *part_s = reinterpret_cast<float2 *>(base + L::part_off(dim));
+    float *red = reinterpret_cast<float *>(base + L::red_off(dim));
+    int *rowflag_s = reinterpret_cast<int *>(base + L::flag_off(dim));   // [BT]: 1 row, 0 none, -1 bad
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int ct = blockIdx.x, bt = blockIdx.y;
-    const int s0 = bt * kExitBT, c0 = ct * kExitCT;
+    const int s0 = bt * BT, c0 = ct * kExitCT;
     const int C = p.head.classes;
     const int Bdev = device_batch(p.in);
     const int B = Bdev < 0 ? 0 : Bdev;
     const bool active = s0 < B;   // uniform over the cluster (same sample tile)
     const int n_k = (dim + KC - 1) / KC;
-    // rows of this CTA: slot j -> sample slot sl = rank + j * ncl; G warps per row
+    // rows of this CTA: slot j -> sample slot sl = rank + j * ncl (nrp slots, a power of two);
+    // G >= 1 warps per row, ngr = kWarps / G rows at a time
     int nrp = 1;
-    while (nrp * ncl < kExitBT) nrp <<= 1;
-    const int G = kWarps / nrp;
-    const int j = warp / G, gt = tid - j * G * 32;   // row slot of this warp, thread index in its group
-    const int sl = rank + j * ncl;
-    const bool has_row = sl < kExitBT;
+    while (nrp * ncl < BT) nrp <<= 1;
+    const int G = nrp >= kWarps ? 1 : kWarps / nrp;
+    const int ngr = kWarps / G;
+    const int jw = warp / G, gt = tid - jw * G * 32;   // row of this warp in a round, thread index in its group
 
+    if (active && kBf16 && warp == 0) {   // the logits tile's accumulator
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(&tmem_base)),
+                     "r"(kExitTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    if (active && kBf16 && tid == 0) {
+        // the head's first weight chunks first: they depend on nothing and take longest to land
+        const int nws = L::w_stages(dim);
+        for (int q = 0; q < nws; ++q) {
+            mbar_init(smem_addr(&wbar[q]), 1);
+            mbar_init(smem_addr(&wempty[q]), 1);
+        }
+        mbar_init(smem_addr(&wdone), 1);
+        s_wfail = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        for (int q = 0; q < nws; ++q) {
+            mbar_expect_tx(smem_addr(&wbar[q]), kExitWStage);
+            tma_load_2d(smem_addr(w_region + (size_t)q * kExitWStage), &wmap, q * 64, c0, smem_addr(&wbar[q]));
+        }
+    }
     if (active) {
-        // own CLS rows, gamma and beta first (group 0), then the head's weight chunks
-        for (int it = tid; it < kExitBT * nchunk; it += kExitThreads) {
+        // own CLS rows, gamma and beta (group 0), then the bias
+        for (int it = tid; it < BT * nchunk; it += kExitThreads) {
             const int jj = it / nchunk, c = it - jj * nchunk;
             const int sli = rank + jj * ncl, si = s0 + sli;
             T *dst = x_s + (size_t)jj * u_stride + c * CH;
             long long row = -1;
-            const bool want = sli < kExitBT && si < B;
+            const bool want = sli < BT && si < B;
             if (want) {
                 row = p.in.offsets[si];
                 if (row < 0 || row >= p.in.max_rows) row = -1;
@@ -599,125 +586,197 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
             cp_async16((isg ? g_s : be_s) + cc * CH,
                        reinterpret_cast<const T *>(isg ? p.head.gamma : p.head.beta) + cc * CH);
         }
+        for (int c = tid; c < kExitCT; c += kExitThreads) {
+            if (c0 + c < C)
+                cp_async4(bias_s + c, p.head.bias + c0 + c);
+            else
+                bias_s[c] = 0.0f;
+        }
         cp_async_commit();
-        for (int c = tid; c < kExitCT; c += kExitThreads) bias_s[c] = (c0 + c < C) ? p.head.bias[c0 + c] : 0.0f;
-        // padding rows 8..15 of the GEMM's A tile
-        for (int it = tid; it < 8 * nchunk; it += kExitThreads) {
+        // padding rows 8..15 of the GEMM's A tile (float32; for bf16 they feed only the unused
+        // columns 8..15 of the tensor-memory product)
+        for (int it = tid; !kBf16 && it < 8 * nchunk; it += kExitThreads) {
             const int r = 8 + it / nchunk, c = it % nchunk;
             *reinterpret_cast<uint4 *>(u_s + (size_t)r * u_stride + c * CH) = make_uint4(0, 0, 0, 0);
-        }
-        if (kBf16 && tid == 0) {
-            for (int q = 0; q < kExitWStages; ++q) mbar_init(smem_addr(&wbar[q]), 1);
-            s_wfail = 0;
-            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&wmap)) : "memory");
         }
     }
     cl.sync();   // every CTA of the cluster runs before any remote shared-memory store
     if (active) {
         cp_async_wait_all();
         __syncthreads();
-        // the head's first weight chunks load while the LayerNorm runs (issued only now: every
-        // CTA's 64 KB at once would hold up the CLS rows above)
-        if constexpr (kBf16) {
-            if (tid == 0) {
-                const int nk64 = (dim + 63) / 64;
-                for (int q = 0; q < kExitWStages && q < nk64; ++q) {
-                    mbar_expect_tx(smem_addr(&wbar[q]), kExitWStage);
-                    tma_load_2d(smem_addr(w_tma + (size_t)q * kExitWStage), &wmap, q * 64, c0, smem_addr(&wbar[q]));
-                }
-            }
-        } else {
+        // float32: the head's first two weight chunks load while the LayerNorm runs (issued
+        // only now: every CTA's 64 KB of cp.async at once would hold up the CLS rows above)
+        if constexpr (!kBf16) {
             issue_w_chunk<T>(p, w_region, c0, 0, dim, C, tid);
             if (n_k > 1) issue_w_chunk<T>(p, w_region + S::w_stage, c0, KC, dim, C, tid);
         }
 
         // ---- LayerNorm, G warps per row: one pass of sum and sum of squares -----------
-        const int rflag = has_row ? rowflag_s[j] : 0;   // checked by the load loop above
-        if (rflag < 0 && gt == 0) raise_status(p.status, FUSION_DEV_BAD_OFFSETS);
-        const bool ok = rflag > 0;
-        const F2 rdim = f2_recip((float)dim);
-        const T *xr = x_s + (size_t)j * u_stride;
-        float s1 = 0.0f, c1 = 0.0f, s2 = 0.0f, c2 = 0.0f, l2 = 0.0f;
-        if (ok) {
-            for (int e = gt; e < dim; e += G * 32) {
-                const float v = to_float(xr[e]);
-                neu_add(s1, c1, v);
-                const F2 sq = two_prod(v, v);
-                neu_add(s2, c2, sq.hi);
-                l2 = __fadd_rn(l2, sq.lo);
-            }
-        }
-        F2 a1 = warp_sum_f2(two_sum(s1, c1));
-        F2 a2 = warp_sum_f2(f2_add_f(two_sum(s2, c2), l2));
-        if (lane == 0) {
-            red[warp * 8 + 0] = a1.hi;
-            red[warp * 8 + 1] = a1.lo;
-            red[warp * 8 + 2] = a2.hi;
-            red[warp * 8 + 3] = a2.lo;
-        }
-        __syncthreads();
-        if (ok) {
-            // the group's G (a power of two) warp sums: every aligned run of G lanes adds them
-            // as a butterfly, so all lanes hold the same bits (f2_add is symmetric)
-            const int wq = j * G + (lane & (G - 1));
-            F2 t1 = {red[wq * 8 + 0], red[wq * 8 + 1]}, t2 = {red[wq * 8 + 2], red[wq * 8 + 3]};
-            for (int m = G >> 1; m >= 1; m >>= 1) {
-                t1 = f2_add(t1, f2_shfl_xor(t1, m));
-                t2 = f2_add(t2, f2_shfl_xor(t2, m));
-            }
-            const F2 mean = f2_mul(t1, rdim);
-            const F2 ex2 = f2_mul(t2, rdim);
-            const F2 m2 = f2_mul(mean, mean);
-            F2 var = f2_add(ex2, {-m2.hi, -m2.lo});
-            if (var.hi < 0.0f) var = {0.0f, 0.0f};
-            const F2 rstd = f2_rsqrt(f2_add_f(var, p.head.eps));
-            if (gt == 0 && !(isfinite(mean.hi) && isfinite(var.hi))) raise_status(p.status, FUSION_DEV_NONFINITE);
-            for (int c = gt; c < nchunk; c += G * 32) {
-                float f[CH], gf[CH], bf[CH];
-                chunk_to_f(*reinterpret_cast<const uint4 *>(xr + c * CH), f);
-                chunk_to_f(*reinterpret_cast<const uint4 *>(g_s + c * CH), gf);
-                chunk_to_f(*reinterpret_cast<const uint4 *>(be_s + c * CH), bf);
-                uint4 outv;
-                if constexpr (kBf16) {
-                    uint32_t w4[4];
-#pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        w4[q] = (uint32_t)ln_out_bf16(f[2 * q], mean, rstd, gf[2 * q], bf[2 * q]) |
-                                ((uint32_t)ln_out_bf16(f[2 * q + 1], mean, rstd, gf[2 * q + 1], bf[2 * q + 1]) << 16);
-                    outv = make_uint4(w4[0], w4[1], w4[2], w4[3]);
-                } else {
-                    outv = make_uint4(__float_as_uint(ln_out_f32(f[0], mean, rstd, gf[0], bf[0])),
-                                      __float_as_uint(ln_out_f32(f[1], mean, rstd, gf[1], bf[1])),
-                                      __float_as_uint(ln_out_f32(f[2], mean, rstd, gf[2], bf[2])),
-                                      __float_as_uint(ln_out_f32(f[3], mean, rstd, gf[3], bf[3])));
+        for (int jb = 0; jb < nrp; jb += ngr) {   // rounds of ngr rows (uniform trip count)
+            const int j = jb + jw, sl = rank + j * ncl;
+            const bool has_row = j < nrp && sl < BT;
+            const int rflag = has_row ? rowflag_s[j] : 0;   // checked by the load loop above
+            if (rflag < 0 && gt == 0) raise_status(p.status, FUSION_DEV_BAD_OFFSETS);
+            const bool ok = rflag > 0;
+            const F2 rdim = f2_recip((float)dim);
+            const T *xr = x_s + (size_t)j * u_stride;
+            float s1 = 0.0f, c1 = 0.0f, s2 = 0.0f, c2 = 0.0f, l2 = 0.0f;
+            if (ok) {
+                for (int e = gt; e < dim; e += G * 32) {
+                    const float v = to_float(xr[e]);
+                    neu_add(s1, c1, v);
+                    const F2 sq = two_prod(v, v);
+                    neu_add(s2, c2, sq.hi);
+                    l2 = __fadd_rn(l2, sq.lo);
                 }
-                T *dst = u_s + (size_t)sl * u_stride + c * CH;
-                for (int r = 0; r < ncl; ++r) *reinterpret_cast<uint4 *>(cl.map_shared_rank(dst, r)) = outv;
             }
-        } else if (has_row) {
-            for (int c = gt; c < nchunk; c += G * 32) {
-                T *dst = u_s + (size_t)sl * u_stride + c * CH;
-                for (int r = 0; r < ncl; ++r)
-                    *reinterpret_cast<uint4 *>(cl.map_shared_rank(dst, r)) = make_uint4(0, 0, 0, 0);
+            F2 a1 = warp_sum_f2(two_sum(s1, c1));
+            F2 a2 = warp_sum_f2(f2_add_f(two_sum(s2, c2), l2));
+            if (lane == 0) {
+                red[warp * 8 + 0] = a1.hi;
+                red[warp * 8 + 1] = a1.lo;
+                red[warp * 8 + 2] = a2.hi;
+                red[warp * 8 + 3] = a2.lo;
             }
+            __syncthreads();
+            if (ok) {
+                // the group's G (a power of two) warp sums: every aligned run of G lanes adds them
+                // as a butterfly, so all lanes hold the same bits (f2_add is symmetric)
+                const int wq = jw * G + (lane & (G - 1));
+                F2 t1 = {red[wq * 8 + 0], red[wq * 8 + 1]}, t2 = {red[wq * 8 + 2], red[wq * 8 + 3]};
+                for (int m = G >> 1; m >= 1; m >>= 1) {
+                    t1 = f2_add(t1, f2_shfl_xor(t1, m));
+                    t2 = f2_add(t2, f2_shfl_xor(t2, m));
+                }
+                const F2 mean = f2_mul(t1, rdim);
+                const F2 ex2 = f2_mul(t2, rdim);
+                const F2 m2 = f2_mul(mean, mean);
+                F2 var = f2_add(ex2, {-m2.hi, -m2.lo});
+                if (var.hi < 0.0f) var = {0.0f, 0.0f};
+                const F2 rstd = f2_rsqrt(f2_add_f(var, p.head.eps));
+                if (gt == 0 && !(isfinite(mean.hi) && isfinite(var.hi))) raise_status(p.status, FUSION_DEV_NONFINITE);
+                for (int c = gt; c < nchunk; c += G * 32) {
+                    float f[CH], gf[CH], bf[CH];
+                    chunk_to_f(*reinterpret_cast<const uint4 *>(xr + c * CH), f);
+                    chunk_to_f(*reinterpret_cast<const uint4 *>(g_s + c * CH), gf);
+                    chunk_to_f(*reinterpret_cast<const uint4 *>(be_s + c * CH), bf);
+                    uint4 outv;
+                    if constexpr (kBf16) {
+                        uint32_t w4[4];
+    #pragma unroll
+                        for (int q = 0; q < 4; ++q)
+                            w4[q] = (uint32_t)ln_out_bf16(f[2 * q], mean, rstd, gf[2 * q], bf[2 * q]) |
+                                    ((uint32_t)ln_out_bf16(f[2 * q + 1], mean, rstd, gf[2 * q + 1], bf[2 * q + 1]) << 16);
+                        outv = make_uint4(w4[0], w4[1], w4[2], w4[3]);
+                    } else {
+                        outv = make_uint4(__float_as_uint(ln_out_f32(f[0], mean, rstd, gf[0], bf[0])),
+                                          __float_as_uint(ln_out_f32(f[1], mean, rstd, gf[1], bf[1])),
+                                          __float_as_uint(ln_out_f32(f[2], mean, rstd, gf[2], bf[2])),
+                                          __float_as_uint(ln_out_f32(f[3], mean, rstd, gf[3], bf[3])));
+                    }
+                    T *dst = kBf16 ? reinterpret_cast<T *>(base + u_tc_off(sl, c)) : u_s + (size_t)sl * u_stride + c * CH;
+                    for (int r = 0; r < ncl; ++r) *reinterpret_cast<uint4 *>(cl.map_shared_rank(dst, r)) = outv;
+                }
+            } else if (has_row) {
+                for (int c = gt; c < nchunk; c += G * 32) {
+                    T *dst = kBf16 ? reinterpret_cast<T *>(base + u_tc_off(sl, c)) : u_s + (size_t)sl * u_stride + c * CH;
+                    for (int r = 0; r < ncl; ++r)
+                        *reinterpret_cast<uint4 *>(cl.map_shared_rank(dst, r)) = make_uint4(0, 0, 0, 0);
+                }
+            }
+            __syncthreads();   // the reduction scratch is reused by the next round
         }
     }
+    // bf16: the u tile, written by the generic proxy here and in the other CTAs, is read by the
+    // tensor core (async proxy) after the barrier
+    if constexpr (kBf16) asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
     cl.sync();   // all LayerNorm rows are in every CTA's shared memory
 
     float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
     float acc2[4] = {0.0f, 0.0f, 0.0f, 0.0f};
     if (active) {
         if constexpr (kBf16) {
-            if (!exit_gemm_tma(&wmap, u_s, w_tma, wbar, &s_wfail, c0, dim, acc, acc2) && tid == 0)
-                raise_status(p.status, FUSION_DEV_TIMEOUT);
+            // ---- D[128 classes][16 samples] = W_tile u^T on tcgen05, issued by one thread: per
+            // 64-dim chunk, wait for its weight stage, four MMAs (K = 16), commit; a stage is
+            // refilled by TMA once its MMAs completed.  Every wait is bounded; after a failure
+            // the copies and products in flight are waited for before anything else runs.
+            const uint32_t tmem = tmem_base;
+            if (tid == 0) {
+                const int nk = (dim + 63) / 64;
+                const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(16 >> 3) << 17) | (8u << 24);
+                const uint32_t ub = smem_addr(base);
+                const int nws = L::w_stages(dim);
+                bool okw = true;
+                int waited = 0, issued = 0, loaded = nws;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                for (int kc = 0; kc < nk; ++kc) {
+                    const int st = kc % nws;
+                    const uint32_t ph = (uint32_t)(kc / nws) & 1u;
+                    if (!mbar_wait(smem_addr(&wbar[st]), ph)) {
+                        okw = false;
+                        break;
+                    }
+                    waited = kc + 1;
+                    const uint32_t a0 = smem_addr(w_region + (size_t)st * kExitWStage), b0 = ub + (uint32_t)kc * 2048u;
+                    const int kw = min(64, dim - kc * 64);
+                    for (int k = 0; k * 16 < kw; ++k)
+                        umma_bf16(tmem, sw128_desc(a0 + k * 32), sw128_desc(b0 + k * 32), idesc, (kc | k) ? 1u : 0u);
+                    umma_commit(smem_addr(&wempty[st]));
+                    issued = kc + 1;
+                    if (kc + nws < nk) {   // the tile is not resident: refill this stage
+                        if (!mbar_wait(smem_addr(&wempty[st]), ph)) {
+                            okw = false;
+                            break;
+                        }
+                        mbar_expect_tx(smem_addr(&wbar[st]), kExitWStage);
+                        tma_load_2d(smem_addr(w_region + (size_t)st * kExitWStage), &wmap, (kc + nws) * 64, c0,
+                                    smem_addr(&wbar[st]));
+                        loaded = kc + nws + 1;
+                    }
+                }
+                if (okw) {
+                    umma_commit(smem_addr(&wdone));
+                    okw = mbar_wait(smem_addr(&wdone), 0u);
+                }
+                if (!okw) {
+                    for (int q = waited; q < loaded; ++q)
+                        (void)mbar_wait(smem_addr(&wbar[q % nws]), (uint32_t)(q / nws) & 1u);
+                    if (issued > 0)
+                        (void)mbar_wait(smem_addr(&wempty[(issued - 1) % nws]), (uint32_t)((issued - 1) / nws) & 1u);
+                    raise_status(p.status, FUSION_DEV_TIMEOUT);
+                }
+                s_wfail = okw ? 0 : 1;
+            }
+            __syncthreads();
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            // logits (+ bias) into shared memory: warp w < 4 reads the lanes (classes) 32w.. of D
+            if (warp < 4) {
+                uint32_t v[16];
+                tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16), v);
+                const int cls = warp * 32 + lane;
+#pragma unroll
+                for (int n = 0; n < BT; ++n)
+                    lg_s[n * kExitCT + cls] = (c0 + cls < C) ? __uint_as_float(v[n]) + bias_s[cls] : -INFINITY;
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncthreads();
+            if (warp == 0)
+                asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kExitTmemCols)
+                             : "memory");
+            if (p.logits) {
+                for (int it = tid; it < BT * kExitCT; it += kExitThreads) {
+                    const int sl = it / kExitCT, col = it - sl * kExitCT;
+                    if (s0 + sl < B && c0 + col < C) p.logits[(size_t)(s0 + sl) * C + c0 + col] = lg_s[it];
+                }
+            }
         } else {
             exit_gemm<T>(p, u_s, w_region, c0, dim, C, n_k, acc, acc2);
+            exit_logits<T>(p, lg_s, bias_s, acc, acc2, s0, c0, B, C);
         }
-        exit_logits<T>(p, lg_s, bias_s, acc, acc2, s0, c0, B, C);
-        // partial softmax of this class tile, warp -> sample slot; to the sample's owner
-        {
-            const int slw = warp, sw = s0 + slw;
+        // partial softmax of this class tile, warp -> sample slots warp, warp + 8, ...; to the
+        // sample's owner
+        for (int slw = warp; slw < BT; slw += kWarps) {
+            const int sw = s0 + slw;
             float m = -INFINITY;
             for (int col = lane; col < kExitCT; col += 32) m = fmaxf(m, lg_s[slw * kExitCT + col]);
 #pragma unroll
@@ -733,8 +792,8 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
         }
     }
     cl.sync();   // every partial is with its owner
-    if (active) {
-        const int slw = warp, sw = s0 + slw;
+    for (int slw = warp; active && slw < BT; slw += kWarps) {
+        const int sw = s0 + slw;
         if (slw % ncl == rank && sw < B) {
             float m = -INFINITY;
             for (int q = lane; q < ncl; q += 32) m = fmaxf(m, part_s[slw * 8 + q].x);
@@ -801,8 +860,10 @@ cudaError_t launch_exit_cluster(const ExitParams &p, cudaStream_t s) {
     const size_t smem = ExitClSmem<T>::total(p.dim);
     cudaError_t e = cudaFuncSetAttribute(k_exit_cl<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
+    ExitParams q = p;   // sample tiles of this kernel's size (the plan's cluster count)
+    q.n_btile = (p.in.max_batch + ExitClSmem<T>::BT - 1) / ExitClSmem<T>::BT;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(p.n_ctile, p.n_btile);
+    cfg.gridDim = dim3(q.n_ctile, q.n_btile);
     cfg.blockDim = dim3(kExitThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
@@ -813,7 +874,7 @@ cudaError_t launch_exit_cluster(const ExitParams &p, cudaStream_t s) {
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, k_exit_cl<T>, wmap, p);
+    return cudaLaunchKernelEx(&cfg, k_exit_cl<T>, wmap, q);
 }
 
 cudaError_t launch_exit(int dtype, const ExitParams &p, cudaStream_t s) {

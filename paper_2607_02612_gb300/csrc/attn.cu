@@ -79,7 +79,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     __shared__ __align__(8) unsigned long long bar_ld, bar_s, bar_o;
     __shared__ uint32_t tmem_base;
     __shared__ int s_fail, s_issued;   // s_issued: operations started (for the drain on a timeout)
-    __shared__ float lsz[kAttnMaxN];   // log2 of the key sizes
+    __shared__ __align__(16) float lsz[kAttnMaxN];   // log2 of the key sizes
     __shared__ float red[2][128];      // the two column halves' row maxima, then row sums
     __shared__ float s_lszmax;         // max_j log2 s_j
 
@@ -204,7 +204,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         mx = fmaf(fmaxf(red[0][r], red[1][r]), kScale2, s_lszmax);
         // ---- P = 2^(logit - max) as bf16 pairs, and the row sum; P goes over S's first columns once
         // ---- every S column of the row has been read (the other half reads some of them) ----------
-        float lsum = 0.0f;
+        float2 lsum2 = make_float2(0.0f, 0.0f);   // even and odd columns (packed float32 pairs)
         uint32_t pk[8][8];   // this half's chunks, at most 8
         if (rows_here) {
 #pragma unroll
@@ -215,7 +215,14 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
                     tmem_ld16(lane_addr + (uint32_t)(16 * c), v);
                     float pr[16];
 #pragma unroll
-                    for (int e = 0; e < 16; ++e) pr[e] = ex2(fmaf(__uint_as_float(v[e]), kScale2, lsz[16 * c + e]) - mx);
+                    for (int e = 0; e < 16; e += 2) {   // fma then subtract, two columns per instruction
+                        const float2 x = __fadd2_rn(
+                            __ffma2_rn(make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])),
+                                       make_float2(kScale2, kScale2), *reinterpret_cast<const float2 *>(&lsz[16 * c + e])),
+                            make_float2(-mx, -mx));
+                        pr[e] = ex2(x.x);
+                        pr[e + 1] = ex2(x.y);
+                    }
                     if (16 * c + 16 > n) {
 #pragma unroll
                         for (int e = 0; e < 16; ++e)
@@ -223,7 +230,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
                     }
 #pragma unroll
                     for (int e = 0; e < 16; e += 2) {
-                        lsum += pr[e] + pr[e + 1];
+                        lsum2 = __fadd2_rn(lsum2, make_float2(pr[e], pr[e + 1]));
                         const __nv_bfloat162 b2 = __floats2bfloat162_rn(pr[e], pr[e + 1]);
                         pk[q][e >> 1] = *reinterpret_cast<const uint32_t *>(&b2);
                     }
@@ -237,10 +244,10 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
                 if (c_lo + q < c_hi) tmem_st8(lane_addr + (uint32_t)(8 * (c_lo + q)), pk[q]);
             asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         }
-        red[half][r] = lsum;
+        red[half][r] = lsum2.x + lsum2.y;
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
         __syncthreads();   // all of P stored before the second product
-        lsum = red[0][r] + red[1][r];
+        const float lsum = red[0][r] + red[1][r];
         // ---- O = P V into columns [128, 192) ---------------------------------------------------
         const bool ok_s = s_fail == 0;   // the S waits' outcome, after the barrier above
         if (tid == 0 && ok_s) {
@@ -311,7 +318,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     __shared__ __align__(8) unsigned long long bar_ld[2], bar_s, bar_o;
     __shared__ uint32_t tmem_base;
     __shared__ int s_fail, s_ld, s_ns, s_no;   // steps whose loads were issued; products S and O issued
-    __shared__ float lsz[kLongMaxN];
+    __shared__ __align__(16) float lsz[kLongMaxN];
     __shared__ float red[2][128];
     __shared__ float s_lszmax;
 
@@ -392,7 +399,8 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     constexpr float kScale2 = 0.18033688011112042f;   // log2(e) / sqrt(64)
     const uint32_t idesc_o =
         (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) | ((uint32_t)(kAttnDh >> 3) << 17) | (8u << 24);
-    float mraw = -INFINITY, mx = 0.0f, lsum = 0.0f;
+    float mraw = -INFINITY, mx = 0.0f;
+    float2 lsum2 = make_float2(0.0f, 0.0f);   // even and odd columns (packed float32 pairs)
     bool stop = false;
     for (int k = 0; k < steps && !stop; ++k) {
         const int t = k / (2 * nkv), pass = (k / nkv) & 1, kb = k % nkv;
@@ -459,13 +467,18 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
                         tmem_ld16(lane_addr + (uint32_t)(16 * c), v);
                         float pr[16];
 #pragma unroll
-                        for (int e = 0; e < 16; ++e)
-                            pr[e] = 16 * c + e < rows_k
-                                        ? ex2(fmaf(__uint_as_float(v[e]), kScale2, lsz[128 * kb + 16 * c + e]) - mx)
-                                        : 0.0f;
+                        for (int e = 0; e < 16; e += 2) {   // fma then subtract, two columns per instruction
+                            const float2 x = __fadd2_rn(
+                                __ffma2_rn(make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])),
+                                           make_float2(kScale2, kScale2),
+                                           *reinterpret_cast<const float2 *>(&lsz[128 * kb + 16 * c + e])),
+                                make_float2(-mx, -mx));
+                            pr[e] = 16 * c + e < rows_k ? ex2(x.x) : 0.0f;
+                            pr[e + 1] = 16 * c + e + 1 < rows_k ? ex2(x.y) : 0.0f;
+                        }
 #pragma unroll
                         for (int e = 0; e < 16; e += 2) {
-                            lsum += pr[e] + pr[e + 1];
+                            lsum2 = __fadd2_rn(lsum2, make_float2(pr[e], pr[e + 1]));
                             const __nv_bfloat162 b2 = __floats2bfloat162_rn(pr[e], pr[e + 1]);
                             pk[q][e >> 1] = *reinterpret_cast<const uint32_t *>(&b2);
                         }
@@ -494,7 +507,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             if (kb == nkv - 1) {
                 // ---- the tile's epilogue: O / row sum -> bf16 --------------------------------------
-                red[half][r] = lsum;
+                red[half][r] = lsum2.x + lsum2.y;
                 __syncthreads();
                 const float l = red[0][r] + red[1][r];
                 if (rows_here && s_fail == 0) {
@@ -521,7 +534,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
                     }
                 }
                 mraw = -INFINITY;
-                lsum = 0.0f;
+                lsum2 = make_float2(0.0f, 0.0f);
             }
         }
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");

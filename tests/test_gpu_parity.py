@@ -212,20 +212,23 @@ def _host_copy(res):
     return r
 
 
-def test_pipeline_overlapped_steps():
+@pytest.mark.parametrize("name,B", [("deit_s_chain12_bf16_b256", 64), ("ragged_b8192_n65_chain4_f32", 256)])
+def test_pipeline_overlapped_steps(name, B):
     """Steps submitted back to back through the two-slot pipeline (input copies overlapping the
     previous step's kernels, results one step late) give, step by step, the results of the same
-    inputs run one at a time; those match the oracle's chain for both inputs."""
-    wa = make_workload("deit_s_chain12_bf16_b256", batch=64)
-    wb = type(wa)(wa.spec, make_workload("deit_s_chain12_bf16_b256", batch=64, seed_offset=1).batch, wa.stages)
+    inputs run one at a time; those match the oracle's chain for both inputs.  The DeiT-S bf16
+    schedule and the float32 65-token schedule with an exit check at every block."""
+    wa = make_workload(name, batch=B)
+    wb = type(wa)(wa.spec, make_workload(name, batch=B, seed_offset=1).batch, wa.stages)
     b = wa.batch
     assert np.array_equal(b.offsets, wb.batch.offsets)
+    bf = b.dtype == "bf16"
     fzr = runner.Fusion(b.batch, max(s.head.classes for s in wa.stages if s.head is not None))
     stages = [runner.ChainStage(P.flags_of(s), *P.stage_tensors(s, b.dtype)) for s in wa.stages]
     ch = runner.Chain(fzr, P.device_batch(b), stages)
 
     def pinned(bb):
-        return {"x": torch.from_numpy(np.ascontiguousarray(bb.x).view(np.int16)).pin_memory(),
+        return {"x": torch.from_numpy(np.ascontiguousarray(bb.x).view(np.int16) if bf else bb.x).pin_memory(),
                 "sizes": torch.from_numpy(bb.sizes).pin_memory(),
                 "scores": torch.from_numpy(bb.scores).pin_memory(),
                 "offsets": torch.from_numpy(bb.offsets).pin_memory()}
@@ -236,9 +239,10 @@ def test_pipeline_overlapped_steps():
     want = []
     for i, w in enumerate((wa, wb)):
         db = solo.inp
-        db.x.view(torch.int16).copy_(hosts[i]["x"])
+        (db.x.view(torch.int16) if bf else db.x).copy_(hosts[i]["x"])
         db.sizes.copy_(hosts[i]["sizes"])
         db.scores.copy_(hosts[i]["scores"])
+        db.offsets.copy_(hosts[i]["offsets"])
         solo.run()
         want.append(_host_copy(hr.fetch()[0]))
         assert want[-1]["status"] == 0
@@ -261,7 +265,7 @@ def test_pipeline_overlapped_steps():
         assert g["batch"] == e["batch"] and g["status"] == 0, (k, i)
         for name in ("offsets", "ids", "sizes", "x"):
             np.testing.assert_array_equal(g[name], e[name], err_msg=f"step {k} input {i} {name}")
-        assert len(g["exits"]) == len(e["exits"]) == 4
+        assert len(g["exits"]) == len(e["exits"]) == sum(1 for s in wa.stages if s.exit)
         for (gm, gp), (em, ep) in zip(g["exits"], e["exits"]):
             np.testing.assert_array_equal(gm, em)
             np.testing.assert_array_equal(gp, ep)

@@ -382,6 +382,27 @@ int fusion_stage(int dtype, int flags, fusion_ragged in, const void *x, int32_t 
                  int32_t *a_match, void *workspace, size_t workspace_bytes, int32_t *dev_status,
                  void *stream);
 
+/*
+ * fusion_stage_mlp: fusion_stage with one of the paper's MLP exit heads (Sec. III-G: a
+ * SpatialPool head at block 8, a CLS-only head at block 10) in place of the linear head.
+ * The exit check is fusion_exit_check_mlp on the stage's INPUT rows: merging never
+ * changes CLS, and it keeps sum_t s_t x_t and sum_t s_t over the patch rows (a merged
+ * token of size s_B + sum s_A carries s_B x_B + sum s_A x_A, Sec. III-C), so the
+ * size-weighted pool of the input equals that of the merged tokens in exact arithmetic.
+ * Arguments as fusion_stage; head as fusion_exit_check_mlp (read only with
+ * FUSION_STAGE_EXIT); workspace: at least fusion_exit_mlp_workspace_size(in.max_batch,
+ * dim, head.hidden, head.classes) bytes with the exit check, else
+ * fusion_workspace_size(in.max_batch, 1), zero-filled before first use and left so.
+ * Errors: those of fusion_stage and fusion_exit_check_mlp.
+ */
+int fusion_stage_mlp(int dtype, int flags, fusion_ragged in, const void *x, int32_t dim,
+                     const void *keys, int32_t key_dim, const float *sizes, const float *scores,
+                     const int32_t *r, const float *rho, fusion_mlp_head head, uint8_t *exit_mask,
+                     float *logits, float *max_prob, void *x_out, float *sizes_out, float *scores_out,
+                     int32_t *offsets_out, int32_t *ids_out, int32_t *batch_out, int32_t *keep_idx,
+                     int32_t *a_match, void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                     void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -312,9 +312,13 @@ def stage(batch, spec) -> Dict[str, object]:
     Order (Sec. III-B): merge (if enabled) -> exit check on the merged tokens
     (if enabled; exited samples leave the batch) -> prune the survivors (if
     enabled).  Per-sample router outputs spec.r / spec.rho are indexed by the
-    samples' original ids.  Returns the output batch fields plus exit_mask,
-    logits, max_prob (indexed by input sample), keep_idx (input row of every
-    output row), a_match (input rows) and the decision margins."""
+    samples' original ids.  With spec.mlp_head (an MLP exit head, Sec. III-G) the
+    exit check reads the stage's input rows: merging keeps CLS and, over the patch
+    rows, sum s_t x_t and sum s_t (Sec. III-C), so the CLS-only and the size-weighted
+    pooled head inputs of the input equal those of the merged tokens in exact
+    arithmetic.  Returns the output batch fields plus exit_mask, logits, max_prob
+    (indexed by input sample), keep_idx (input row of every output row), a_match
+    (input rows) and the decision margins."""
     dtype = batch.dtype
     B = batch.batch
     ids = np.arange(B, dtype=np.int32) if batch.ids is None else np.asarray(batch.ids, np.int32)
@@ -334,10 +338,15 @@ def stage(batch, spec) -> Dict[str, object]:
     mask = np.zeros(B, np.uint8)
     res["exit_gap"] = np.full(B, np.inf)
     if spec.exit:
-        e = exit_check(dtype, offsets, x, spec.head)
-        mask = e["exit_mask"]
-        res.update(exit_mask=mask, logits=e["logits"], max_prob=e["max_prob"],
-                   exit_gap=e["exit_gap"], u=e["u"])
+        if getattr(spec, "mlp_head", None) is not None:
+            e = exit_mlp(dtype, batch.offsets, batch.x[:T], batch.sizes[:T], spec.mlp_head)
+            mask = e["exit_mask"]
+            res.update(exit_mask=mask, logits=e["logits"], max_prob=e["max_prob"], exit_gap=e["exit_gap"])
+        else:
+            e = exit_check(dtype, offsets, x, spec.head)
+            mask = e["exit_mask"]
+            res.update(exit_mask=mask, logits=e["logits"], max_prob=e["max_prob"],
+                       exit_gap=e["exit_gap"], u=e["u"])
         c = compact(dtype, offsets, x, sizes, scores, mask, ids)
         x, sizes, scores, offsets = c["x"], c["sizes"], c["scores"], c["offsets"]
         keep = keep[c["keep_idx"]]

@@ -45,7 +45,7 @@ FUSION_POOL_SPATIAL = 1
 EXPORTED = ("fusion_status_string", "fusion_version", "fusion_profile_next", "fusion_workspace_size",
             "fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune", "fusion_compact",
             "fusion_stage", "fusion_merge_router", "fusion_token_scores", "fusion_exit_mlp_workspace_size",
-            "fusion_exit_check_mlp", "fusion_attention")
+            "fusion_exit_check_mlp", "fusion_attention", "fusion_stage_mlp")
 
 
 class FusionError(RuntimeError):
@@ -113,9 +113,11 @@ def load(path: Optional[str] = None):
     lib.fusion_exit_mlp_workspace_size.restype = SZ
     lib.fusion_exit_check_mlp.argtypes = [ctypes.c_int, R, V, I32, V, fusion_mlp_head, V, V, V, V, SZ, V, V]
     lib.fusion_attention.argtypes = [ctypes.c_int, R, V, I32, I32, V, V, V, V]
+    lib.fusion_stage_mlp.argtypes = [ctypes.c_int, ctypes.c_int, R, V, I32, V, I32, V, V, V, V, fusion_mlp_head, V,
+                                     V, V, V, V, V, V, V, V, V, V, V, SZ, V, V]
     for name in ("fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune",
                  "fusion_compact", "fusion_stage", "fusion_merge_router", "fusion_token_scores",
-                 "fusion_exit_check_mlp", "fusion_attention"):
+                 "fusion_exit_check_mlp", "fusion_attention", "fusion_stage_mlp"):
         getattr(lib, name).restype = ctypes.c_int
     del I64, F
     if path is None:
@@ -276,3 +278,16 @@ def fusion_stage(dtype, flags, in_, x, dim, keys, key_dim, sizes, scores, r, rho
                                _ptr(offsets_out), _ptr(ids_out), _ptr(batch_out), _ptr(keep_idx),
                                _ptr(a_match), _ptr(workspace), int(workspace_bytes), _ptr(dev_status),
                                _stream(stream))
+
+
+def fusion_stage_mlp(dtype, flags, in_, x, dim, keys, key_dim, sizes, scores, r, rho, head, exit_mask, logits,
+                     max_prob, x_out, sizes_out, scores_out, offsets_out, ids_out, batch_out, keep_idx, a_match,
+                     workspace, workspace_bytes, dev_status, stream=None) -> int:
+    if head is None:
+        head = fusion_mlp_head()
+    return load().fusion_stage_mlp(int(dtype), int(flags), in_, _ptr(x), int(dim), _ptr(keys), int(key_dim),
+                                   _ptr(sizes), _ptr(scores), _ptr(r), _ptr(rho), head, _ptr(exit_mask),
+                                   _ptr(logits), _ptr(max_prob), _ptr(x_out), _ptr(sizes_out), _ptr(scores_out),
+                                   _ptr(offsets_out), _ptr(ids_out), _ptr(batch_out), _ptr(keep_idx),
+                                   _ptr(a_match), _ptr(workspace), int(workspace_bytes), _ptr(dev_status),
+                                   _stream(stream))

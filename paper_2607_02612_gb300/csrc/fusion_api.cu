@@ -377,33 +377,29 @@ MlpWs mlp_ws_layout(int32_t max_batch, int32_t dim, int32_t hidden, int32_t clas
 }
 }  // namespace
 
-size_t fusion_exit_mlp_workspace_size(int32_t max_batch, int32_t dim, int32_t hidden, int32_t classes) {
-    if (max_batch < 0) max_batch = 0;
-    return mlp_ws_layout(max_batch, dim < 16 ? 16 : dim, hidden < 16 ? 16 : hidden, classes < 1 ? 1 : classes).total;
-}
-
-int fusion_exit_check_mlp(int dtype, fusion_ragged in, const void *x, int32_t dim, const float *sizes,
-                          fusion_mlp_head head, uint8_t *exit_mask, float *logits, float *max_prob,
-                          void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream) {
-    FZ_TRY(check_dtype(dtype));
-    FZ_TRY(check_ragged(in));
-    FZ_TRY(check_dim(dim));
+namespace {
+int check_mlp_head(const fusion_mlp_head &head, const float *sizes) {
     FZ_TRY(check_dim(head.hidden));
     if (head.classes < 1) return FUSION_ERR_SHAPE;
     if (head.pool != FUSION_POOL_CLS && head.pool != FUSION_POOL_SPATIAL) return FUSION_ERR_INVALID_ARG;
     if (head.pool == FUSION_POOL_SPATIAL && !sizes) return FUSION_ERR_INVALID_ARG;
-    if (!x || !exit_mask || !aligned16(x)) return FUSION_ERR_INVALID_ARG;
     if (!head.ln_gamma || !head.ln_beta || !head.w1 || !head.b1 || !head.w2 || !head.b2) return FUSION_ERR_INVALID_ARG;
     if (!aligned16(head.ln_gamma) || !aligned16(head.ln_beta) || !aligned16(head.w1) || !aligned16(head.w2))
         return FUSION_ERR_INVALID_ARG;
+    return FUSION_OK;
+}
+
+// The MLP exit head's three launches (pool; LayerNorm, first layer and GELU; second layer,
+// softmax maximum and exit rule) on the rows of `in`, scratch from a checked workspace.
+// `mid` (may be NULL) is recorded between the first layer and the second.
+int launch_exit_mlp(int dtype, const fusion_ragged &in, const void *x, int32_t dim, const float *sizes,
+                    const fusion_mlp_head &head, uint8_t *exit_mask, float *logits, float *max_prob, void *workspace,
+                    int32_t *dev_status, cudaStream_t s, cudaEvent_t mid) {
     const MlpWs L = mlp_ws_layout(in.max_batch, dim, head.hidden, head.classes);
-    if (!workspace || !aligned16(workspace)) return FUSION_ERR_WORKSPACE;
-    if (workspace_bytes < L.total) return FUSION_ERR_WORKSPACE;
     unsigned char *wb = static_cast<unsigned char *>(workspace);
     float *u = reinterpret_cast<float *>(wb + L.u);
     void *hid = wb + L.hid;
     const Ws w = carve(workspace, in.max_batch, head.classes);
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
     const int n_btile = ceil_div(in.max_batch > 0 ? in.max_batch : 1, kExitBT);
 
     PoolParams pp{};
@@ -445,12 +441,34 @@ int fusion_exit_check_mlp(int dtype, fusion_ragged in, const void *x, int32_t di
     l2.in_mode = 1;
     l2.skip_ln = 1;
 
-    const ProfileEvents ev = take_profile();
-    record(ev.start, s);
     int rc = cuda_rc(launch_head_pool(dtype, pp, s));
     if (rc == FUSION_OK) rc = cuda_rc(launch_exit(dtype, l1, s));
-    record(ev.mid, s);
+    record(mid, s);
     if (rc == FUSION_OK) rc = cuda_rc(launch_exit(dtype, l2, s));
+    return rc;
+}
+}  // namespace
+
+size_t fusion_exit_mlp_workspace_size(int32_t max_batch, int32_t dim, int32_t hidden, int32_t classes) {
+    if (max_batch < 0) max_batch = 0;
+    return mlp_ws_layout(max_batch, dim < 16 ? 16 : dim, hidden < 16 ? 16 : hidden, classes < 1 ? 1 : classes).total;
+}
+
+int fusion_exit_check_mlp(int dtype, fusion_ragged in, const void *x, int32_t dim, const float *sizes,
+                          fusion_mlp_head head, uint8_t *exit_mask, float *logits, float *max_prob,
+                          void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream) {
+    FZ_TRY(check_dtype(dtype));
+    FZ_TRY(check_ragged(in));
+    FZ_TRY(check_dim(dim));
+    FZ_TRY(check_mlp_head(head, sizes));
+    if (!x || !exit_mask || !aligned16(x)) return FUSION_ERR_INVALID_ARG;
+    if (!workspace || !aligned16(workspace)) return FUSION_ERR_WORKSPACE;
+    if (workspace_bytes < mlp_ws_layout(in.max_batch, dim, head.hidden, head.classes).total) return FUSION_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const ProfileEvents ev = take_profile();
+    record(ev.start, s);
+    const int rc = launch_exit_mlp(dtype, in, x, dim, sizes, head, exit_mask, logits, max_prob, workspace, dev_status,
+                                   s, ev.mid);
     record(ev.end, s);
     return rc;
 }
@@ -503,13 +521,18 @@ int fusion_token_scores(int dtype, fusion_ragged in, const void *x, int32_t dim,
     return rc;
 }
 
-int fusion_stage(int dtype, int flags, fusion_ragged in, const void *x, int32_t dim,
-                 const void *keys, int32_t key_dim, const float *sizes, const float *scores,
-                 const int32_t *r, const float *rho, fusion_exit_head head, uint8_t *exit_mask,
-                 float *logits, float *max_prob, void *x_out, float *sizes_out, float *scores_out,
-                 int32_t *offsets_out, int32_t *ids_out, int32_t *batch_out, int32_t *keep_idx,
-                 int32_t *a_match, void *workspace, size_t workspace_bytes, int32_t *dev_status,
-                 void *stream) {
+}  // extern "C"
+
+namespace {
+// The fused stage with either exit head: `lin` (the linear head, one exit kernel that may run
+// the plan) or `mlp` (the MLP head's three launches on the stage's input rows, then the plan
+// kernel when the per-sample kernel does not fuse it).
+int stage_impl(int dtype, int flags, const fusion_ragged &in, const void *x, int32_t dim, const void *keys,
+               int32_t key_dim, const float *sizes, const float *scores, const int32_t *r, const float *rho,
+               const fusion_exit_head *lin, const fusion_mlp_head *mlp, uint8_t *exit_mask, float *logits,
+               float *max_prob, void *x_out, float *sizes_out, float *scores_out, int32_t *offsets_out,
+               int32_t *ids_out, int32_t *batch_out, int32_t *keep_idx, int32_t *a_match, void *workspace,
+               size_t workspace_bytes, int32_t *dev_status, void *stream) {
     FZ_TRY(check_dtype(dtype));
     if (flags < 0 || flags > (FUSION_STAGE_MERGE | FUSION_STAGE_EXIT | FUSION_STAGE_PRUNE))
         return FUSION_ERR_INVALID_ARG;
@@ -528,12 +551,18 @@ int fusion_stage(int dtype, int flags, fusion_ragged in, const void *x, int32_t 
     }
     if (do_prune && (!rho || !scores)) return FUSION_ERR_INVALID_ARG;
     if (!do_merge && a_match) return FUSION_ERR_INVALID_ARG;
-    const int classes = do_exit ? head.classes : 1;
+    const int classes = do_exit ? (mlp ? mlp->classes : lin->classes) : 1;
     if (do_exit) {
-        FZ_TRY(check_head(head));
+        FZ_TRY(mlp ? check_mlp_head(*mlp, sizes) : check_head(*lin));
         if (!exit_mask) return FUSION_ERR_INVALID_ARG;
     }
-    FZ_TRY(check_workspace(workspace, workspace_bytes, in.max_batch, classes));
+    if (do_exit && mlp) {   // the MLP head's scratch, whose first part is the stage's own
+        if (!workspace || !aligned16(workspace)) return FUSION_ERR_WORKSPACE;
+        if (workspace_bytes < mlp_ws_layout(in.max_batch, dim, mlp->hidden, mlp->classes).total)
+            return FUSION_ERR_WORKSPACE;
+    } else {
+        FZ_TRY(check_workspace(workspace, workspace_bytes, in.max_batch, classes));
+    }
     const ImageGeometry G = image_geometry(dtype, in.max_tokens, do_merge ? key_dim : dim, do_merge);
     if (!G.ok) return FUSION_ERR_SHAPE;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -554,7 +583,12 @@ int fusion_stage(int dtype, int flags, fusion_ragged in, const void *x, int32_t 
     pa.slot = w.slot;
     pa.plan = w.plan;
     pa.status = dev_status;
-    if (do_exit) {
+    if (do_exit && mlp) {
+        FZ_TRY(launch_exit_mlp(dtype, in, x, dim, sizes, *mlp, exit_mask, logits, max_prob, workspace, dev_status, s,
+                               nullptr));
+        if (!fuse_plan(in)) FZ_TRY(cuda_rc(launch_plan(pa, s)));
+    } else if (do_exit) {
+        const fusion_exit_head &head = *lin;
         ExitParams e{};
         e.in = dev(in);
         e.x = x;
@@ -583,6 +617,33 @@ int fusion_stage(int dtype, int flags, fusion_ragged in, const void *x, int32_t 
     const int rc = cuda_rc(launch_sample_kernel(dtype, p, G, s));
     record(ev.end, s);
     return rc;
+}
+}  // namespace
+
+extern "C" {
+
+int fusion_stage(int dtype, int flags, fusion_ragged in, const void *x, int32_t dim,
+                 const void *keys, int32_t key_dim, const float *sizes, const float *scores,
+                 const int32_t *r, const float *rho, fusion_exit_head head, uint8_t *exit_mask,
+                 float *logits, float *max_prob, void *x_out, float *sizes_out, float *scores_out,
+                 int32_t *offsets_out, int32_t *ids_out, int32_t *batch_out, int32_t *keep_idx,
+                 int32_t *a_match, void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                 void *stream) {
+    return stage_impl(dtype, flags, in, x, dim, keys, key_dim, sizes, scores, r, rho, &head, nullptr, exit_mask, logits,
+                      max_prob, x_out, sizes_out, scores_out, offsets_out, ids_out, batch_out, keep_idx, a_match,
+                      workspace, workspace_bytes, dev_status, stream);
+}
+
+int fusion_stage_mlp(int dtype, int flags, fusion_ragged in, const void *x, int32_t dim,
+                     const void *keys, int32_t key_dim, const float *sizes, const float *scores,
+                     const int32_t *r, const float *rho, fusion_mlp_head head, uint8_t *exit_mask,
+                     float *logits, float *max_prob, void *x_out, float *sizes_out, float *scores_out,
+                     int32_t *offsets_out, int32_t *ids_out, int32_t *batch_out, int32_t *keep_idx,
+                     int32_t *a_match, void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                     void *stream) {
+    return stage_impl(dtype, flags, in, x, dim, keys, key_dim, sizes, scores, r, rho, nullptr, &head, exit_mask, logits,
+                      max_prob, x_out, sizes_out, scores_out, offsets_out, ids_out, batch_out, keep_idx, a_match,
+                      workspace, workspace_bytes, dev_status, stream);
 }
 
 }  // extern "C"

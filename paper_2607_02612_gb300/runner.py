@@ -182,13 +182,18 @@ class Fusion:
         o = dict(exit_mask=torch.zeros(b.max_batch, dtype=torch.uint8, device=dev),
                  logits=torch.zeros((b.max_batch, head.classes), dtype=torch.float32, device=dev),
                  max_prob=torch.zeros(b.max_batch, dtype=torch.float32, device=dev))
+        ws, nbytes = self.mlp_workspace(b, head)
+        fb.check(fb.fusion_exit_check_mlp(DTYPE_CODE[b.dtype], b.ragged(), b.x, b.dim, b.sizes, head.c_struct(),
+                                          o["exit_mask"], o["logits"], o["max_prob"], ws, nbytes, self.status))
+        return o
+
+    def mlp_workspace(self, b: DeviceBatch, head: "MlpHeadTensors"):
+        """The zero-filled scratch of the MLP-head calls (it grows to the largest head seen;
+        a Chain sizes it for all its stages before any graph capture)."""
         nbytes = fb.fusion_exit_mlp_workspace_size(b.max_batch, b.dim, head.hidden, head.classes)
         if self._mlp_ws is None or self._mlp_ws.numel() < nbytes:
-            self._mlp_ws = torch.zeros(nbytes, dtype=torch.uint8, device=dev)
-        fb.check(fb.fusion_exit_check_mlp(DTYPE_CODE[b.dtype], b.ragged(), b.x, b.dim, b.sizes, head.c_struct(),
-                                          o["exit_mask"], o["logits"], o["max_prob"], self._mlp_ws, nbytes,
-                                          self.status))
-        return o
+            self._mlp_ws = torch.zeros(nbytes, dtype=torch.uint8, device=self.device)
+        return self._mlp_ws, nbytes
 
     def attention(self, b: DeviceBatch, qkv: torch.Tensor, heads: int, sizes: Optional[torch.Tensor] = None,
                   out: Optional[torch.Tensor] = None) -> torch.Tensor:
@@ -227,8 +232,17 @@ class Fusion:
         return o
 
     def stage(self, b: DeviceBatch, flags: int, r=None, rho=None, head: Optional[HeadTensors] = None,
-              a_match: bool = False, out: Optional[Dict[str, torch.Tensor]] = None) -> Dict[str, torch.Tensor]:
-        o = out if out is not None else self.stage_outputs(b, flags, head, a_match)
+              a_match: bool = False, out: Optional[Dict[str, torch.Tensor]] = None,
+              mlp_head: Optional["MlpHeadTensors"] = None) -> Dict[str, torch.Tensor]:
+        """One fused stage; the exit check uses `head` (linear) or `mlp_head` (an MLP exit head)."""
+        o = out if out is not None else self.stage_outputs(b, flags, head, a_match, mlp_head=mlp_head)
+        if mlp_head is not None:
+            ws, nbytes = self.mlp_workspace(b, mlp_head)
+            fb.check(fb.fusion_stage_mlp(
+                DTYPE_CODE[b.dtype], flags, b.ragged(), b.x, b.dim, b.keys, b.key_dim, b.sizes, b.scores, r, rho,
+                mlp_head.c_struct(), o["exit_mask"], o["logits"], o["max_prob"], o["x"], o["sizes"], o["scores"],
+                o["offsets"], o["ids"], o["batch"], o["keep_idx"], o.get("a_match"), ws, nbytes, self.status))
+            return o
         fb.check(fb.fusion_stage(
             DTYPE_CODE[b.dtype], flags, b.ragged(), b.x, b.dim, b.keys, b.key_dim, b.sizes, b.scores, r, rho,
             head.c_struct() if head is not None else None, o["exit_mask"], o["logits"], o["max_prob"], o["x"],
@@ -236,15 +250,16 @@ class Fusion:
             self.workspace, self.ws_bytes, self.status))
         return o
 
-    def stage_outputs(self, b: DeviceBatch, flags: int, head: Optional[HeadTensors], a_match: bool = False):
+    def stage_outputs(self, b: DeviceBatch, flags: int, head: Optional[HeadTensors], a_match: bool = False,
+                      mlp_head: Optional["MlpHeadTensors"] = None):
         dev = self.device
         o = self._outputs(b, b.scores is not None)
         o["ids"] = torch.zeros(b.max_batch, dtype=torch.int32, device=dev)
         o["batch"] = torch.zeros(1, dtype=torch.int32, device=dev)
         has_exit = bool(flags & fb.FUSION_STAGE_EXIT)
         o["exit_mask"] = torch.zeros(b.max_batch, dtype=torch.uint8, device=dev) if has_exit else None
-        o["logits"] = (torch.zeros((b.max_batch, head.classes), dtype=torch.float32, device=dev)
-                       if has_exit else None)
+        classes = (mlp_head or head).classes if has_exit else 0
+        o["logits"] = torch.zeros((b.max_batch, classes), dtype=torch.float32, device=dev) if has_exit else None
         o["max_prob"] = torch.zeros(b.max_batch, dtype=torch.float32, device=dev) if has_exit else None
         o["a_match"] = torch.full((b.max_rows,), -1, dtype=torch.int32, device=dev) if a_match else None
         return o
@@ -263,6 +278,7 @@ class ChainStage:
     r: Optional[torch.Tensor] = None
     rho: Optional[torch.Tensor] = None
     head: Optional[HeadTensors] = None
+    mlp_head: Optional[MlpHeadTensors] = None   # an MLP exit head in place of `head`
 
 
 @dataclass
@@ -278,13 +294,23 @@ class Chain:
     def __post_init__(self):
         b = self.inp
         for st in self.stages:
-            o = self.fusion.stage_outputs(b, st.flags, st.head)
+            o = self.fusion.stage_outputs(b, st.flags, st.head, mlp_head=st.mlp_head)
+            if st.mlp_head is not None:
+                self.fusion.mlp_workspace(b, st.mlp_head)   # sized before any capture
             self.outs.append(o)
             self.batches.append(b)
             b = output_batch(b, o)
 
     def run_stage(self, s: int, stream=None):
         st, b, o = self.stages[s], self.batches[s], self.outs[s]
+        if st.mlp_head is not None:
+            ws, nbytes = self.fusion.mlp_workspace(b, st.mlp_head)
+            fb.check(fb.fusion_stage_mlp(
+                DTYPE_CODE[b.dtype], st.flags, b.ragged(), b.x, b.dim, b.keys, b.key_dim, b.sizes, b.scores, st.r,
+                st.rho, st.mlp_head.c_struct(), o["exit_mask"], o["logits"], o["max_prob"], o["x"], o["sizes"],
+                o["scores"], o["offsets"], o["ids"], o["batch"], o["keep_idx"], None, ws, nbytes, self.fusion.status,
+                stream))
+            return
         fb.check(fb.fusion_stage(
             DTYPE_CODE[b.dtype], st.flags, b.ragged(), b.x, b.dim, b.keys, b.key_dim, b.sizes, b.scores, st.r,
             st.rho, st.head.c_struct() if st.head is not None else None, o["exit_mask"], o["logits"],

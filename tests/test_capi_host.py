@@ -215,6 +215,48 @@ def test_exit_check_mlp_rejects_bad_arguments(lib):
     assert call(workspace_bytes=ws - 1) == fz.FUSION_ERR_WORKSPACE
 
 
+def _mlp_head(**kw):
+    h = dict(pool=fz.FUSION_POOL_SPATIAL, gamma=FAKE, beta=FAKE, eps=1e-6, w1=FAKE, b1=FAKE, hidden=768,
+             w2=FAKE, b2=FAKE, classes=1000, tau=0.5)
+    h.update(kw)
+    return fz.mlp_head(*h.values())
+
+
+def _stage_mlp(**kw):
+    args = dict(dtype=fz.FUSION_BF16, flags=7, in_=_r(), x=FAKE, dim=384, keys=FAKE, key_dim=384, sizes=FAKE,
+                scores=FAKE, r=FAKE, rho=FAKE, head=_mlp_head(), exit_mask=FAKE, logits=FAKE, max_prob=FAKE,
+                x_out=FAKE, sizes_out=FAKE, scores_out=FAKE, offsets_out=FAKE, ids_out=FAKE, batch_out=FAKE,
+                keep_idx=None, a_match=None, workspace=FAKE,
+                workspace_bytes=fz.fusion_exit_mlp_workspace_size(4, 384, 768, 1000), dev_status=FAKE, stream=0)
+    args.update(kw)
+    return fz.fusion_stage_mlp(*args.values())
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(dtype=4), fz.FUSION_ERR_DTYPE),
+    (dict(flags=8), fz.FUSION_ERR_INVALID_ARG),
+    (dict(head=_mlp_head(hidden=100)), fz.FUSION_ERR_SHAPE),
+    (dict(head=_mlp_head(classes=0)), fz.FUSION_ERR_SHAPE),
+    (dict(head=_mlp_head(pool=2)), fz.FUSION_ERR_INVALID_ARG),
+    (dict(head=_mlp_head(w1=None)), fz.FUSION_ERR_INVALID_ARG),
+    (dict(head=_mlp_head(w2=FAKE + 4)), fz.FUSION_ERR_INVALID_ARG),
+    (dict(exit_mask=None), fz.FUSION_ERR_INVALID_ARG),
+    (dict(sizes=None), fz.FUSION_ERR_INVALID_ARG),
+    (dict(rho=None), fz.FUSION_ERR_INVALID_ARG),
+    (dict(flags=6, a_match=FAKE), fz.FUSION_ERR_INVALID_ARG),
+    (dict(workspace=None), fz.FUSION_ERR_WORKSPACE),
+    (dict(workspace=FAKE + 8), fz.FUSION_ERR_WORKSPACE),
+    # the linear head's scratch is too small for the MLP head's
+    (dict(workspace_bytes=fz.fusion_workspace_size(4, 1000)), fz.FUSION_ERR_WORKSPACE),
+    (dict(workspace_bytes=fz.fusion_exit_mlp_workspace_size(4, 384, 768, 1000) - 1), fz.FUSION_ERR_WORKSPACE),
+    # without the exit check the stage's own scratch is enough, and a bad head is not read
+    (dict(flags=5, head=_mlp_head(pool=2), workspace_bytes=fz.fusion_workspace_size(4, 1) - 1),
+     fz.FUSION_ERR_WORKSPACE),
+])
+def test_stage_mlp_rejects_bad_arguments(lib, kw, code):
+    assert _stage_mlp(**kw) == code
+
+
 def test_attention_rejects_bad_arguments(lib):
     def call(**kw):
         args = dict(dtype=fz.FUSION_BF16, in_=_r(max_tokens=197), qkv=FAKE, heads=6, head_dim=64, sizes=None,

@@ -272,6 +272,67 @@ def test_pipeline_overlapped_steps(name, B):
     assert want[0]["batch"] != want[1]["batch"] or not np.array_equal(want[0]["ids"], want[1]["ids"])
 
 
+def _mlp_heads_at(w, placement, seed):
+    """Put MLP exit heads on the given exit stages ({stage index: pool}) and set each tau in
+    the widest gap of the oracle's max_prob values around the median at that stage's input,
+    so that about half its images exit and none sits at the threshold.  Returns the oracle's
+    chain."""
+    from workloads import make_mlp_head
+    b = w.batch
+    rng = np.random.default_rng(seed)
+    outs = []
+    bb = b
+    for si, spec in enumerate(w.stages):
+        if si in placement:
+            head = make_mlp_head(rng, placement[si], b.dim, 2 * b.dim, 1000, b.dtype)
+            T = int(bb.offsets[-1])
+            mp = np.sort(oracle.exit_mlp(b.dtype, bb.offsets, bb.x[:T], bb.sizes[:T], head)["max_prob"])
+            lo = max(0, len(mp) // 2 - 5)
+            k = lo + int(np.argmax(np.diff(mp[lo:lo + 11])))
+            head.tau = float(np.float32(0.5 * (mp[k] + mp[k + 1])))
+            spec.mlp_head = head
+            spec.head = None
+        res = oracle.stage(bb, spec)
+        outs.append(res)
+        bb = oracle.next_batch(bb, res)
+    return outs
+
+
+@pytest.mark.parametrize("graph", [True, False])
+def test_chain_with_mlp_heads(graph):
+    """The DeiT-S schedule with the paper's MLP exit heads inside the fused stage: SpatialPool
+    at block 8, CLS-only at block 10 (the linear head at blocks 4 and 6); every stage against
+    the oracle, whose MLP exit check reads the stage input as the fused stage does."""
+    from workloads import POOL_CLS, POOL_SPATIAL
+    w = make_workload("deit_s_chain12_bf16_b256", batch=64)
+    o_outs = _mlp_heads_at(w, {7: POOL_SPATIAL, 9: POOL_CLS}, 21)
+    g_outs, status = P.chain_on_gpu(w, graph=graph)
+    assert status == 0
+    rep = P.Report()
+    P.compare_chain(rep, w, g_outs, o_outs)
+    assert rep.compared_samples > 0
+    for si in (7, 9):
+        n = int(o_outs[si]["exit_mask"].sum())
+        assert 0 < n < len(o_outs[si]["exit_mask"]), (si, n)
+    _report(rep, f"chain with MLP heads, graph={graph}")
+
+
+@pytest.mark.parametrize("pool", [0, 1])
+def test_stage_mlp_f32(pool):
+    """One fused float32 stage (merge, MLP exit check, prune) on the 65-token schedule."""
+    w = make_workload("ragged_b8192_n65_chain4_f32", batch=300, seed_offset=3)
+    w = type(w)(w.spec, w.batch, w.stages[:1])
+    w.stages[0].prune = True
+    w.stages[0].rho = np.full(w.batch.batch, 0.7, np.float32)
+    o_outs = _mlp_heads_at(w, {0: pool}, 31 + pool)
+    g_outs, status = P.chain_on_gpu(w)
+    assert status == 0
+    rep = P.Report()
+    P.compare_chain(rep, w, g_outs, o_outs)
+    assert rep.compared_samples > 0
+    _report(rep, f"f32 MLP stage pool {pool}")
+
+
 def _subset(batch: Batch, idx: np.ndarray) -> Batch:
     """The images idx of a batch, repacked (ids keep the original image numbers)."""
     counts = np.diff(batch.offsets)[idx]

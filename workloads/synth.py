@@ -126,6 +126,7 @@ class StageSpec:
     r: Optional[np.ndarray] = None     # [B_orig] int32, indexed by original image id
     rho: Optional[np.ndarray] = None   # [B_orig] f32, indexed by original image id
     head: Optional[Head] = None
+    mlp_head: Optional["MlpHead"] = None   # an MLP exit head in place of `head`
 
 
 @dataclass

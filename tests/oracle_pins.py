@@ -785,7 +785,38 @@ def pin_attention_closed_forms():
                                   oracle.attention("f32", np.array([0, 4], np.int32), x, H, np.ones(4, np.float32)))
 
 
+def pin_spatial_pool_merge_invariant():
+    """The reading behind the MLP exit check of a fused stage (Sec. III-C, III-G): merging keeps
+    sum s_t x_t and sum s_t over the patch rows, so the SpatialPool of a sample's input equals
+    that of its merged tokens, up to the rounding of the merged means (float32 here: a relative
+    2^-24 per merged element), and the CLS row is unchanged.  Also an oracle stage with an MLP
+    head takes its exit decision from the input rows (same mask as exit_mlp on the input)."""
+    from workloads import make_mlp_head, make_workload
+    w = make_workload("deit_s_stage_f32_b8")
+    b, spec = w.batch, w.stages[0]
+    T = int(b.offsets[-1])
+    m = oracle.merge(b.dtype, b.offsets, b.x[:T], b.keys[:T], b.sizes[:T], b.scores[:T], spec.r)
+    assert int(m["offsets"][-1]) < T   # tokens were merged
+    head = make_mlp_head(np.random.default_rng(5), POOL_SPATIAL, b.dim, 2 * b.dim, 10, b.dtype)
+    pin_ = oracle.exit_mlp(b.dtype, b.offsets, b.x[:T], b.sizes[:T], head)["pool"]
+    pm = oracle.exit_mlp(b.dtype, m["offsets"], m["x"], m["sizes"], head)["pool"]
+    scale = np.abs(b.x[:T]).max()
+    assert np.abs(pin_ - pm).max() <= 4 * 2.0 ** -24 * scale, np.abs(pin_ - pm).max() / scale
+    for i in range(b.batch):   # CLS rows untouched
+        np.testing.assert_array_equal(m["x"][m["offsets"][i]], b.x[b.offsets[i]])
+    ch = make_mlp_head(np.random.default_rng(6), POOL_CLS, b.dim, 2 * b.dim, 10, b.dtype)
+    np.testing.assert_array_equal(oracle.exit_mlp(b.dtype, b.offsets, b.x[:T], b.sizes[:T], ch)["pool"],
+                                  oracle.exit_mlp(b.dtype, m["offsets"], m["x"], m["sizes"], ch)["pool"])
+    import dataclasses
+    e_in = oracle.exit_mlp(b.dtype, b.offsets, b.x[:T], b.sizes[:T], head)
+    head.tau = float(np.float32(np.median(e_in["max_prob"])))
+    res = oracle.stage(b, dataclasses.replace(spec, head=None, mlp_head=head, exit=True))
+    np.testing.assert_array_equal(res["exit_mask"],
+                                  oracle.exit_mlp(b.dtype, b.offsets, b.x[:T], b.sizes[:T], head)["exit_mask"])
+
+
 ALL_PINS = [
+    pin_spatial_pool_merge_invariant,
     pin_bf16_rounding_table,
     pin_bf16_rounding_vs_torch,
     pin_merge_worked_examples,

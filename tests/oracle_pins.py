@@ -816,7 +816,6 @@ def pin_spatial_pool_merge_invariant():
 
 
 ALL_PINS = [
-    pin_spatial_pool_merge_invariant,
     pin_bf16_rounding_table,
     pin_bf16_rounding_vs_torch,
     pin_merge_worked_examples,
@@ -842,4 +841,5 @@ ALL_PINS = [
     pin_exit_mlp_special_cases,
     pin_attention_vs_torch,
     pin_attention_closed_forms,
+    pin_spatial_pool_merge_invariant,
 ]

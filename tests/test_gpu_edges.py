@@ -321,6 +321,48 @@ def test_malformed_inputs_with_exit_check_write_nothing():
     assert torch.all(o["keep_idx"] == -5) and torch.all(o["x"] == 7)
 
 
+def _stage_raw_mlp(db, offsets=None, batch=None, ids=None):
+    """bf16 merge + MLP exit (SpatialPool) + prune through fusion_stage_mlp, malformed inputs."""
+    from workloads import POOL_SPATIAL, make_mlp_head
+    head = runner.mlp_head_tensors(make_mlp_head(np.random.default_rng(4), POOL_SPATIAL, db.dim, 2 * db.dim, 10,
+                                                 "bf16", tau=0.5), "bf16")
+    f = runner.Fusion(db.max_batch, 10)
+    o = f.stage_outputs(db, 7, None, mlp_head=head)
+    o["x"].fill_(7)
+    o["keep_idx"].fill_(-5)
+    ws, nbytes = f.mlp_workspace(db, head)
+    rr = torch.full((db.max_batch,), 2, dtype=torch.int32, device="cuda")
+    rho = torch.full((db.max_batch,), 0.5, dtype=torch.float32, device="cuda")
+    rg = fz.ragged(db.max_batch, db.max_tokens, db.max_rows, offsets if offsets is not None else db.offsets,
+                   batch, ids)
+    fz.check(fz.fusion_stage_mlp(fz.FUSION_BF16, 7, rg, db.x, db.dim, db.keys, db.key_dim, db.sizes, db.scores, rr,
+                                 rho, head.c_struct(), o["exit_mask"], o["logits"], o["max_prob"], o["x"],
+                                 o["sizes"], o["scores"], o["offsets"], o["ids"], o["batch"], o["keep_idx"], None,
+                                 ws, nbytes, f.status))
+    torch.cuda.synchronize()
+    return int(f.status.item()), o
+
+
+def test_malformed_inputs_with_mlp_exit_write_nothing():
+    """The fused stage with an MLP exit head on malformed offsets, device batch count and ids:
+    the status bit is raised and no token row or keep index is written."""
+    b = make_batch([20, 20, 20], 64, "bf16", seed=11, sizes="u1to4")
+    db = P.device_batch(b)
+    st, o = _stage_raw_mlp(db)
+    assert st == 0
+    for bad in ([0, 20, 10, 60], [0, 20, 40, 99], [-3, 20, 40, 60], [0, 0, 40, 60]):
+        st, o = _stage_raw_mlp(db, offsets=torch.tensor(bad, dtype=torch.int32, device="cuda"))
+        assert st & fz.FUSION_DEV_BAD_OFFSETS, bad
+        assert torch.all(o["keep_idx"] == -5) and torch.all(o["x"] == 7), bad
+        assert int(o["batch"][0]) == 0 and int(o["offsets"][0]) == 0, bad
+    st, o = _stage_raw_mlp(db, batch=torch.full((1,), 4, dtype=torch.int32, device="cuda"))
+    assert st & fz.FUSION_DEV_BAD_BATCH
+    assert torch.all(o["keep_idx"] == -5) and torch.all(o["x"] == 7)
+    st, o = _stage_raw_mlp(db, ids=torch.tensor([0, 9, 1], dtype=torch.int32, device="cuda"))
+    assert st & fz.FUSION_DEV_BAD_IDS
+    assert torch.all(o["keep_idx"] == -5) and torch.all(o["x"] == 7)
+
+
 def test_nonfinite_keys_raise_status():
     b = make_batch([9, 9], 16, "f32", seed=10, keys="separate")
     db = P.device_batch(b)

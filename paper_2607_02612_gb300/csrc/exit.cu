@@ -241,6 +241,9 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
     if (active) {
         issue_w_chunk<T>(p, w_region, c0, 0, dim, C, tid);
         if (n_k > 1) issue_w_chunk<T>(p, w_region + S::w_stage, c0, KC, dim, C, tid);
+        // launched as a programmatic dependent of the kernel before it (the MLP head's layers):
+        // the weights above are this call's own input; the rows below may be that kernel's output
+        asm volatile("griddepcontrol.wait;" ::: "memory");
         for (int it = tid; it < 16 * nchunk; it += kExitThreads) {
             const int sl = it / nchunk, c = it - sl * nchunk;
             const int s = s0 + sl;
@@ -894,6 +897,30 @@ cudaError_t launch_exit(int dtype, const ExitParams &p, cudaStream_t s) {
         k_exit<float><<<grid, kExitThreads, smem, s>>>(p);
     }
     return cudaGetLastError();
+}
+
+// The general kernel as a programmatic dependent launch: its CTAs may start as the previous
+// kernel on the stream finishes and wait for its results after issuing their weight loads.
+cudaError_t launch_exit_pdl(int dtype, const ExitParams &p, cudaStream_t s) {
+    const size_t smem = exit_smem_bytes(dtype, p.dim);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(p.n_ctile, p.n_btile);
+    cfg.blockDim = dim3(kExitThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (dtype == FUSION_BF16) {
+        cudaError_t e = cudaFuncSetAttribute(k_exit<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        return cudaLaunchKernelEx(&cfg, k_exit<__nv_bfloat16>, p);
+    }
+    cudaError_t e = cudaFuncSetAttribute(k_exit<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    return cudaLaunchKernelEx(&cfg, k_exit<float>, p);
 }
 
 namespace {

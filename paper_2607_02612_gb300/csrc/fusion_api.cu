@@ -7,6 +7,11 @@
 
 #include "launch.h"
 
+namespace fz {
+// The general exit kernel as a programmatic dependent launch (exit.cu), for the MLP head's layers.
+cudaError_t launch_exit_pdl(int dtype, const ExitParams &p, cudaStream_t s);
+}  // namespace fz
+
 using namespace fz;
 
 namespace {
@@ -441,10 +446,11 @@ int launch_exit_mlp(int dtype, const fusion_ragged &in, const void *x, int32_t d
     l2.in_mode = 1;
     l2.skip_ln = 1;
 
+    // each layer a programmatic dependent of the kernel before it (exit.cu)
     int rc = cuda_rc(launch_head_pool(dtype, pp, s));
-    if (rc == FUSION_OK) rc = cuda_rc(launch_exit(dtype, l1, s));
+    if (rc == FUSION_OK) rc = cuda_rc(launch_exit_pdl(dtype, l1, s));
     record(mid, s);
-    if (rc == FUSION_OK) rc = cuda_rc(launch_exit(dtype, l2, s));
+    if (rc == FUSION_OK) rc = cuda_rc(launch_exit_pdl(dtype, l2, s));
     return rc;
 }
 }  // namespace

@@ -18,7 +18,11 @@ roofline  the per-sample kernel (merge + prune + gather), which moves almost all
           bandwidth.
 e2e       the same metric through the public C ABI with host buffers: pinned
           host -> device copy of the step's inputs, the chain, device -> host read
-          of the results, all inside the timed region.
+          of the results, all inside the timed region, through runner.Pipeline (two
+          buffer slots, each step's input copy overlapping the previous step's kernels).
+side legs the merge router, the pruning router's scores, the MLP exit head, the
+          size-aware attention, one full stage alone, and the schedule with the paper's
+          MLP exit heads at blocks 8 and 10 (paper_heads).
 
 --impl reference times the CPU oracle (the only other implementation of the
 method here) on the host cores, on a bounded sample of the same workload.

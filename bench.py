@@ -183,17 +183,22 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 # algorithmic bytes (compulsory traffic) of one stage, from its inputs and outputs
 # ---------------------------------------------------------------------------
-def stage_bytes(spec, dtype, dim, in_off, in_ids, out_off, out_ids, classes):
+def stage_bytes(spec, dtype, dim, in_off, in_ids, out_off, out_ids, classes, row_ids=False):
+    """Algorithmic bytes (first kernel, per-sample kernel) of one stage.  Logits are counted for
+    the samples that exit only (the call writes no other row); the input row id of every output
+    row only when the caller asked for it (row_ids)."""
     eb = 2 if dtype == "bf16" else 4
     B_in = len(in_off) - 1
     B_out = len(out_off) - 1
     counts_in = np.diff(in_off).astype(np.int64)
     counts_out = np.diff(out_off).astype(np.int64)
     surv = {int(t): j for j, t in enumerate(out_ids)}
+    per_out = 8 + (4 if row_ids else 0)                                              # size, score (+ row id)
     first = 0
     if spec.exit:
+        n_exit = B_in - B_out                                                        # every sample that leaves exited
         first += B_in * dim * eb + classes * dim * eb + classes * 4 + 2 * dim * eb   # CLS rows, W, b, gamma/beta
-        first += B_in * (classes * 4 + 1 + 4)                                        # logits, mask, max-prob
+        first += n_exit * classes * 4 + B_in * (1 + 4)                               # exited logits, mask, max-prob
     first += (B_in + 1) * 4 + B_in * 8 + B_out * 12 + 4                              # offsets, r/rho, plan outputs
     image = 0
     for i in range(B_in):
@@ -205,7 +210,7 @@ def stage_bytes(spec, dtype, dim, in_off, in_ids, out_off, out_ids, classes):
         r_eff = min(max(int(spec.r[t]), 0), (n_in - 1) // 2) if spec.merge else 0
         rows_read = n_in if r_eff > 0 else n_out     # all keys (= tokens) are needed to decide a merge
         image += rows_read * dim * eb + n_in * 8 + 16                                # tokens, sizes+scores, scalars
-        image += n_out * (dim * eb + 12)                                            # tokens, size, score, row id
+        image += n_out * (dim * eb + per_out)                                       # tokens, size, score (, row id)
     return first, image
 
 
@@ -514,6 +519,7 @@ def run_solo_full_stage(args, fz, runner, w, b, dev, flush, peak):
     fus = runner.Fusion(b.batch, spec.head.classes, dev)
     db = runner.device_batch(b.dtype, b.offsets, b.x, b.keys, b.sizes, b.scores, device=dev)
     ch = runner.Chain(fus, db, [runner.ChainStage(flags, r, rho, head)])
+    ch.outs[0]["keep_idx"] = None   # as in the schedule: the next block needs no row ids
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
     for e in ev:
         e.record()

@@ -203,8 +203,9 @@ int fusion_merge(int dtype, fusion_ragged in, const void *x, int32_t dim, const 
  * variance (rounded to bf16 when dtype is FUSION_BF16); logits l = W u + b;
  * c = max_k softmax(l)_k; exit iff c >= tau.
  * Outputs: exit_mask [max_batch] uint8 (1 = exits), logits [max_batch, classes]
- * float32 (every sample's row is written; may be NULL), max_prob [max_batch]
- * float32 (may be NULL).  Entries beyond the actual count are untouched.
+ * float32 (the early prediction: only the rows of samples that exit are written,
+ * the other rows are untouched; may be NULL), max_prob [max_batch] float32 (may be
+ * NULL).  Entries beyond the actual count are untouched.
  */
 int fusion_exit_check(int dtype, fusion_ragged in, const void *x, int32_t dim,
                       fusion_exit_head head, uint8_t *exit_mask, float *logits, float *max_prob,
@@ -248,8 +249,9 @@ int fusion_exit_check_mlp(int dtype, fusion_ragged in, const void *x, int32_t di
  * inside the library, present on every GPU that loads the library until the
  * process exits.  A batch bound and class count whose scratch exceeds 1 MiB (see
  * fusion_workspace_size) is rejected with FUSION_ERR_WORKSPACE before anything is
- * enqueued.  The first call on a device looks up the array's device address, so
- * make that first call before any stream capture.  Calls allocate nothing
+ * enqueued.  Every call looks up the array's device address in the current context
+ * (a host-side query); the first call on a device may load the library's device code
+ * there, so make that first call before any stream capture.  Calls allocate nothing
  * (no cudaMalloc / cudaFree); each one clears the counters it needs with an
  * asynchronous memset on `stream`.  All calls on a device share the one array:
  * calls that may run concurrently on the GPU (unordered streams) race and must

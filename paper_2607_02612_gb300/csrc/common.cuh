@@ -42,12 +42,17 @@ constexpr int kImageWarps = kImageThreads / 32;
 
 // Workspace layout (bytes from the workspace base; every block 256-aligned).
 // The slot map and the plan come first, so their offsets depend on max_batch
-// only; the exit counters and partial softmax sums follow.
+// only; the exit counters and partial softmax sums follow, then the logits tiles of
+// the general exit kernel (heads of more than kExitClMaxTiles class tiles only: its
+// CTAs cannot wait for one another, so the last CTA of a sample tile copies the rows
+// of the samples that exit from there).
+constexpr int kExitClMaxTiles = 8;   // class tiles of the cluster exit kernel (portable cluster size)
 struct WsLayout {
     size_t slot;       // int[max_batch]: output sample of every input sample
     size_t plan;       // int[4]: batch valid, survivor count
     size_t counters;   // int[n_btile + 1], zero between calls
     size_t partials;   // float2[n_btile * kExitBT * n_ctile]
+    size_t lg;         // float[n_btile * kExitBT][classes] (empty for heads of <= kExitClMaxTiles tiles)
     size_t total;
 };
 
@@ -67,6 +72,8 @@ __host__ __device__ inline WsLayout ws_layout(int max_batch, int classes) {
     off += align256(sizeof(int) * (size_t)(nbt + 1));
     L.partials = off;
     off += align256(sizeof(float) * 2 * (size_t)nbt * kExitBT * (size_t)nct);
+    L.lg = off;
+    if (nct > kExitClMaxTiles) off += align256(sizeof(float) * (size_t)nbt * kExitBT * (size_t)(classes > 0 ? classes : 1));
     L.total = off;
     return L;
 }

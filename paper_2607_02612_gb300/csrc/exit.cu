@@ -204,10 +204,10 @@ __device__ __forceinline__ void exit_logits(const ExitParams &p, float *lg_s, co
         }
     }
     __syncthreads();
-    if (p.logits) {
+    if (p.lg_tmp) {   // staged: the last CTA of the sample tile writes the rows of the samples that exit
         for (int it = tid; it < kExitBT * kExitCT; it += kExitThreads) {
             const int sl = it / kExitCT, col = it - sl * kExitCT;
-            if (s0 + sl < B && c0 + col < C) p.logits[(size_t)(s0 + sl) * C + c0 + col] = lg_s[it];
+            if (s0 + sl < B && c0 + col < C) p.lg_tmp[(size_t)(s0 + sl) * C + c0 + col] = lg_s[it];
         }
     }
 }
@@ -404,12 +404,16 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
             }
 #pragma unroll
             for (int o = 16; o >= 1; o >>= 1) z += __shfl_xor_sync(0xFFFFFFFFu, z, o);
+            const float c = 1.0f / z;   // max_k softmax = exp(l_max - l_max) / sum
+            const bool ex = c >= p.head.tau;
             if (lane == 0) {
-                const float c = 1.0f / z;   // max_k softmax = exp(l_max - l_max) / sum
-                p.exit_mask[s] = (c >= p.head.tau) ? 1 : 0;
+                p.exit_mask[s] = ex ? 1 : 0;
                 if (p.max_prob) p.max_prob[s] = c;
                 if (!isfinite(m)) raise_status(p.status, FUSION_DEV_NONFINITE);
             }
+            if (ex && p.logits && p.lg_tmp)   // logits only for the samples that exit
+                for (int col = lane; col < p.head.classes; col += 32)
+                    p.logits[(size_t)s * p.head.classes + col] = __ldcg(&p.lg_tmp[(size_t)s * p.head.classes + col]);
         }
     }
     if (tid == 0) p.counters[bt] = 0;
@@ -544,6 +548,7 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
     const int ngr = kWarps / G;
     const int jw = warp / G, gt = tid - jw * G * 32;   // row of this warp in a round, thread index in its group
 
+    if (tid == 0) s_wfail = 0;
     if (active && kBf16 && warp == 0) {   // the logits tile's accumulator
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(&tmem_base)),
                      "r"(kExitTmemCols)
@@ -558,7 +563,6 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
             mbar_init(smem_addr(&wempty[q]), 1);
         }
         mbar_init(smem_addr(&wdone), 1);
-        s_wfail = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         for (int q = 0; q < nws; ++q) {
             mbar_expect_tx(smem_addr(&wbar[q]), kExitWStage);
@@ -753,7 +757,8 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
             __syncthreads();
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             // logits (+ bias) into shared memory: warp w < 4 reads the lanes (classes) 32w.. of D
-            if (warp < 4) {
+            // (not after a timed-out wait: the product may be incomplete)
+            if (warp < 4 && s_wfail == 0) {
                 uint32_t v[16];
                 tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16), v);
                 const int cls = warp * 32 + lane;
@@ -766,18 +771,13 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
             if (warp == 0)
                 asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kExitTmemCols)
                              : "memory");
-            if (p.logits) {
-                for (int it = tid; it < BT * kExitCT; it += kExitThreads) {
-                    const int sl = it / kExitCT, col = it - sl * kExitCT;
-                    if (s0 + sl < B && c0 + col < C) p.logits[(size_t)(s0 + sl) * C + c0 + col] = lg_s[it];
-                }
-            }
         } else {
             exit_gemm<T>(p, u_s, w_region, c0, dim, C, n_k, acc, acc2);
             exit_logits<T>(p, lg_s, bias_s, acc, acc2, s0, c0, B, C);
         }
-        // partial softmax of this class tile, warp -> sample slots warp, warp + 8, ...; to the
-        // sample's owner
+        // partial softmax of this class tile, warp -> sample slots warp, warp + 8, ...; to every
+        // CTA of the cluster (a tile whose product timed out sends z = -1: no decision)
+        const bool failed = s_wfail != 0;
         for (int slw = warp; slw < BT; slw += kWarps) {
             const int sw = s0 + slw;
             float m = -INFINITY;
@@ -791,31 +791,43 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
             }
 #pragma unroll
             for (int o = 16; o >= 1; o >>= 1) z += __shfl_xor_sync(0xFFFFFFFFu, z, o);
-            if (lane == 0 && sw < B) *cl.map_shared_rank(part_s + slw * 8 + rank, slw % ncl) = make_float2(m, z);
+            if (lane < ncl && sw < B)
+                *cl.map_shared_rank(part_s + slw * 8 + rank, lane) = failed ? make_float2(0.0f, -1.0f) : make_float2(m, z);
         }
     }
-    cl.sync();   // every partial is with its owner
+    cl.sync();   // every CTA holds every partial of the tile's samples
+    // Every CTA merges the partials in the same order (so all agree on every decision); the
+    // owner writes the exit mask and c, every CTA its logits tile of the samples that exit.
     for (int slw = warp; active && slw < BT; slw += kWarps) {
         const int sw = s0 + slw;
-        if (slw % ncl == rank && sw < B) {
-            float m = -INFINITY;
-            for (int q = lane; q < ncl; q += 32) m = fmaxf(m, part_s[slw * 8 + q].x);
-#pragma unroll
-            for (int o = 16; o >= 1; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
-            float z = 0.0f;
-            for (int q = lane; q < ncl; q += 32) {
-                const float2 pz = part_s[slw * 8 + q];
-                z += pz.y * expf(pz.x - m);
-            }
-#pragma unroll
-            for (int o = 16; o >= 1; o >>= 1) z += __shfl_xor_sync(0xFFFFFFFFu, z, o);
-            if (lane == 0) {
-                const float c = 1.0f / z;   // max_k softmax = exp(l_max - l_max) / sum
-                p.exit_mask[sw] = (c >= p.head.tau) ? 1 : 0;
-                if (p.max_prob) p.max_prob[sw] = c;
-                if (!isfinite(m)) raise_status(p.status, FUSION_DEV_NONFINITE);
-            }
+        if (sw >= B) continue;
+        float m = -INFINITY;
+        bool bad = false;
+        for (int q = lane; q < ncl; q += 32) {
+            const float2 pz = part_s[slw * 8 + q];
+            m = fmaxf(m, pz.x);
+            bad = bad || pz.y < 0.0f;
         }
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+        if (__any_sync(0xFFFFFFFFu, bad)) continue;   // a product timed out: no decision (status raised)
+        float z = 0.0f;
+        for (int q = lane; q < ncl; q += 32) {
+            const float2 pz = part_s[slw * 8 + q];
+            z += pz.y * expf(pz.x - m);
+        }
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) z += __shfl_xor_sync(0xFFFFFFFFu, z, o);
+        const float c = 1.0f / z;   // max_k softmax = exp(l_max - l_max) / sum
+        const bool ex = c >= p.head.tau;
+        if (slw % ncl == rank && lane == 0) {
+            p.exit_mask[sw] = ex ? 1 : 0;
+            if (p.max_prob) p.max_prob[sw] = c;
+            if (!isfinite(m)) raise_status(p.status, FUSION_DEV_NONFINITE);
+        }
+        if (ex && p.logits)   // logits only for the samples that exit
+            for (int col = lane; col < kExitCT; col += 32)
+                if (c0 + col < C) p.logits[(size_t)sw * C + c0 + col] = lg_s[slw * kExitCT + col];
     }
     if (!p.do_plan) {
         if (Bdev < 0 && bt == 0 && rank == 0 && tid == 0) raise_status(p.status, FUSION_DEV_BAD_BATCH);
@@ -863,8 +875,10 @@ cudaError_t launch_exit_cluster(const ExitParams &p, cudaStream_t s) {
     const size_t smem = ExitClSmem<T>::total(p.dim);
     cudaError_t e = cudaFuncSetAttribute(k_exit_cl<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    ExitParams q = p;   // sample tiles of this kernel's size (the plan's cluster count)
-    q.n_btile = (p.in.max_batch + ExitClSmem<T>::BT - 1) / ExitClSmem<T>::BT;
+    ExitParams q = p;   // sample tiles of this kernel's size (the plan's cluster count), at least
+                        // one: with max_batch == 0 the kernel still runs the plan
+    q.n_btile = ceil_div(p.in.max_batch > 0 ? p.in.max_batch : 1, ExitClSmem<T>::BT);
+    q.lg_tmp = nullptr;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(q.n_ctile, q.n_btile);
     cfg.blockDim = dim3(kExitThreads);
@@ -883,7 +897,7 @@ cudaError_t launch_exit_cluster(const ExitParams &p, cudaStream_t s) {
 cudaError_t launch_exit(int dtype, const ExitParams &p, cudaStream_t s) {
     // the class tiles of a sample tile as one cluster (portable size: at most 8 tiles,
     // 1024 classes); larger heads take the kernel with a global last-CTA merge
-    if (p.n_ctile <= 8 && p.n_btile > 0 && p.in_mode == 0 && !p.skip_ln && p.out_mode == 0)
+    if (p.n_ctile <= kExitClMaxTiles && p.in_mode == 0 && !p.skip_ln && p.out_mode == 0)
         return dtype == FUSION_BF16 ? launch_exit_cluster<__nv_bfloat16>(p, s) : launch_exit_cluster<float>(p, s);
     const size_t smem = exit_smem_bytes(dtype, p.dim);
     const dim3 grid(p.n_ctile, p.n_btile);

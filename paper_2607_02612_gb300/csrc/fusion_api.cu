@@ -60,13 +60,15 @@ struct Ws {
     int *plan;
     int *counters;
     float2 *partials;
+    float *lg;   // logits tiles of the general exit kernel (NULL for heads it does not run)
 };
 
 Ws carve(void *ws, int32_t max_batch, int32_t classes) {
     const WsLayout L = ws_layout(max_batch, classes);
     unsigned char *b = static_cast<unsigned char *>(ws);
     return Ws{reinterpret_cast<int *>(b + L.slot), reinterpret_cast<int *>(b + L.plan),
-              reinterpret_cast<int *>(b + L.counters), reinterpret_cast<float2 *>(b + L.partials)};
+              reinterpret_cast<int *>(b + L.counters), reinterpret_cast<float2 *>(b + L.partials),
+              L.total > L.lg ? reinterpret_cast<float *>(b + L.lg) : nullptr};
 }
 
 int cuda_rc(cudaError_t e) { return e == cudaSuccess ? FUSION_OK : FUSION_ERR_CUDA; }
@@ -251,6 +253,7 @@ int fusion_exit_check(int dtype, fusion_ragged in, const void *x, int32_t dim,
     e.max_prob = max_prob;
     e.counters = w.counters;
     e.partials = w.partials;
+    e.lg_tmp = logits ? w.lg : nullptr;
     e.n_ctile = ceil_div(head.classes, kExitCT);
     e.n_btile = ceil_div(in.max_batch > 0 ? in.max_batch : 1, kExitBT);
     e.do_plan = 0;
@@ -370,14 +373,18 @@ namespace {
 // fusion_exit_check_mlp scratch: the linear exit workspace for `classes`, then the pooled
 // rows [max_batch, dim] float32 and the hidden rows [max_batch, hidden] (float32 size).
 struct MlpWs {
-    size_t u, hid, total;
+    size_t u, hid, lg, total;
 };
+// The stage's own scratch, the pooled rows (float32), the hidden rows (at most float32) and
+// the second layer's logits tiles (the general exit kernel writes exited rows from there).
 MlpWs mlp_ws_layout(int32_t max_batch, int32_t dim, int32_t hidden, int32_t classes) {
     const size_t mb = (size_t)(max_batch > 0 ? max_batch : 1);
+    const size_t tiles = (size_t)ceil_div(max_batch > 0 ? max_batch : 1, kExitBT) * kExitBT;
     MlpWs L;
     L.u = (ws_layout(max_batch, classes).total + 255) / 256 * 256;
     L.hid = (L.u + mb * (size_t)dim * sizeof(float) + 255) / 256 * 256;
-    L.total = (L.hid + mb * (size_t)hidden * sizeof(float) + 255) / 256 * 256;
+    L.lg = (L.hid + mb * (size_t)hidden * sizeof(float) + 255) / 256 * 256;
+    L.total = (L.lg + tiles * (size_t)classes * sizeof(float) + 255) / 256 * 256;
     return L;
 }
 }  // namespace
@@ -440,6 +447,7 @@ int launch_exit_mlp(int dtype, const fusion_ragged &in, const void *x, int32_t d
     l2.max_prob = max_prob;
     l2.counters = w.counters;
     l2.partials = w.partials;
+    l2.lg_tmp = logits ? reinterpret_cast<float *>(wb + L.lg) : nullptr;
     l2.n_ctile = ceil_div(head.classes, kExitCT);
     l2.n_btile = n_btile;
     l2.status = dev_status;
@@ -605,6 +613,7 @@ int stage_impl(int dtype, int flags, const fusion_ragged &in, const void *x, int
         e.max_prob = max_prob;
         e.counters = w.counters;
         e.partials = w.partials;
+    e.lg_tmp = logits ? w.lg : nullptr;
         e.n_ctile = ceil_div(head.classes, kExitCT);
         e.n_btile = ceil_div(in.max_batch > 0 ? in.max_batch : 1, kExitBT);
         e.do_plan = !fuse_plan(in);

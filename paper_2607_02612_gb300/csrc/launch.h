@@ -19,6 +19,9 @@ struct ExitParams {
     float *max_prob;
     int *counters;   // workspace: [n_btile + 1], zero on entry, zero on exit
     float2 *partials;
+    float *lg_tmp;   // workspace [n_btile * kExitBT][classes]: logits tiles of the general kernel (its
+                     // last CTA per sample tile writes the rows of the samples that exit); NULL when
+                     // no logits are requested or the cluster kernel runs
     int n_ctile;
     int n_btile;
     int do_plan;     // run the compaction plan in the last CTA

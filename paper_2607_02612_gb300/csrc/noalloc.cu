@@ -9,38 +9,30 @@
 // per-sample plan) lives in one file-scope device array.
 //
 // Limits and sharing: the array holds kNoAllocScratchBytes bytes on every GPU that
-// loads the library, for the life of the process.  A call whose batch bound and
+// loads the library, for the life of the process.  The first call on a device may load
+// the library's device code there (lazy module loading), so make it before any stream
+// capture.  A call whose batch bound and
 // class count need more returns FUSION_ERR_WORKSPACE and enqueues nothing.  All
 // calls on a device share the same array and it keeps the previous call's
 // contents, so each call first clears the counters that must start at zero;
 // calls that overlap on the GPU (different streams, no ordering between them)
 // race on the array and must not be issued.
-#include <mutex>
-
 #include "launch.h"
 
 namespace {
 
 constexpr size_t kNoAllocScratchBytes = 1u << 20;   // 1 MiB
-constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
-std::mutex g_setup_mutex;
-void *g_scratch_addr[kMaxDevices] = {};
-
-// Device address of the scratch array on the current device, looked up once per
-// device (the host-side symbol is only a stand-in, not a device address).
+// Device address of the scratch array in the current device's context.  The host-side
+// symbol is only a stand-in, not a device address.  The address is looked up on every
+// call (a host-side query), so a context that was torn down and created again (after
+// cudaDeviceReset, for instance) never receives a stale address.
 int scratch_on_current_device(unsigned char **out) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return FUSION_ERR_CUDA;
-    std::lock_guard<std::mutex> lock(g_setup_mutex);
-    if (!g_scratch_addr[dev]) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return FUSION_ERR_CUDA;
-        g_scratch_addr[dev] = p;
-    }
-    *out = static_cast<unsigned char *>(g_scratch_addr[dev]);
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return FUSION_ERR_CUDA;
+    *out = static_cast<unsigned char *>(p);
     return FUSION_OK;
 }
 
@@ -79,6 +71,7 @@ extern "C" int fusion_exit_check_noalloc(int dtype, fusion_ragged in, const void
     e.max_prob = max_prob;
     e.counters = reinterpret_cast<int *>(base + L.counters);
     e.partials = reinterpret_cast<float2 *>(base + L.partials);
+    e.lg_tmp = (logits && L.total > L.lg) ? reinterpret_cast<float *>(base + L.lg) : nullptr;
     e.n_ctile = ceil_div(head.classes, kExitCT);
     e.n_btile = ceil_div(in.max_batch > 0 ? in.max_batch : 1, kExitBT);
     e.do_plan = 0;

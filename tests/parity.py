@@ -99,12 +99,19 @@ def compare_exit(rep: Report, dtype: str, ids: np.ndarray, g_mask, g_logits, g_m
             else:
                 rep.fail(f"exit mask differs for sample id {ids[i]} (c={o['max_prob'][i]}, gap={gap[i]:.3g})")
     keep = np.array([int(t) not in skip for t in ids], bool)
-    if g_logits is not None and keep.any():
-        e = rel_err_rows(g_logits[keep], o["logits"][keep])
-        rep.max_rel_err["logits"] = max(rep.max_rel_err["logits"], float(e.max()))
-        bad = np.nonzero(e > TOL[dtype])[0]
-        for b in bad[:3]:
-            rep.fail(f"logits of sample {np.nonzero(keep)[0][b]} off by {e[b]:.3g} (rel)")
+    if g_logits is not None:
+        # logits are the early prediction: written for the samples that exit, the other rows
+        # are left as they were (zero in every caller here)
+        ex = keep & (o["exit_mask"] == 1) & (g_mask == o["exit_mask"])
+        if ex.any():
+            e = rel_err_rows(g_logits[ex], o["logits"][ex])
+            rep.max_rel_err["logits"] = max(rep.max_rel_err["logits"], float(e.max()))
+            bad = np.nonzero(e > TOL[dtype])[0]
+            for b in bad[:3]:
+                rep.fail(f"logits of sample {np.nonzero(ex)[0][b]} off by {e[b]:.3g} (rel)")
+        stay = keep & (g_mask == 0)
+        if stay.any() and np.any(g_logits[stay] != 0):
+            rep.fail(f"logits written for {int(np.sum(np.any(g_logits[stay] != 0, axis=1)))} samples that continue")
     if g_maxp is not None and keep.any():
         e = np.abs(g_maxp[keep].astype(np.float64) - o["max_prob"][keep]) / np.maximum(o["max_prob"][keep], 1e-30)
         rep.max_rel_err["max_prob"] = max(rep.max_rel_err["max_prob"], float(e.max()))
@@ -244,10 +251,13 @@ def compare_chain(rep: Report, workload, g_outs, o_outs):
                     rep.fail(f"stage {s}: exit mask differs for sample id {t} "
                              f"(c={o['max_prob'][i]}, gap={gap:.3g})")
                     continue
-                e = rel_err_rows(g["logits"][ig:ig + 1], o["logits"][i:i + 1])[0]
-                rep.max_rel_err["logits"] = max(rep.max_rel_err["logits"], float(e))
-                if e > tol_l:
-                    rep.fail(f"stage {s}: logits of sample id {t} off by {e:.3g}")
+                if o["exit_mask"][i]:   # logits are written only for the samples that exit
+                    e = rel_err_rows(g["logits"][ig:ig + 1], o["logits"][i:i + 1])[0]
+                    rep.max_rel_err["logits"] = max(rep.max_rel_err["logits"], float(e))
+                    if e > tol_l:
+                        rep.fail(f"stage {s}: logits of sample id {t} off by {e:.3g}")
+                elif np.any(g["logits"][ig] != 0):
+                    rep.fail(f"stage {s}: logits written for sample id {t}, which continues")
                 ep = abs(float(g["max_prob"][ig]) - float(o["max_prob"][i])) / max(float(o["max_prob"][i]), 1e-30)
                 rep.max_rel_err["max_prob"] = max(rep.max_rel_err["max_prob"], ep)
                 if ep > tol_p:

@@ -1,11 +1,12 @@
 """bench.py's algorithmic bytes per stage (the roofline's numerator), on hand-counted cases (CPU).
 
 Per stage: the exit check reads every input CLS row, the head (W, bias, gamma, beta) and writes
-logits, mask and max-prob per input image; the plan reads offsets and r/rho and writes the output
-offsets, ids and slots.  Per surviving image the per-sample kernel reads all its keys when it
-merges (every key takes part in the decision), else only the rows it keeps, plus sizes and scores
-of every input row and a few scalars, and writes each output row with its size, score and row id.
-An exited image costs nothing in the per-sample kernel.
+mask and max-prob per input image and logits per image that exits; the plan reads offsets and
+r/rho and writes the output offsets, ids and slots.  Per surviving image the per-sample kernel
+reads all its keys when it merges (every key takes part in the decision), else only the rows it
+keeps, plus sizes and scores of every input row and a few scalars, and writes each output row with
+its size and score (and its input row id when the caller asks for it).  An exited image costs
+nothing in the per-sample kernel.
 """
 import os
 import sys
@@ -28,13 +29,17 @@ def test_stage_bytes_hand_counted():
     in_ids = np.array([0, 1, 2], np.int32)
     out_off = np.array([0, 2, 5], np.int32)
     out_ids = np.array([1, 2], np.int32)
-    first, image = bench.stage_bytes(spec, "bf16", d, in_off, in_ids, out_off, out_ids, C)
-    exit_bytes = 3 * 32 + C * 32 + C * 4 + 2 * 32 + 3 * (C * 4 + 1 + 4)   # CLS rows, W, b, gamma+beta; outputs
+    first, image = bench.stage_bytes(spec, "bf16", d, in_off, in_ids, out_off, out_ids, C, row_ids=True)
+    exit_bytes = 3 * 32 + C * 32 + C * 4 + 2 * 32 + 1 * C * 4 + 3 * (1 + 4)   # CLS rows, W, b, gamma+beta;
+    #                                                                         logits of the 1 exit, mask, c
     plan_bytes = 4 * 4 + 3 * 8 + 2 * 12 + 4                                # offsets, r+rho, per output, count
-    assert first == exit_bytes + plan_bytes == 655 + 68
+    assert first == exit_bytes + plan_bytes == 575 + 68
     img1 = 3 * 32 + 3 * 8 + 16 + 2 * (32 + 12)     # all 3 keys read (it merges), 2 rows written
     img2 = 3 * 32 + 4 * 8 + 16 + 3 * (32 + 12)     # no merge: only the 3 kept rows read
     assert image == img1 + img2 == 224 + 276
+    # without row ids (the timed chain does not ask for them): 4 bytes fewer per output row
+    _, image2 = bench.stage_bytes(spec, "bf16", d, in_off, in_ids, out_off, out_ids, C)
+    assert image2 == image - 5 * 4
 
 
 def test_stage_bytes_without_exit():
@@ -43,4 +48,4 @@ def test_stage_bytes_without_exit():
     first, image = bench.stage_bytes(spec, "f32", d, np.array([0, 7], np.int32), np.array([0], np.int32),
                                      np.array([0, 6], np.int32), np.array([0], np.int32), 0)
     assert first == 2 * 4 + 8 + 12 + 4
-    assert image == 7 * 128 + 7 * 8 + 16 + 6 * (128 + 12)
+    assert image == 7 * 128 + 7 * 8 + 16 + 6 * (128 + 8)

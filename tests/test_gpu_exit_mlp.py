@@ -43,8 +43,10 @@ def _run(b, head, batch=None, max_tokens=None):
 
 def _compare(dtype, g, o, label, n=None):
     n = len(o["max_prob"]) if n is None else n
-    e = P.rel_err_rows(g["logits"][:n], o["logits"][:n])
+    ex = (o["exit_mask"][:n] == 1) & (g["exit_mask"][:n] == 1)   # logits: the rows of samples that exit
+    e = P.rel_err_rows(g["logits"][:n][ex], o["logits"][:n][ex]) if ex.any() else np.zeros(1)
     assert e.max() <= TOL_LOGITS[dtype], (label, float(e.max()), int(e.argmax()))
+    assert not np.any(g["logits"][:n][g["exit_mask"][:n] == 0]), (label, "logits written for samples that continue")
     pe = np.abs(g["max_prob"][:n].astype(np.float64) - o["max_prob"][:n]) / o["max_prob"][:n]
     assert pe.max() <= TOL_MAXP[dtype], (label, float(pe.max()))
     near = o["exit_gap"][:n] < TOL_MAXP[dtype] * o["max_prob"][:n]

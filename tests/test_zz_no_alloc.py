@@ -1,11 +1,12 @@
-"""fusion_exit_check_noalloc against fusion_exit_check (GPU only).
+"""fusion_exit_check_noalloc against fusion_exit_check and the oracle (GPU only).
 
 The no-allocation variant serves callers that cannot call cudaMalloc (plugin hosts
 that pass only inputs and outputs, programs without a device allocator).  It must
 give the same exit decisions, logits and max-probabilities as the workspace-based
-call, on two calls in a row (the built-in scratch keeps the previous call's
-contents, so the second call checks that the per-call reset works), and it must
-refuse a batch whose scratch would not fit.  This file is collected last.
+call and as the oracle, on two calls in a row that share the built-in scratch, and
+it must refuse a batch whose scratch would not fit.  Logits are written only for the
+samples that exit; the other rows keep what the caller put there.  This file is
+collected last.
 """
 import ctypes
 import os
@@ -17,6 +18,7 @@ import torch
 
 sys.path.insert(0, os.path.dirname(os.path.abspath(__file__)))
 
+import oracle  # noqa: E402
 import parity as P  # noqa: E402
 import paper_2607_02612_gb300 as fz  # noqa: E402
 from paper_2607_02612_gb300 import _binding as fb  # noqa: E402
@@ -40,6 +42,11 @@ def test_noalloc_matches_workspace_call_twice(name, B):
     ref = f.exit_check(db, head)
     torch.cuda.synchronize()
     assert int(f.status.item()) == 0
+    orc = oracle.exit_check(b.dtype, b.offsets, b.x, spec.head)
+    ref_mask = ref["exit_mask"].cpu().numpy()
+    decided = orc["exit_gap"] >= P.NEAR_TIE   # decisions with an oracle margin below 1e-6 are only counted
+    assert np.array_equal(ref_mask[decided], orc["exit_mask"][decided]), "workspace call differs from the oracle"
+    ex = ref_mask == 1
     for call in range(2):
         mask = torch.full((b.batch,), 7, dtype=torch.uint8, device="cuda")
         logits = torch.full((b.batch, head.classes), float("nan"), dtype=torch.float32, device="cuda")
@@ -53,10 +60,18 @@ def test_noalloc_matches_workspace_call_twice(name, B):
         assert int(status.item()) == 0
         assert torch.equal(mask, ref["exit_mask"]), f"call {call}: exit masks differ"
         tol = P.TOL[b.dtype]
-        e = P.rel_err_rows(logits.cpu().numpy(), ref["logits"].cpu().numpy())
-        assert e.max() <= tol, f"call {call}: logits off by {e.max()}"
-        ep = np.abs(maxp.cpu().numpy() - ref["max_prob"].cpu().numpy()) / ref["max_prob"].cpu().numpy()
+        lg = logits.cpu().numpy()
+        if ex.any():
+            e = P.rel_err_rows(lg[ex], ref["logits"].cpu().numpy()[ex])
+            assert e.max() <= tol, f"call {call}: logits off by {e.max()}"
+            eo = P.rel_err_rows(lg[ex], orc["logits"][ex])
+            assert eo.max() <= tol, f"call {call}: logits off the oracle's by {eo.max()}"
+        assert np.all(np.isnan(lg[~ex])), f"call {call}: logits written for samples that continue"
+        mp = maxp.cpu().numpy()
+        ep = np.abs(mp - ref["max_prob"].cpu().numpy()) / ref["max_prob"].cpu().numpy()
         assert ep.max() <= tol, f"call {call}: max_prob off by {ep.max()}"
+        epo = np.abs(mp.astype(np.float64) - orc["max_prob"]) / orc["max_prob"]
+        assert epo.max() <= tol, f"call {call}: max_prob off the oracle's by {epo.max()}"
 
 
 def test_noalloc_rejects_batches_beyond_its_scratch():

@@ -613,7 +613,7 @@ int stage_impl(int dtype, int flags, const fusion_ragged &in, const void *x, int
         e.max_prob = max_prob;
         e.counters = w.counters;
         e.partials = w.partials;
-    e.lg_tmp = logits ? w.lg : nullptr;
+        e.lg_tmp = logits ? w.lg : nullptr;
         e.n_ctile = ceil_div(head.classes, kExitCT);
         e.n_btile = ceil_div(in.max_batch > 0 ? in.max_batch : 1, kExitBT);
         e.do_plan = !fuse_plan(in);

@@ -557,12 +557,13 @@ __device__ __forceinline__ uint4 merged_value(const MetaPtrs &m, const MergedIte
         return merged_compute<T>(m, it, load);
 }
 
-// Requires sel / match / mkey / tsize / tscore ready (after a barrier).  `load(pos, c)`
-// returns the 16-byte chunk c of input token pos.  Returns false (after raising
-// FUSION_DEV_INTERNAL) if the token count disagrees with the plan; uniform per CTA.
-template <typename T, int NT, typename Loader>
-__device__ bool finish_sample(const ImageParams &p, const SampleInfo &s, MetaPtrs &m, const Loader &load) {
-    constexpr int CH = Elem<T>::kPerChunk;
+// The decisions after the matching, up to the output position of every kept token:
+// merged set, merged sizes and scores, pruning, the scan of kept tokens and the source of
+// every output row.  Requires sel / match / mkey / tsize / tscore ready (after a barrier);
+// needs s.out_n but not s.out_start.  Returns false (after raising FUSION_DEV_INTERNAL) if
+// the token count disagrees with the plan; uniform per CTA.
+template <int NT>
+__device__ bool finish_decide(const ImageParams &p, const SampleInfo &s, MetaPtrs &m) {
     const int tid = threadIdx.x;
     const int N = s.N, nB = s.nB, R = s.r_eff;
 
@@ -658,6 +659,17 @@ __device__ bool finish_sample(const ImageParams &p, const SampleInfo &s, MetaPtr
     for (int pos = tid; pos < N; pos += NT)
         if (m.kflag[pos]) m.srcpos[m.opos[pos]] = m.mflag[pos] == 2 ? ~pos : pos;
     __syncthreads();
+    return true;
+}
+
+// The outputs of a decided sample (after finish_decide): index outputs, copied token rows
+// and merged token rows at s.out_start.  `load(pos, c)` returns the 16-byte chunk c of
+// input token pos.
+template <typename T, int NT, typename Loader>
+__device__ void finish_write(const ImageParams &p, const SampleInfo &s, MetaPtrs &m, const Loader &load) {
+    constexpr int CH = Elem<T>::kPerChunk;
+    const int tid = threadIdx.x;
+    const int N = s.N;
 
     // index outputs
     const int start = s.start, out_start = s.out_start, out_n = s.out_n;
@@ -720,6 +732,13 @@ __device__ bool finish_sample(const ImageParams &p, const SampleInfo &s, MetaPtr
             *reinterpret_cast<uint4 *>(xo + m.opos[cur.pos] * dim + cur.c * CH) = merged_value<T>(m, cur, load);
         cur = nxt;
     }
+}
+
+// finish_decide then finish_write (the plan's output offsets already known).
+template <typename T, int NT, typename Loader>
+__device__ bool finish_sample(const ImageParams &p, const SampleInfo &s, MetaPtrs &m, const Loader &load) {
+    if (!finish_decide<NT>(p, s, m)) return false;
+    finish_write<T, NT>(p, s, m, load);
     return true;
 }
 

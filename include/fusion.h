@@ -385,16 +385,26 @@ int fusion_stage(int dtype, int flags, fusion_ragged in, const void *x, int32_t 
                  void *stream);
 
 /*
+ * Bytes of scratch of fusion_stage_mlp with both FUSION_STAGE_MERGE and FUSION_STAGE_EXIT:
+ * the MLP head's scratch (fusion_exit_mlp_workspace_size) and room for the merged batch
+ * (max_rows token rows of dim elements at 4 bytes each, their sizes, scores and input rows,
+ * and max_batch + 1 offsets).  Zero-filled before its first use, left zero-filled by every call.
+ */
+size_t fusion_stage_mlp_workspace_size(int32_t max_batch, int64_t max_rows, int32_t dim, int32_t hidden,
+                                       int32_t classes);
+
+/*
  * fusion_stage_mlp: fusion_stage with one of the paper's MLP exit heads (Sec. III-G: a
  * SpatialPool head at block 8, a CLS-only head at block 10) in place of the linear head.
- * The exit check is fusion_exit_check_mlp on the stage's INPUT rows: merging never
- * changes CLS, and it keeps sum_t s_t x_t and sum_t s_t over the patch rows (a merged
- * token of size s_B + sum s_A carries s_B x_B + sum s_A x_A, Sec. III-C), so the
- * size-weighted pool of the input equals that of the merged tokens in exact arithmetic.
- * Arguments as fusion_stage; head as fusion_exit_check_mlp (read only with
- * FUSION_STAGE_EXIT); workspace: at least fusion_exit_mlp_workspace_size(in.max_batch,
- * dim, head.hidden, head.classes) bytes with the exit check, else
- * fusion_workspace_size(in.max_batch, 1), zero-filled before first use and left so.
+ * The exit check reads the merged tokens (Sec. III-B): with FUSION_STAGE_MERGE the call merges
+ * into its workspace, runs fusion_exit_check_mlp on that batch (pooling the merged rows as
+ * stored, rounded to the dtype), then compacts and prunes from it; keep_idx and a_match still
+ * refer to the input rows.  Arguments as fusion_stage; head as fusion_exit_check_mlp (read
+ * only with FUSION_STAGE_EXIT); workspace: at least fusion_stage_mlp_workspace_size(
+ * in.max_batch, in.max_rows, dim, head.hidden, head.classes) bytes with both merging and the
+ * exit check, fusion_exit_mlp_workspace_size(in.max_batch, dim, head.hidden, head.classes)
+ * with the exit check alone, else fusion_workspace_size(in.max_batch, 1); zero-filled before
+ * first use and left so.
  * Errors: those of fusion_stage and fusion_exit_check_mlp.
  */
 int fusion_stage_mlp(int dtype, int flags, fusion_ragged in, const void *x, int32_t dim,

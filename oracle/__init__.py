@@ -313,10 +313,8 @@ def stage(batch, spec) -> Dict[str, object]:
     (if enabled; exited samples leave the batch) -> prune the survivors (if
     enabled).  Per-sample router outputs spec.r / spec.rho are indexed by the
     samples' original ids.  With spec.mlp_head (an MLP exit head, Sec. III-G) the
-    exit check reads the stage's input rows: merging keeps CLS and, over the patch
-    rows, sum s_t x_t and sum s_t (Sec. III-C), so the CLS-only and the size-weighted
-    pooled head inputs of the input equal those of the merged tokens in exact
-    arithmetic.  Returns the output batch fields plus exit_mask, logits, max_prob
+    exit check reads the merged tokens as stored (rounded to the dtype), as Sec. III-B
+    defines it for every exit head.  Returns the output batch fields plus exit_mask, logits, max_prob
     (indexed by input sample), keep_idx (input row of every output row), a_match
     (input rows) and the decision margins."""
     dtype = batch.dtype
@@ -339,7 +337,7 @@ def stage(batch, spec) -> Dict[str, object]:
     res["exit_gap"] = np.full(B, np.inf)
     if spec.exit:
         if getattr(spec, "mlp_head", None) is not None:
-            e = exit_mlp(dtype, batch.offsets, batch.x[:T], batch.sizes[:T], spec.mlp_head)
+            e = exit_mlp(dtype, offsets, x, sizes, spec.mlp_head)
             mask = e["exit_mask"]
             res.update(exit_mask=mask, logits=e["logits"], max_prob=e["max_prob"], exit_gap=e["exit_gap"])
         else:

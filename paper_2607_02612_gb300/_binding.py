@@ -45,7 +45,8 @@ FUSION_POOL_SPATIAL = 1
 EXPORTED = ("fusion_status_string", "fusion_version", "fusion_profile_next", "fusion_workspace_size",
             "fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune", "fusion_compact",
             "fusion_stage", "fusion_merge_router", "fusion_token_scores", "fusion_exit_mlp_workspace_size",
-            "fusion_exit_check_mlp", "fusion_attention", "fusion_stage_mlp")
+            "fusion_exit_check_mlp", "fusion_attention", "fusion_stage_mlp",
+            "fusion_stage_mlp_workspace_size")
 
 
 class FusionError(RuntimeError):
@@ -111,13 +112,16 @@ def load(path: Optional[str] = None):
     lib.fusion_token_scores.argtypes = [ctypes.c_int, R, V, I32, V, ctypes.c_float, V, V, V]
     lib.fusion_exit_mlp_workspace_size.argtypes = [I32, I32, I32, I32]
     lib.fusion_exit_mlp_workspace_size.restype = SZ
+    lib.fusion_stage_mlp_workspace_size.argtypes = [I32, I64, I32, I32, I32]
+    lib.fusion_stage_mlp_workspace_size.restype = SZ
     lib.fusion_exit_check_mlp.argtypes = [ctypes.c_int, R, V, I32, V, fusion_mlp_head, V, V, V, V, SZ, V, V]
     lib.fusion_attention.argtypes = [ctypes.c_int, R, V, I32, I32, V, V, V, V]
     lib.fusion_stage_mlp.argtypes = [ctypes.c_int, ctypes.c_int, R, V, I32, V, I32, V, V, V, V, fusion_mlp_head, V,
                                      V, V, V, V, V, V, V, V, V, V, V, SZ, V, V]
     for name in ("fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune",
                  "fusion_compact", "fusion_stage", "fusion_merge_router", "fusion_token_scores",
-                 "fusion_exit_check_mlp", "fusion_attention", "fusion_stage_mlp"):
+                 "fusion_exit_check_mlp", "fusion_attention", "fusion_stage_mlp",
+            "fusion_stage_mlp_workspace_size"):
         getattr(lib, name).restype = ctypes.c_int
     del I64, F
     if path is None:
@@ -231,6 +235,11 @@ def fusion_token_scores(dtype, in_, x, dim, w, b, scores_out, dev_status, stream
     """Prune scores from a linear pruning router, s = w . z + b per token row (Sec. III-E, Eq. 8)."""
     return load().fusion_token_scores(int(dtype), in_, _ptr(x), int(dim), _ptr(w), float(b), _ptr(scores_out),
                                       _ptr(dev_status), _stream(stream))
+
+
+def fusion_stage_mlp_workspace_size(max_batch: int, max_rows: int, dim: int, hidden: int, classes: int) -> int:
+    return int(load().fusion_stage_mlp_workspace_size(int(max_batch), int(max_rows), int(dim), int(hidden),
+                                                       int(classes)))
 
 
 def fusion_exit_mlp_workspace_size(max_batch: int, dim: int, hidden: int, classes: int) -> int:

@@ -179,6 +179,29 @@ __device__ __forceinline__ void exit_logits(const ExitParams &p, float *lg_s, co
     }
 }
 
+// Error scale of a hidden unit's pre-activation from the product above (bf16 mma.sync,
+// float32 sums flushed every 64 dims): about sqrt(30) roundings of at most 2^-24 relative to
+// partial sums bounded by sum |w u| <= ||w|| ||u||, with a safety factor of 8.
+constexpr float kHidErr = 0x1p-19f;
+
+// A hidden unit exactly: a = w . u + b1 from exact bf16 x bf16 products summed in float-float,
+// then GELU in double in the erf form, rounded once to bf16.
+static __device__ __noinline__ uint16_t hidden_exact_bf16(const __nv_bfloat16 *w, const __nv_bfloat16 *u, int dim,
+                                                          float b1) {
+    F2 acc = {0.0f, 0.0f};
+    for (int c = 0; c < dim; c += 8) {
+        float wf[8], uf[8];
+        chunk_to_f(ldg16(w + c), wf);
+        chunk_to_f(*reinterpret_cast<const uint4 *>(u + c), uf);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc = f2_add_f(acc, __fmul_rn(wf[e], uf[e]));
+    }
+    acc = f2_add_f(acc, b1);
+    const double a = (double)acc.hi + (double)acc.lo;
+    const double g = 0.5 * a * (1.0 + erf(a / sqrt(2.0)));
+    return __bfloat16_as_ushort(__double2bfloat16(g));
+}
+
 template <typename T>
 __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
@@ -243,6 +266,17 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
         T *xr = u_s + (size_t)warp * u_stride;
         // the row's chunk c as floats: from the tile, or from the float32 input rows
         const float *ur = p.in_mode == 2 && ok ? p.u_in + (size_t)s * dim : nullptr;
+        const float *url = ur && p.u_in_lo ? p.u_in_lo + (size_t)s * dim : nullptr;   // float-float low parts
+        auto in_lo = [&](int c, float (&f)[CH]) {
+#pragma unroll
+            for (int e = 0; e < CH; e += 4) {
+                const float4 v = url ? *reinterpret_cast<const float4 *>(url + c * CH + e) : make_float4(0.f, 0.f, 0.f, 0.f);
+                f[e] = v.x;
+                f[e + 1] = v.y;
+                f[e + 2] = v.z;
+                f[e + 3] = v.w;
+            }
+        };
         auto in_chunk = [&](int c, float (&f)[CH]) {
             if (ur) {
 #pragma unroll
@@ -258,24 +292,30 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
             }
         };
         if (ok && !p.skip_ln) {
-            float ss = 0.0f, sc = 0.0f;
+            float ss = 0.0f, sc = 0.0f, sl_lo = 0.0f;
             for (int c = lane; c < nchunk; c += 32) {
-                float f[CH];
+                float f[CH], fl[CH];
                 in_chunk(c, f);
 #pragma unroll
                 for (int e = 0; e < CH; ++e) neu_add(ss, sc, f[e]);
+                if (url) {
+                    in_lo(c, fl);
+#pragma unroll
+                    for (int e = 0; e < CH; ++e) sl_lo = __fadd_rn(sl_lo, fl[e]);
+                }
             }
             const F2 rdim = f2_recip((float)dim);
-            const F2 mean = f2_mul(warp_sum_f2(two_sum(ss, sc)), rdim);
+            const F2 mean = f2_mul(warp_sum_f2(url ? f2_add_f(two_sum(ss, sc), sl_lo) : two_sum(ss, sc)), rdim);
             ss = sc = 0.0f;
             float lo = 0.0f;
             for (int c = lane; c < nchunk; c += 32) {
-                float f[CH];
+                float f[CH], fl[CH];
                 in_chunk(c, f);
+                in_lo(c, fl);
 #pragma unroll
                 for (int e = 0; e < CH; ++e) {
                     F2 d = two_sum(f[e], -mean.hi);
-                    d.lo = __fsub_rn(d.lo, mean.lo);
+                    d.lo = url ? __fadd_rn(__fsub_rn(d.lo, mean.lo), fl[e]) : __fsub_rn(d.lo, mean.lo);
                     const F2 sq = two_prod(d.hi, d.hi);
                     neu_add(ss, sc, sq.hi);
                     lo = __fmaf_rn(2.0f * d.hi, d.lo, __fadd_rn(lo, sq.lo));
@@ -287,23 +327,33 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
             const T *g = reinterpret_cast<const T *>(p.head.gamma);
             const T *bb = reinterpret_cast<const T *>(p.head.beta);
             for (int c = lane; c < nchunk; c += 32) {
-                float f[CH], gf[CH], bf[CH];
+                float f[CH], fl[CH], gf[CH], bf[CH];
                 in_chunk(c, f);
+                in_lo(c, fl);
                 chunk_to_f(ldg16(g + c * CH), gf);
                 chunk_to_f(ldg16(bb + c * CH), bf);
                 if constexpr (kBf16) {
                     uint32_t w4[4];
+                    if (url) {
 #pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        w4[q] = (uint32_t)ln_out_bf16(f[2 * q], mean, rstd, gf[2 * q], bf[2 * q]) |
-                                ((uint32_t)ln_out_bf16(f[2 * q + 1], mean, rstd, gf[2 * q + 1], bf[2 * q + 1]) << 16);
+                        for (int q = 0; q < 4; ++q)
+                            w4[q] = (uint32_t)ln_out_bf16_lo(f[2 * q], fl[2 * q], mean, rstd, gf[2 * q], bf[2 * q]) |
+                                    ((uint32_t)ln_out_bf16_lo(f[2 * q + 1], fl[2 * q + 1], mean, rstd, gf[2 * q + 1],
+                                                              bf[2 * q + 1])
+                                     << 16);
+                    } else {
+#pragma unroll
+                        for (int q = 0; q < 4; ++q)
+                            w4[q] = (uint32_t)ln_out_bf16(f[2 * q], mean, rstd, gf[2 * q], bf[2 * q]) |
+                                    ((uint32_t)ln_out_bf16(f[2 * q + 1], mean, rstd, gf[2 * q + 1], bf[2 * q + 1]) << 16);
+                    }
                     *reinterpret_cast<uint4 *>(xr + c * CH) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
                 } else {
                     float4 o;
-                    o.x = ln_out_f32(f[0], mean, rstd, gf[0], bf[0]);
-                    o.y = ln_out_f32(f[1], mean, rstd, gf[1], bf[1]);
-                    o.z = ln_out_f32(f[2], mean, rstd, gf[2], bf[2]);
-                    o.w = ln_out_f32(f[3], mean, rstd, gf[3], bf[3]);
+                    o.x = url ? ln_out_f32_lo(f[0], fl[0], mean, rstd, gf[0], bf[0]) : ln_out_f32(f[0], mean, rstd, gf[0], bf[0]);
+                    o.y = url ? ln_out_f32_lo(f[1], fl[1], mean, rstd, gf[1], bf[1]) : ln_out_f32(f[1], mean, rstd, gf[1], bf[1]);
+                    o.z = url ? ln_out_f32_lo(f[2], fl[2], mean, rstd, gf[2], bf[2]) : ln_out_f32(f[2], mean, rstd, gf[2], bf[2]);
+                    o.w = url ? ln_out_f32_lo(f[3], fl[3], mean, rstd, gf[3], bf[3]) : ln_out_f32(f[3], mean, rstd, gf[3], bf[3]);
                     *reinterpret_cast<float4 *>(xr + c * CH) = o;
                 }
             }
@@ -320,14 +370,67 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
         exit_gemm<T>(p, u_s, w_region, c0, dim, C, n_k, acc, acc2);
         exit_logits<T>(p, lg_s, bias_s, acc, acc2, s0, c0, B, C);
         if (p.out_mode == 1) {
-            // ---- hidden layer of an MLP head: GELU (erf form), rounded to the dtype -------
+            // ---- hidden layer of an MLP head: GELU, rounded to the dtype ----------------------
+            // GELU(a) = a (1 + erf(a / sqrt 2)) / 2 = a erfc(-a / sqrt 2) / 2; the erfc form is
+            // accurate in float for both signs.  bf16: a unit whose GELU lies within the error
+            // scale of the product above (kHidErr ||w_j|| ||u||, Cauchy-Schwarz on sum |w u|) plus
+            // that of the float evaluation of a bf16 rounding midpoint is evaluated again exactly:
+            // the dot product in float-float from exact bf16 x bf16 products, GELU in double.
+            __shared__ float wn2[2][kExitCT], un[kExitBT];
+            if constexpr (kBf16) {
+                {   // ||w_j||^2 of this tile's rows, two threads per row
+                    const int r = tid & (kExitCT - 1), h = tid / kExitCT;
+                    float acc = 0.0f;
+                    if (c0 + r < C) {
+                        const T *wr = reinterpret_cast<const T *>(p.head.weight) + (size_t)(c0 + r) * dim;
+                        for (int c = h; c < nchunk; c += 2) {
+                            float f[CH];
+                            chunk_to_f(ldg16(wr + c * CH), f);
+#pragma unroll
+                            for (int e = 0; e < CH; ++e) acc = fmaf(f[e], f[e], acc);
+                        }
+                    }
+                    wn2[h][r] = acc;
+                }
+                {   // ||u||^2 of each sample's row (warp -> sample slot)
+                    const T *ur = u_s + (size_t)warp * u_stride;
+                    float acc = 0.0f;
+                    for (int c = lane; c < nchunk; c += 32) {
+                        float f[CH];
+                        chunk_to_f(*reinterpret_cast<const uint4 *>(ur + c * CH), f);
+#pragma unroll
+                        for (int e = 0; e < CH; ++e) acc = fmaf(f[e], f[e], acc);
+                    }
+#pragma unroll
+                    for (int o = 16; o >= 1; o >>= 1) acc += __shfl_xor_sync(0xFFFFFFFFu, acc, o);
+                    if (lane == 0) un[warp] = sqrtf(acc);
+                }
+                __syncthreads();
+            }
             T *ho = reinterpret_cast<T *>(p.hidden_out);
             for (int it = tid; it < kExitBT * kExitCT; it += kExitThreads) {
                 const int sl = it / kExitCT, col = it - sl * kExitCT;
                 if (s0 + sl < B && c0 + col < C) {
                     const float a = lg_s[it];
-                    const float g = 0.5f * a * (1.0f + erff(a * 0.70710678118654752f));
-                    ho[(size_t)(s0 + sl) * C + c0 + col] = from_float<T>(g);
+                    const float g = 0.5f * a * erfcf(-a * 0.70710678118654752f);
+                    if constexpr (kBf16) {
+                        const float ea = kHidErr * sqrtf(1.0001f * (wn2[0][col] + wn2[1][col])) * un[sl] +
+                                         fabsf(a) * 0x1p-20f;
+                        const float eg = 1.13f * ea + fabsf(g) * 0x1p-16f;
+                        const float mid = __uint_as_float((__float_as_uint(g) & 0xFFFF0000u) | 0x8000u);
+                        uint16_t hb;
+                        if (isfinite(g) && fabsf(g - mid) > eg) {
+                            hb = __bfloat16_as_ushort(__float2bfloat16_rn(g));
+                        } else {
+                            hb = hidden_exact_bf16(reinterpret_cast<const __nv_bfloat16 *>(p.head.weight) +
+                                                       (size_t)(c0 + col) * dim,
+                                                   reinterpret_cast<const __nv_bfloat16 *>(u_s + (size_t)sl * u_stride),
+                                                   dim, p.head.bias[c0 + col]);
+                        }
+                        reinterpret_cast<uint16_t *>(ho)[(size_t)(s0 + sl) * C + c0 + col] = hb;
+                    } else {
+                        ho[(size_t)(s0 + sl) * C + c0 + col] = from_float<T>(g);
+                    }
                 }
             }
         } else {

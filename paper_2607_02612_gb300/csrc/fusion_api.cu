@@ -373,18 +373,37 @@ namespace {
 // fusion_exit_check_mlp scratch: the linear exit workspace for `classes`, then the pooled
 // rows [max_batch, dim] float32 and the hidden rows [max_batch, hidden] (float32 size).
 struct MlpWs {
-    size_t u, hid, lg, total;
+    size_t u, ulo, hid, lg, total;
 };
-// The stage's own scratch, the pooled rows (float32), the hidden rows (at most float32) and
-// the second layer's logits tiles (the general exit kernel writes exited rows from there).
+// The stage's own scratch, the pooled rows (float-float: high then low parts), the hidden rows
+// (at most float32) and the second layer's logits tiles (the general exit kernel writes exited
+// rows from there).
 MlpWs mlp_ws_layout(int32_t max_batch, int32_t dim, int32_t hidden, int32_t classes) {
     const size_t mb = (size_t)(max_batch > 0 ? max_batch : 1);
     const size_t tiles = (size_t)ceil_div(max_batch > 0 ? max_batch : 1, kExitBT) * kExitBT;
     MlpWs L;
     L.u = (ws_layout(max_batch, classes).total + 255) / 256 * 256;
-    L.hid = (L.u + mb * (size_t)dim * sizeof(float) + 255) / 256 * 256;
+    L.ulo = (L.u + mb * (size_t)dim * sizeof(float) + 255) / 256 * 256;
+    L.hid = (L.ulo + mb * (size_t)dim * sizeof(float) + 255) / 256 * 256;
     L.lg = (L.hid + mb * (size_t)hidden * sizeof(float) + 255) / 256 * 256;
     L.total = (L.lg + tiles * (size_t)classes * sizeof(float) + 255) / 256 * 256;
+    return L;
+}
+// fusion_stage_mlp with merging and the exit check: the MLP head's scratch, then the merged
+// batch (tokens at 4 bytes per element whatever the dtype, sizes, scores, input row of every
+// merged row, offsets) that the head reads and the compaction and pruning start from.
+struct StageMlpWs {
+    size_t x, sizes, scores, keep, offsets, total;
+};
+StageMlpWs stage_mlp_ws_layout(int32_t max_batch, int64_t max_rows, int32_t dim, int32_t hidden, int32_t classes) {
+    const size_t mr = (size_t)(max_rows > 0 ? max_rows : 1);
+    StageMlpWs L;
+    L.x = mlp_ws_layout(max_batch, dim, hidden, classes).total;
+    L.sizes = align256(L.x + mr * (size_t)dim * 4);
+    L.scores = align256(L.sizes + mr * 4);
+    L.keep = align256(L.scores + mr * 4);
+    L.offsets = align256(L.keep + mr * 4);
+    L.total = align256(L.offsets + (size_t)(max_batch > 0 ? max_batch + 1 : 1) * 4);
     return L;
 }
 }  // namespace
@@ -421,6 +440,7 @@ int launch_exit_mlp(int dtype, const fusion_ragged &in, const void *x, int32_t d
     pp.sizes = sizes;
     pp.pool = head.pool;
     pp.u_out = u;
+    pp.u_lo = reinterpret_cast<float *>(wb + L.ulo);
     pp.status = dev_status;
 
     ExitParams l1{};   // LayerNorm, first layer and GELU
@@ -434,6 +454,7 @@ int launch_exit_mlp(int dtype, const fusion_ragged &in, const void *x, int32_t d
     l1.status = dev_status;
     l1.in_mode = 2;
     l1.u_in = u;
+    l1.u_in_lo = reinterpret_cast<const float *>(wb + L.ulo);
     l1.out_mode = 1;
     l1.hidden_out = hid;
 
@@ -462,6 +483,13 @@ int launch_exit_mlp(int dtype, const fusion_ragged &in, const void *x, int32_t d
     return rc;
 }
 }  // namespace
+
+size_t fusion_stage_mlp_workspace_size(int32_t max_batch, int64_t max_rows, int32_t dim, int32_t hidden,
+                                       int32_t classes) {
+    return stage_mlp_ws_layout(max_batch < 0 ? 0 : max_batch, max_rows, dim < 16 ? 16 : dim, hidden < 16 ? 16 : hidden,
+                               classes < 1 ? 1 : classes)
+        .total;
+}
 
 size_t fusion_exit_mlp_workspace_size(int32_t max_batch, int32_t dim, int32_t hidden, int32_t classes) {
     if (max_batch < 0) max_batch = 0;
@@ -572,8 +600,9 @@ int stage_impl(int dtype, int flags, const fusion_ragged &in, const void *x, int
     }
     if (do_exit && mlp) {   // the MLP head's scratch, whose first part is the stage's own
         if (!workspace || !aligned16(workspace)) return FUSION_ERR_WORKSPACE;
-        if (workspace_bytes < mlp_ws_layout(in.max_batch, dim, mlp->hidden, mlp->classes).total)
-            return FUSION_ERR_WORKSPACE;
+        const size_t need = do_merge ? stage_mlp_ws_layout(in.max_batch, in.max_rows, dim, mlp->hidden, mlp->classes).total
+                                     : mlp_ws_layout(in.max_batch, dim, mlp->hidden, mlp->classes).total;
+        if (workspace_bytes < need) return FUSION_ERR_WORKSPACE;
     } else {
         FZ_TRY(check_workspace(workspace, workspace_bytes, in.max_batch, classes));
     }
@@ -597,6 +626,49 @@ int stage_impl(int dtype, int flags, const fusion_ragged &in, const void *x, int
     pa.slot = w.slot;
     pa.plan = w.plan;
     pa.status = dev_status;
+    if (do_exit && mlp && do_merge) {
+        // The MLP head reads the merged tokens (Sec. III-B): merge into the workspace, the exit
+        // check on that batch, then compaction and pruning from it (keep_idx mapped back to the
+        // input rows through the merge's row ids).
+        const StageMlpWs M = stage_mlp_ws_layout(in.max_batch, in.max_rows, dim, mlp->hidden, mlp->classes);
+        unsigned char *wb = static_cast<unsigned char *>(workspace);
+        void *x_m = wb + M.x;
+        float *sizes_m = reinterpret_cast<float *>(wb + M.sizes);
+        float *scores_m = scores ? reinterpret_cast<float *>(wb + M.scores) : nullptr;
+        int32_t *keep_m = reinterpret_cast<int32_t *>(wb + M.keep);
+        int32_t *offs_m = reinterpret_cast<int32_t *>(wb + M.offsets);
+        PlanArgs pm = pa;
+        pm.prune = 0;
+        pm.exit_mask = nullptr;
+        pm.offsets_out = offs_m;
+        pm.ids_out = nullptr;
+        pm.batch_out = nullptr;
+        if (!fuse_plan(in)) FZ_TRY(cuda_rc(launch_plan(pm, s)));
+        ImageParams q = image_params(in, x, dim, keys, key_dim, sizes, scores, r, nullptr, 1, 0, w, offs_m, x_m, sizes_m,
+                                     scores_m, keep_m, nullptr, a_match, dev_status, G);
+        q.fused_plan = fuse_plan(in);
+        q.plan_args = pm;
+        FZ_TRY(cuda_rc(launch_sample_kernel(dtype, q, G, s)));
+        fusion_ragged in_m = in;
+        in_m.offsets = offs_m;
+        FZ_TRY(launch_exit_mlp(dtype, in_m, x_m, dim, sizes_m, *mlp, exit_mask, logits, max_prob, workspace, dev_status,
+                               s, nullptr));
+        record(ev.mid, s);
+        PlanArgs pc = pa;
+        pc.in = dev(in_m);
+        pc.merge = 0;
+        if (!fuse_plan(in)) FZ_TRY(cuda_rc(launch_plan(pc, s)));
+        const ImageGeometry G2 = image_geometry(dtype, in.max_tokens, dim, 0);
+        if (!G2.ok) return FUSION_ERR_SHAPE;
+        ImageParams c = image_params(in_m, x_m, dim, nullptr, dim, sizes_m, scores_m, nullptr, rho, 0, do_prune, w,
+                                     offsets_out, x_out, sizes_out, scores_out, keep_idx, nullptr, nullptr, dev_status, G2);
+        c.keep_map = keep_m;
+        c.fused_plan = fuse_plan(in);
+        c.plan_args = pc;
+        const int rc = cuda_rc(launch_sample_kernel(dtype, c, G2, s));
+        record(ev.end, s);
+        return rc;
+    }
     if (do_exit && mlp) {
         FZ_TRY(launch_exit_mlp(dtype, in, x, dim, sizes, *mlp, exit_mask, logits, max_prob, workspace, dev_status, s,
                                nullptr));

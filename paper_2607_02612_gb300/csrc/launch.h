@@ -31,7 +31,8 @@ struct ExitParams {
     int in_mode;     // 0: CLS rows of the ragged batch x; 1: dense rows x[s] of [B, dim]; 2: dense float32 rows u_in[s]
     int skip_ln;     // 1: the rows enter the product as they are (no LayerNorm)
     int out_mode;    // 0: softmax maximum and exit rule; 1: GELU(W u + b) rounded to the dtype into hidden_out
-    const float *u_in;   // [max_batch, dim] for in_mode 2
+    const float *u_in;   // [max_batch, dim] for in_mode 2 (float-float high parts)
+    const float *u_in_lo;   // [max_batch, dim] their low parts
     void *hidden_out;    // [max_batch, classes] for out_mode 1
 };
 cudaError_t launch_exit(int dtype, const ExitParams &p, cudaStream_t s);
@@ -57,7 +58,8 @@ struct PoolParams {
     int dim;
     const float *sizes;
     int pool;        // FUSION_POOL_CLS or FUSION_POOL_SPATIAL
-    float *u_out;    // [max_batch, dim]
+    float *u_out;    // [max_batch, dim]: the pooled rows, float-float high parts
+    float *u_lo;     // [max_batch, dim]: their low parts
     int *status;
 };
 cudaError_t launch_head_pool(int dtype, const PoolParams &p, cudaStream_t s);
@@ -121,6 +123,7 @@ struct ImageParams {
     float *sizes_out;
     float *scores_out;
     int *keep_idx;
+    const int *keep_map;   // NULL, or the input row of every row of x (keep_idx = keep_map[row])
     int *dst_map;
     int *a_match;
     int *status;

@@ -40,4 +40,27 @@ __device__ __forceinline__ float ln_out_f32(float x, F2 mean, F2 rstd, float g, 
     return __fmaf_rn(__fmul_rn(d, rstd.hi), g, b);
 }
 
+// ln_out_bf16 / ln_out_f32 for a float-float input element x + xlo (|xlo| <= ulp(x) / 2).
+__device__ __forceinline__ uint16_t ln_out_bf16_lo(float x, float xlo, F2 mean, F2 rstd, float g, float b) {
+    const float d = __fadd_rn(__fsub_rn(__fsub_rn(x, mean.hi), mean.lo), xlo);
+    const float v = __fmul_rn(__fmul_rn(d, rstd.hi), g);
+    const float u = __fadd_rn(v, b);
+    const uint32_t low = __float_as_uint(u) & 0xFFFFu;
+    const uint32_t dist = low > 0x8000u ? low - 0x8000u : 0x8000u - low;
+    if (dist > 24u && fabsf(u) >= 0.5f * fabsf(v)) {
+        const uint32_t bits = __float_as_uint(u);
+        if ((bits & 0x7F800000u) == 0x7F800000u) return (uint16_t)((bits >> 16) | ((bits & 0x7FFFFFu) ? 0x40u : 0u));
+        return (uint16_t)((bits + (low > 0x8000u ? 0x8000u : 0u)) >> 16);
+    }
+    F2 dd = two_sum(x, -mean.hi);
+    dd.lo = __fadd_rn(__fsub_rn(dd.lo, mean.lo), xlo);
+    F2 t = f2_mul(quick_two_sum(dd.hi, dd.lo), rstd);
+    t = f2_mul(t, {g, 0.0f});
+    return f2_to_bf16_bits(f2_add_f(t, b));
+}
+__device__ __forceinline__ float ln_out_f32_lo(float x, float xlo, F2 mean, F2 rstd, float g, float b) {
+    const float d = __fadd_rn(__fsub_rn(__fsub_rn(x, mean.hi), mean.lo), xlo);
+    return __fmaf_rn(__fmul_rn(d, rstd.hi), g, b);
+}
+
 }  // namespace fz

@@ -679,7 +679,7 @@ __device__ void finish_write(const ImageParams &p, const SampleInfo &s, MetaPtrs
         const long long orow = (long long)out_start + o;
         p.sizes_out[orow] = m.msize[pos];
         if (p.scores_out) p.scores_out[orow] = m.mscore[pos];
-        if (p.keep_idx) p.keep_idx[orow] = start + pos;
+        if (p.keep_idx) p.keep_idx[orow] = p.keep_map ? p.keep_map[start + pos] : start + pos;
     }
     if (p.a_match)
         for (int pos = tid; pos < N; pos += NT)

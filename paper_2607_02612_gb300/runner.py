@@ -190,7 +190,8 @@ class Fusion:
     def mlp_workspace(self, b: DeviceBatch, head: "MlpHeadTensors"):
         """The zero-filled scratch of the MLP-head calls (it grows to the largest head seen;
         a Chain sizes it for all its stages before any graph capture)."""
-        nbytes = fb.fusion_exit_mlp_workspace_size(b.max_batch, b.dim, head.hidden, head.classes)
+        # the stage's size covers the exit check alone too (its layout starts with the same scratch)
+        nbytes = fb.fusion_stage_mlp_workspace_size(b.max_batch, b.max_rows, b.dim, head.hidden, head.classes)
         if self._mlp_ws is None or self._mlp_ws.numel() < nbytes:
             self._mlp_ws = torch.zeros(nbytes, dtype=torch.uint8, device=self.device)
         return self._mlp_ws, nbytes

@@ -1,14 +1,16 @@
 """The exit check with the paper's MLP exit heads (Sec. III-D, Eq. 6-7; SpatialPool head at
 block 8, CLS-only head at block 10, each a 2-layer MLP) on the GPU against the oracle.
 
-Tolerances follow from where the kernel's arithmetic differs from the oracle's double
-evaluation: the SpatialPool sum in float32 (relative error below N 2^-24), the float32
-accumulation of both products, and, for bf16, the rounding of the LayerNorm output and of
-the hidden layer, where a value within that error of a bf16 rounding boundary may round the
-other way (one bf16 ulp, 2^-8 relative, moving a logit by about |W2| 2^-8 |h|).  Logits:
-2e-2 (bf16) / 1e-4 (f32) of the row's largest magnitude; max_prob: 2e-3 / 1e-4 relative; an
-exit decision may differ only where |c - tau| is below that max_prob tolerance (counted and
-reported)."""
+Where the kernels' arithmetic differs from the oracle's double evaluation: the pool is summed
+in float-float (exact products, compensated sums) and the LayerNorm statistics too, so the bf16
+LayerNorm output rounds as the oracle's does (a float evaluation is kept only when it lies more
+than 24 float ulps from a bf16 rounding midpoint); the hidden layer's GELU is evaluated in
+float in the erfc form and a unit within the product's error scale of a bf16 midpoint is
+evaluated again exactly (float-float dot product, GELU in double), so the bf16 hidden units
+match; the two products accumulate in float32.  What remains is float32 accumulation and the
+softmax: logits within 1e-4 of the row's largest magnitude (both dtypes), max_prob within 1e-4
+relative, and exit decisions equal wherever the oracle's margin |c - tau| is at least 1e-6
+(closer ones are counted and reported)."""
 import os
 import sys
 
@@ -26,8 +28,8 @@ from workloads import POOL_CLS, POOL_SPATIAL, make_mlp_head, make_workload  # no
 
 pytestmark = pytest.mark.gpu
 
-TOL_LOGITS = {"f32": 1e-4, "bf16": 2e-2}
-TOL_MAXP = {"f32": 1e-4, "bf16": 2e-3}
+TOL_LOGITS = {"f32": 1e-4, "bf16": 1e-4}
+TOL_MAXP = {"f32": 1e-4, "bf16": 1e-4}
 
 
 def _run(b, head, batch=None, max_tokens=None):
@@ -49,7 +51,7 @@ def _compare(dtype, g, o, label, n=None):
     assert not np.any(g["logits"][:n][g["exit_mask"][:n] == 0]), (label, "logits written for samples that continue")
     pe = np.abs(g["max_prob"][:n].astype(np.float64) - o["max_prob"][:n]) / o["max_prob"][:n]
     assert pe.max() <= TOL_MAXP[dtype], (label, float(pe.max()))
-    near = o["exit_gap"][:n] < TOL_MAXP[dtype] * o["max_prob"][:n]
+    near = o["exit_gap"][:n] < P.NEAR_TIE
     diff = g["exit_mask"][:n] != o["exit_mask"][:n]
     assert not (diff & ~near).any(), (label, np.nonzero(diff & ~near)[0][:5])
     print(f"[{label}] {n} samples, {int(o['exit_mask'][:n].sum())} exit, logits rel err {e.max():.2e}, "

@@ -272,11 +272,12 @@ def test_pipeline_overlapped_steps(name, B):
     assert want[0]["batch"] != want[1]["batch"] or not np.array_equal(want[0]["ids"], want[1]["ids"])
 
 
-def _mlp_heads_at(w, placement, seed):
-    """Put MLP exit heads on the given exit stages ({stage index: pool}) and set each tau in
-    the widest gap of the oracle's max_prob values around the median at that stage's input,
-    so that about half its images exit and none sits at the threshold.  Returns the oracle's
-    chain."""
+def _mlp_heads_at(w, placement, seed, tau_mode="gap"):
+    """Put MLP exit heads on the given exit stages ({stage index: pool}) and set each tau from the
+    oracle's max_prob values of that stage's merged tokens (what the head reads, Sec. III-B):
+    "gap" puts tau in the widest gap around the median, so that about half the images exit and
+    none sits at the threshold; "drawn" draws tau uniformly between the 25th and 75th
+    percentiles with the seeded generator, wherever it falls.  Returns the oracle's chain."""
     from workloads import make_mlp_head
     b = w.batch
     rng = np.random.default_rng(seed)
@@ -286,10 +287,20 @@ def _mlp_heads_at(w, placement, seed):
         if si in placement:
             head = make_mlp_head(rng, placement[si], b.dim, 2 * b.dim, 1000, b.dtype)
             T = int(bb.offsets[-1])
-            mp = np.sort(oracle.exit_mlp(b.dtype, bb.offsets, bb.x[:T], bb.sizes[:T], head)["max_prob"])
-            lo = max(0, len(mp) // 2 - 5)
-            k = lo + int(np.argmax(np.diff(mp[lo:lo + 11])))
-            head.tau = float(np.float32(0.5 * (mp[k] + mp[k + 1])))
+            ids = np.arange(bb.batch, dtype=np.int32) if bb.ids is None else np.asarray(bb.ids, np.int32)
+            if spec.merge:
+                m = oracle.merge(b.dtype, bb.offsets, bb.x[:T], bb.keys[:T], bb.sizes[:T], bb.scores[:T],
+                                 spec.r[ids])
+                offs, xs, szs = m["offsets"], m["x"], m["sizes"]
+            else:
+                offs, xs, szs = bb.offsets, bb.x[:T], bb.sizes[:T]
+            mp = np.sort(oracle.exit_mlp(b.dtype, offs, xs, szs, head)["max_prob"])
+            if tau_mode == "gap":
+                lo = max(0, len(mp) // 2 - 5)
+                k = lo + int(np.argmax(np.diff(mp[lo:lo + 11])))
+                head.tau = float(np.float32(0.5 * (mp[k] + mp[k + 1])))
+            else:
+                head.tau = float(np.float32(rng.uniform(np.percentile(mp, 25), np.percentile(mp, 75))))
             spec.mlp_head = head
             spec.head = None
         res = oracle.stage(bb, spec)
@@ -298,14 +309,16 @@ def _mlp_heads_at(w, placement, seed):
     return outs
 
 
-@pytest.mark.parametrize("graph", [True, False])
-def test_chain_with_mlp_heads(graph):
+@pytest.mark.parametrize("graph,tau_mode", [(True, "gap"), (False, "gap"), (True, "drawn")])
+def test_chain_with_mlp_heads(graph, tau_mode):
     """The DeiT-S schedule with the paper's MLP exit heads inside the fused stage: SpatialPool
     at block 8, CLS-only at block 10 (the linear head at blocks 4 and 6); every stage against
-    the oracle, whose MLP exit check reads the stage input as the fused stage does."""
+    the oracle, whose MLP exit check reads the merged tokens as stored.  Exit decisions must
+    agree wherever the oracle's margin |c - tau| is at least 1e-6 (closer ones are counted); one
+    case draws tau from the generator instead of placing it in a gap."""
     from workloads import POOL_CLS, POOL_SPATIAL
     w = make_workload("deit_s_chain12_bf16_b256", batch=64)
-    o_outs = _mlp_heads_at(w, {7: POOL_SPATIAL, 9: POOL_CLS}, 21)
+    o_outs = _mlp_heads_at(w, {7: POOL_SPATIAL, 9: POOL_CLS}, 21, tau_mode)
     g_outs, status = P.chain_on_gpu(w, graph=graph)
     assert status == 0
     rep = P.Report()
@@ -314,17 +327,18 @@ def test_chain_with_mlp_heads(graph):
     for si in (7, 9):
         n = int(o_outs[si]["exit_mask"].sum())
         assert 0 < n < len(o_outs[si]["exit_mask"]), (si, n)
-    _report(rep, f"chain with MLP heads, graph={graph}")
+    _report(rep, f"chain with MLP heads, graph={graph}, tau {tau_mode}")
 
 
 @pytest.mark.parametrize("pool", [0, 1])
 def test_stage_mlp_f32(pool):
-    """One fused float32 stage (merge, MLP exit check, prune) on the 65-token schedule."""
+    """One fused float32 stage (merge, MLP exit check on the merged tokens, prune) on the
+    65-token schedule, tau drawn from the generator."""
     w = make_workload("ragged_b8192_n65_chain4_f32", batch=300, seed_offset=3)
     w = type(w)(w.spec, w.batch, w.stages[:1])
     w.stages[0].prune = True
     w.stages[0].rho = np.full(w.batch.batch, 0.7, np.float32)
-    o_outs = _mlp_heads_at(w, {0: pool}, 31 + pool)
+    o_outs = _mlp_heads_at(w, {0: pool}, 31 + pool, "drawn")
     g_outs, status = P.chain_on_gpu(w)
     assert status == 0
     rep = P.Report()

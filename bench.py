@@ -20,6 +20,11 @@ e2e       the same metric through the public C ABI with host buffers: pinned
           host -> device copy of the step's inputs, the chain, device -> host read
           of the results, all inside the timed region, through runner.Pipeline (two
           buffer slots, each step's input copy overlapping the previous step's kernels).
+cpu_baseline  the oracle on the host: one process per core, each on a seeded shard of the
+          workload (value, cores), and single-threaded on the whole batch (single_core).
+parity    the timed steps' outputs against that single-threaded oracle run: per stage batch
+          count, offsets, ids, exit masks and tokens (bf16 bit-exact), with the count of
+          decisions whose oracle margin is below 1e-6 (near_ties).
 side legs the merge router, the pruning router's scores, the MLP exit head, the
           size-aware attention, one full stage alone, and the schedule with the paper's
           MLP exit heads at blocks 8 and 10 (paper_heads).
@@ -247,19 +252,94 @@ def run_reference(args, world, rank):
     return 0
 
 
+def _oracle_shard(args):
+    """One process's share of the all-cores oracle run: the full schedule on its own seeded
+    shard of images of the workload (images are independent; compaction is per shard)."""
+    name, batch, seed_offset = args
+    import oracle
+    from workloads import make_workload
+    w = make_workload(name, batch=batch, seed_offset=seed_offset)
+    t0 = time.perf_counter()
+    res = oracle.chain(w)
+    dt = time.perf_counter() - t0
+    return batch + sum(int(r["n_out"]) for r in res[:-1]), dt
+
+
 def cpu_baseline(workload_name: str):
+    """The oracle on the host cores: single thread on the whole batch (its results also serve
+    the parity check of the bench's own outputs), then one process per core, each on its own
+    seeded shard of the same workload, started with spawn before any GPU work.  Returns the
+    cpu_baseline entry and the oracle's chain."""
+    import multiprocessing as mp
     import oracle
     from workloads import make_workload
     w = make_workload(workload_name)
-    n = min(w.batch.batch, 256)
-    sub = make_workload(workload_name, batch=n) if n != w.batch.batch else w
+    n = w.batch.batch
     t0 = time.perf_counter()
-    res = oracle.chain(sub)
+    res = oracle.chain(w)
     dt = time.perf_counter() - t0
     units = n + sum(int(r["n_out"]) for r in res[:-1])
-    return {"value": units / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{n} of {w.batch.batch} images, one full {len(w.stages)}-stage schedule "
-                      f"({dt:.1f} s, single thread)"}
+    one = {"value": units / dt, "unit": UNIT, "cores": 1,
+           "sample": f"all {n} images, one full {len(w.stages)}-stage schedule ({dt:.1f} s)"}
+    procs = max(1, os.cpu_count() or 1)
+    per = max(1, min(n, 2 * n // procs))   # about two single-thread runs' worth of work in total
+    ctx = mp.get_context("spawn")
+    with ctx.Pool(procs) as pool:
+        pool.map(_oracle_shard, [(workload_name, 1, 1000 + k) for k in range(procs)])   # workers up
+        t0 = time.perf_counter()
+        outs = pool.map(_oracle_shard, [(workload_name, per, 2000 + k) for k in range(procs)])
+        wall = time.perf_counter() - t0
+    units_all = sum(u for u, _ in outs)
+    entry = {"value": units_all / wall, "unit": UNIT, "cores": procs, "kind": "oracle",
+             "sample": f"{procs} processes x {per} images (seeded shards of the workload), full "
+                       f"{len(w.stages)}-stage schedule each, {wall:.1f} s wall",
+             "single_core": one}
+    return entry, res
+
+
+def parity_vs_oracle(chain, o_outs, dtype):
+    """The bench's own outputs against the oracle's chain on the same inputs: per stage the
+    batch count, offsets, ids and exit masks (bit-exact), tokens bit-exact (bf16) or within
+    1e-5 of the row's largest magnitude (f32), sizes exact; decisions whose oracle margin is
+    below 1e-6 are counted (argmax gap, top-r boundary gap, prune boundary gap, |c - tau|)."""
+    near = {"argmax": 0, "topr": 0, "prune": 0, "exit": 0}
+    mism, stages_checked = 0, 0
+    detail = []
+    for s, (g, o) in enumerate(zip(chain.outs, o_outs)):
+        near["argmax"] += int(np.sum(np.asarray(o["argmax_gap"]) < 1e-6))
+        near["topr"] += int(np.sum(np.asarray(o["topr_gap"]) < 1e-6))
+        near["prune"] += int(np.sum(np.asarray(o["prune_gap"]) < 1e-6))
+        near["exit"] += int(np.sum(np.asarray(o["exit_gap"]) < 1e-6))
+        nb = int(g["batch"].item())
+        ok = nb == int(o["n_out"])
+        if ok:
+            ok = (np.array_equal(g["offsets"][:nb + 1].cpu().numpy(), o["offsets"]) and
+                  np.array_equal(g["ids"][:nb].cpu().numpy(), o["ids"]))
+        if ok and g.get("exit_mask") is not None:
+            ok = np.array_equal(g["exit_mask"][:len(o["exit_mask"])].cpu().numpy(), o["exit_mask"])
+        if ok:
+            t = int(o["offsets"][-1])
+            ok = np.array_equal(g["sizes"][:t].cpu().numpy(), o["sizes"])
+            if dtype == "bf16":
+                gx = g["x"][:t].contiguous().view(torch_int16()).cpu().numpy().view(np.uint16)
+                ok = ok and np.array_equal(gx, o["x"])
+            else:
+                gx = g["x"][:t].float().cpu().numpy().astype(np.float64)
+                ox = np.asarray(o["x"], np.float64)
+                scale = np.maximum(np.abs(ox).max(axis=1, keepdims=True), 1e-30)
+                ok = ok and bool(np.all(np.abs(gx - ox) <= 1e-5 * scale))
+        stages_checked += 1
+        if not ok:
+            mism += 1
+            detail.append(s + 1)
+    return {"stages_checked": stages_checked, "mismatches": mism, "mismatched_stages": detail,
+            "near_ties": near, "rule": "indices and bf16 tokens bit-exact; decisions with an oracle "
+                                       "margin below 1e-6 counted, not excused"}
+
+
+def torch_int16():
+    import torch
+    return torch.int16
 
 
 def oracle_side_legs(b):
@@ -326,14 +406,14 @@ def main():
     lib = fz.load()
     assert lib is not None
 
-    # cpu baseline first (before any GPU work forks nothing; single thread)
-    cpu = None
+    # cpu baseline first, before any GPU work (its worker processes are spawned, not forked)
+    cpu, o_chain = None, None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(args.workload)
+        cpu, o_chain = cpu_baseline(args.workload)
 
     w = make_workload(args.workload, seed_offset=rank)
     b = w.batch
-    side_cpu = oracle_side_legs(b) if cpu is not None else {}
+    side_cpu = oracle_side_legs(b) if cpu is not None and args.workload == DEFAULT_WORKLOAD else {}
     specs = w.stages
     classes = max([s.head.classes for s in specs if s.head is not None] + [1])
     fus = runner.Fusion(b.batch, classes, dev)
@@ -412,6 +492,8 @@ def main():
     first_ms = np.array(first_rows)
     image_ms = stage_ms - first_ms
     clocks = clk.summary()
+    # the outputs of the timed steps against the oracle's chain on the same inputs
+    parity = parity_vs_oracle(chain, o_chain, b.dtype) if o_chain is not None else None
 
     # images entering each stage and algorithmic bytes, from the (deterministic) outputs
     in_off, in_ids = b.offsets, np.arange(b.batch, dtype=np.int32)
@@ -455,12 +537,14 @@ def main():
         full_stats = {"stages": [s + 1 for s in full],
                       "images_per_s": sum(per_stage[s]["images_in"] for s in full) * args.steps / t_full,
                       "achieved_gbs": b_full / t_full / 1e9, "frac": b_full / t_full / 1e9 / peak}
-    solo = run_solo_full_stage(args, fz, runner, w, b, dev, flush, peak) if full else None
-    router = run_router(args, fz, runner, b, dev, flush, peak)
-    scores = run_token_scores(args, fz, runner, b, dev, flush, peak)
-    exit_mlp = run_exit_mlp(args, fz, runner, b, dev, flush, peak)
-    attention = run_attention(args, fz, runner, b, dev, flush, peak)
-    paper_heads = run_paper_heads(args, fz, runner, w, chain, dev, flush)
+    # the side legs are defined on the DeiT-S batch; other workloads time their own schedule only
+    side = args.workload == DEFAULT_WORKLOAD
+    solo = run_solo_full_stage(args, fz, runner, w, b, dev, flush, peak) if full and side else None
+    router = run_router(args, fz, runner, b, dev, flush, peak) if side else None
+    scores = run_token_scores(args, fz, runner, b, dev, flush, peak) if side else None
+    exit_mlp = run_exit_mlp(args, fz, runner, b, dev, flush, peak) if side else None
+    attention = run_attention(args, fz, runner, b, dev, flush, peak) if side else None
+    paper_heads = run_paper_heads(args, fz, runner, w, chain, dev, flush) if side else None
     for name, leg in (("router", router), ("pruning_router", scores), ("exit_mlp", exit_mlp), ("attention", attention)):
         if name in side_cpu:
             leg["cpu_oracle"] = side_cpu[name]
@@ -483,6 +567,7 @@ def main():
                      "algorithmic_bytes_per_launch": bytes_image / S,
                      "whole_step_frac": step_achieved / peak},
         "cpu_baseline": cpu,
+        "parity": parity,
         "e2e": e2e,
         "gpu_launches": sum(1 + int(has_first[s]) for s in range(S)) * args.steps,
         "clocks": clocks,

@@ -270,42 +270,46 @@ __device__ __forceinline__ uint16_t f2_to_bf16_bits(F2 v) {
 }
 
 // ---------------------------------------------------------------------------
-// block-wide exclusive scan of v[0..n) in shared memory, n <= 2 * blockDim.x.
-// All threads must call; tmp needs 33 ints.  Returns the total.
+// block-wide exclusive scan of v[0..n) in shared memory, in chunks of 2 * blockDim.x
+// elements (one chunk for n <= 2 * blockDim.x).  All threads must call; tmp needs 33 ints.
+// Returns the total.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ int block_scan_excl(int *v, int n, int *tmp) {
     const int t = threadIdx.x;
     const int lane = t & 31, w = t >> 5, nw = (blockDim.x + 31) >> 5;
-    const int i0 = 2 * t, i1 = 2 * t + 1;
-    const int a = (i0 < n) ? v[i0] : 0;
-    const int b = (i1 < n) ? v[i1] : 0;
-    const int s = a + b;
-    int incl = s;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-        if (lane >= o) incl += y;
-    }
-    if (lane == 31) tmp[w] = incl;
-    __syncthreads();
-    if (w == 0) {
-        const int x = (lane < nw) ? tmp[lane] : 0;
-        int ix = x;
+    int base = 0;
+    for (int c0 = 0; c0 < n; c0 += 2 * (int)blockDim.x) {
+        const int i0 = c0 + 2 * t, i1 = i0 + 1;
+        const int a = (i0 < n) ? v[i0] : 0;
+        const int b = (i1 < n) ? v[i1] : 0;
+        const int s = a + b;
+        int incl = s;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(0xFFFFFFFFu, ix, o);
-            if (lane >= o) ix += y;
+            const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+            if (lane >= o) incl += y;
         }
-        if (lane < nw) tmp[lane] = ix - x;
-        if (lane == 31) tmp[32] = ix;
+        if (lane == 31) tmp[w] = incl;
+        __syncthreads();
+        if (w == 0) {
+            const int x = (lane < nw) ? tmp[lane] : 0;
+            int ix = x;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(0xFFFFFFFFu, ix, o);
+                if (lane >= o) ix += y;
+            }
+            if (lane < nw) tmp[lane] = ix - x;
+            if (lane == 31) tmp[32] = ix;
+        }
+        __syncthreads();
+        const int excl = base + tmp[w] + incl - s;
+        if (i0 < n) v[i0] = excl;
+        if (i1 < n) v[i1] = excl + a;
+        base += tmp[32];
+        __syncthreads();
     }
-    __syncthreads();
-    const int excl = tmp[w] + incl - s;
-    if (i0 < n) v[i0] = excl;
-    if (i1 < n) v[i1] = excl + a;
-    const int total = tmp[32];
-    __syncthreads();
-    return total;
+    return base;
 }
 
 // ceil(rho * P) with rho taken exactly, clamped to [0, P]; NaN keeps nothing; NaN and

@@ -299,10 +299,302 @@ __global__ void __launch_bounds__(kTcThreads, 2)
 }
 
 // ---------------------------------------------------------------------------
+// Samples whose halves exceed one tile (|A| or |B| above 128; ViT-L/16 at 384: 288 x 288 x
+// 1024): one CTA per SM, tensor memory of 256 or 512 columns.  Half A is taken in M-tiles of
+// 128 rows; half B in N-blocks of at most 256 columns, all of them held in tensor memory at once.
+// For every M-tile the K-blocks of (that tile's A rows, all B rows) stream by TMA through the
+// ring (stage q = M-tile q / n_kb, K-block q % n_kb); the B rows are loaded again for every
+// M-tile (from L2 after the first).  The tile's products accumulate over its K-blocks, its
+// epilogue keeps each A row's best column, and the next tile reuses the accumulators.  Row
+// norms: A rows of each tile and, during the first tile, the B rows, one thread per row.
+// ---------------------------------------------------------------------------
+constexpr int kTiledMaxStages = 8;
+
+__global__ void __launch_bounds__(kTcThreads, 1)
+    k_image_tc_tiled(const __grid_constant__ TcMaps maps, ImageParams p, TcGeometry g) {
+    extern __shared__ unsigned char sm_raw[];
+    unsigned char *sm = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~uintptr_t(1023));
+    __shared__ __align__(8) unsigned long long bar_full[kTiledMaxStages], bar_empty[kTiledMaxStages], bar_done, bar_drain;
+    __shared__ uint32_t tmem_base;
+    __shared__ int s_fail;
+    __shared__ unsigned long long half_best[kTcThreads / 2];
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(&tmem_base)),
+                     "r"(g.tmem_cols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    if (tid >= 32 && tid < 36) {
+        const CUtensorMap *mp = tid == 32 ? &maps.e32 : tid == 33 ? &maps.o32 : tid == 34 ? &maps.e8 : &maps.o8;
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(mp)) : "memory");
+    }
+    SampleInfo s;
+    if (!sample_begin<kTcThreads>(p, blockIdx.x, s)) {
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncthreads();
+        if (warp == 0)
+            asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(g.tmem_cols)
+                         : "memory");
+        return;
+    }
+    const bool dec = s.decide;
+    const int nkb = g.n_kb;
+    int issued = 0;   // stages issued (thread 0's count; warp 0 issues the first ones)
+    const int nM = (s.nA + 127) >> 7;               // M-tiles of half A
+    const int rowsB = (s.nB + 7) & ~7;
+    const int npad = (s.nB + 15) & ~15;             // columns of the product
+    const int nNB = (npad + 255) >> 8;              // N-blocks of at most 256 columns
+    // stage: [128 A rows][rowsB B rows] x 128 B; an MMA reads 128 A rows and up to npad B rows
+    const uint32_t aBytes = 128u * 128u;
+    const uint32_t kbs = aBytes + (uint32_t)rowsB * 128u;
+    const uint32_t reach = aBytes + (uint32_t)npad * 128u;
+    const int nq = nM * nkb;
+    int S = min(min(nq, kTiledMaxStages), (int)(g.stage_region / kbs));
+    while (S > 1 && (uint32_t)(S - 1) * kbs + reach > g.usable) --S;
+    const int yB = (s.start + 1) >> 1, yA0 = (s.start + 2) >> 1;
+    const bool oddA = (s.start + 2) & 1, oddB = (s.start + 1) & 1;
+    // boxes of stage q: the A rows of its M-tile (32-row boxes, then 8-row boxes), then all B rows
+    auto tile_rows = [&](int mt) { return min(128, s.nA - mt * 128); };
+    auto nboxes = [&](int n) { return (n >> 5) + (((n & 31) + 7) >> 3); };
+    auto stage_tx = [&](int mt) { return (uint32_t)(((tile_rows(mt) + 7) & ~7) + rowsB) * 128u; };
+    auto issue_box = [&](int q, int b) {
+        const int st = q % S, mt = q / nkb, kb = q - mt * nkb;
+        const int nA_t = tile_rows(mt);
+        const int nbA = nboxes(nA_t);
+        const bool half = b >= nbA;   // B rows
+        const int qq = half ? b - nbA : b;
+        const int n = half ? s.nB : nA_t;
+        const int n32 = n >> 5;
+        const bool big = qq < n32;
+        const int row0 = big ? qq * 32 : n32 * 32 + (qq - n32) * 8;
+        const bool odd = half ? oddB : oddA;
+        const CUtensorMap *map = big ? (odd ? &maps.o32 : &maps.e32) : (odd ? &maps.o8 : &maps.e8);
+        unsigned char *base = sm + (size_t)st * kbs + (half ? aBytes : 0u);
+        tma_load_2d(smem_addr(base + (size_t)row0 * 128), map, kb * 64, (half ? yB : yA0 + mt * 128) + row0,
+                    smem_addr(&bar_full[st]));
+    };
+    auto boxes_of = [&](int q) { return nboxes(tile_rows(q / nkb)) + nboxes(s.nB); };
+    auto produce = [&](int q) {
+        mbar_expect_tx(smem_addr(&bar_full[q % S]), stage_tx(q / nkb));
+        const int nb = boxes_of(q);
+        for (int b = 0; b < nb; ++b) issue_box(q, b);
+    };
+
+    MetaPtrs m(sm, meta_layout(p.in.max_tokens, g.meta_base));
+    meta_prefetch<kTcThreads>(p, s, m);
+    if (warp == 0) {
+        if (lane == 0) s_fail = 0;
+        if (dec) {
+            if (lane < S) {
+                mbar_init(smem_addr(&bar_full[lane]), 1);
+                mbar_init(smem_addr(&bar_empty[lane]), 1 + kTcThreads / 32);
+            }
+            if (lane == 31) mbar_init(smem_addr(&bar_done), 1);
+            if (lane == 30) mbar_init(smem_addr(&bar_drain), 1);
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            __syncwarp();
+            issued = min(S, nq);
+            for (int q = 0; q < min(S, nq); ++q) {   // each stage's boxes from all lanes
+                if (lane == 0) mbar_expect_tx(smem_addr(&bar_full[q]), stage_tx(q / nkb));
+                __syncwarp();
+                const int nb = boxes_of(q);
+                for (int b = lane; b < nb; b += 32) issue_box(q, b);
+            }
+        }
+    }
+    meta_init_rest<kTcThreads>(p, s, m);
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+
+    if (dec) {
+        const uint32_t tmem = tmem_base;
+        bool ok = true;
+        for (int mt = 0; mt < nM && ok; ++mt) {
+            const int nA_t = tile_rows(mt);
+            // norms: thread t < 128 owns A row t of this tile; during tile 0 threads 128.. own the
+            // B rows 128 apart
+            float ssA = 0.0f, scA = 0.0f;
+            float ssB[4] = {0.0f, 0.0f, 0.0f, 0.0f}, scB[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+            for (int kb = 0; kb < nkb; ++kb) {
+                const int q = mt * nkb + kb;
+                const int st = q % S;
+                const uint32_t par = (uint32_t)(q / S) & 1u;
+                if (!mbar_wait(smem_addr(&bar_full[st]), par)) {
+                    ok = false;
+                    break;
+                }
+                const unsigned char *stA = sm + (size_t)st * kbs, *stB = stA + aBytes;
+                if (tid == 32) {
+                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                    for (int nb = 0; nb < nNB; ++nb) {
+                        const int ncols = min(256, npad - nb * 256);
+                        const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(ncols >> 3) << 17) |
+                                               (8u << 24);
+                        const uint32_t a0 = smem_addr(stA), b0 = smem_addr(stB + (size_t)nb * 256 * 128);
+#pragma unroll
+                        for (int k = 0; k < 4; ++k)
+                            umma_bf16(tmem + (uint32_t)(nb * 256), sw128_desc(a0 + k * 32), sw128_desc(b0 + k * 32),
+                                      idesc, (kb | k) ? 1u : 0u);
+                    }
+                    umma_commit(smem_addr(&bar_empty[st]));
+                    if (kb == nkb - 1) umma_commit(smem_addr(&bar_done));
+                }
+                if (tid < 128) {
+                    if (tid < nA_t) {
+                        const unsigned char *rb = stA + tid * 128;
+#pragma unroll
+                        for (int j = 0; j < 8; ++j)
+                            neumaier_add(ssA, scA, chunk_sq(*reinterpret_cast<const uint4 *>(rb + ((j ^ (tid & 7)) << 4))));
+                    }
+                } else if (mt == 0) {
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const int br = tid - 128 + u * 128;
+                        if (br < s.nB) {
+                            const unsigned char *rb = stB + br * 128;
+#pragma unroll
+                            for (int j = 0; j < 8; ++j)
+                                neumaier_add(ssB[u], scB[u],
+                                             chunk_sq(*reinterpret_cast<const uint4 *>(rb + ((j ^ (br & 7)) << 4))));
+                        }
+                    }
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_addr(&bar_empty[st]));
+                if (tid == 0 && q + S < nq) {   // refill this stage (possibly with the next tile's K-block)
+                    if (!mbar_wait(smem_addr(&bar_empty[st]), par)) {
+                        ok = false;
+                        break;
+                    }
+                    produce(q + S);
+                    ++issued;
+                }
+            }
+            if (!ok) atomicOr(&s_fail, 1);
+            if (tid < nA_t) {
+                const float sq = __fadd_rn(ssA, scA);
+                if (!isfinite(sq)) raise_status(p.status, FUSION_DEV_NONFINITE);
+                m.inv_a[mt * 128 + tid] = 1.0f / fmaxf(sqrtf(sq), 1e-12f);
+            }
+            if (mt == 0 && tid >= 128) {
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int br = tid - 128 + u * 128;
+                    if (br < s.nB) {
+                        const float sq = __fadd_rn(ssB[u], scB[u]);
+                        if (!isfinite(sq)) raise_status(p.status, FUSION_DEV_NONFINITE);
+                        m.inv_b[br] = 1.0f / fmaxf(sqrtf(sq), 1e-12f);
+                    }
+                }
+            }
+            __syncthreads();
+            const bool mma_ok = s_fail == 0 && mbar_wait(smem_addr(&bar_done), (uint32_t)mt & 1u);
+            if (!mma_ok) atomicOr(&s_fail, 2);
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            __syncthreads();
+            if (s_fail != 0) {
+                ok = false;
+                break;
+            }
+            // epilogue of the tile: thread -> A row (tid % 128); the warpgroups split the columns
+            const int wg = tid >> 7, r = tid & 127;
+            const int half_cols = ((npad / 16 + 1) / 2) * 16;
+            const int c_lo = wg ? half_cols : 0, c_hi = wg ? npad : half_cols;
+            const uint32_t lane_addr = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+            const int arow = mt * 128 + r;
+            const float ia = r < nA_t ? m.inv_a[arow] : 0.0f;
+            unsigned long long bk = 0ull;
+            for (int c0 = c_lo; c0 < c_hi; c0 += 16) {
+                uint32_t v[16];
+                tmem_ld16(lane_addr + (uint32_t)c0, v);
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    const int col = c0 + e;
+                    if (r < nA_t && col < s.nB) {
+                        const float cs = (__uint_as_float(v[e]) * ia) * m.inv_b[col];
+                        const unsigned long long k = rank_key(cs, col);
+                        bk = k > bk ? k : bk;
+                    }
+                }
+            }
+            if (wg == 1) half_best[r] = bk;
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncthreads();   // the next tile's products overwrite the accumulators after this
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            if (wg == 0 && r < nA_t) {
+                const unsigned long long o = half_best[r];
+                m.best[arow] = o > bk ? o : bk;
+            }
+            __syncthreads();   // half_best is reused by the next tile
+        }
+        if (s_fail != 0) {
+            // a wait gave up: let the copies and products in flight land (bounded) before the
+            // shared and tensor memory are released
+            if (tid == 0) {
+                raise_status(p.status, FUSION_DEV_TIMEOUT);
+                for (int q = max(0, issued - S); q < issued; ++q)
+                    (void)mbar_wait(smem_addr(&bar_full[q % S]), (uint32_t)(q / S) & 1u);
+            }
+            if (tid == 32) {
+                umma_commit(smem_addr(&bar_drain));
+                (void)mbar_wait(smem_addr(&bar_drain), 0u);
+            }
+        } else {
+            select_top_r<kTcThreads>(s, m);
+        }
+        __syncthreads();
+    }
+    if (s_fail == 0) {
+        const GlobalLoader<__nv_bfloat16> gl{reinterpret_cast<const __nv_bfloat16 *>(p.x), (long long)s.start, p.dim};
+        finish_sample<__nv_bfloat16, kTcThreads>(p, s, m, gl);
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(g.tmem_cols)
+                     : "memory");
+}
+
+// ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
 int ceil8(int v) { return (v + 7) & ~7; }
 
+}  // namespace
+
+namespace {
+// Geometry of k_image_tc_tiled: one CTA per SM, a ring of [128 A rows | all B rows] stages.
+TcGeometry tiled_geometry(int max_tokens, int kdim) {
+    TcGeometry g{};
+    const int nBmax = max_tokens / 2;
+    const int npad_max = (nBmax + 15) & ~15;
+    g.tiled = 1;
+    g.n_kb = kdim / 64;
+    g.tmem_cols = npad_max <= 256 ? 256 : 512;
+    g.kb_a = 128u * 128u;
+    g.kb_b = (uint32_t)ceil8(nBmax) * 128u;
+    const size_t per_stage = g.kb_a + g.kb_b;
+    const size_t reach = g.kb_a + (size_t)npad_max * 128;
+    const size_t budget = 227 * 1024 - 4096;   // room for static shared memory
+    auto need = [&](int S) {
+        const size_t meta_base = (size_t)S * per_stage + 2048;
+        return std::max(meta_layout(max_tokens, meta_base).total, (size_t)(S - 1) * per_stage + reach);
+    };
+    int S = kTiledMaxStages;
+    while (S > 2 && need(S) + 1024 > budget) --S;
+    if (need(S) + 1024 > budget) return TcGeometry{};
+    g.stages = S;
+    g.stage_region = (uint32_t)(S * per_stage);
+    g.meta_base = (uint32_t)(S * per_stage + 2048);
+    g.usable = (uint32_t)need(S);
+    g.smem = g.usable + 1024;
+    g.ok = 1;
+    return g;
+}
 }  // namespace
 
 TcGeometry image_tc_geometry(int dtype, int max_tokens, int kdim, long long max_rows, int do_merge,
@@ -310,7 +602,7 @@ TcGeometry image_tc_geometry(int dtype, int max_tokens, int kdim, long long max_
     TcGeometry g{};
     if (dtype != FUSION_BF16 || !do_merge || kdim % 64 != 0 || max_rows < 2) return g;
     const int nAmax = (max_tokens - 1) / 2, nBmax = max_tokens / 2;
-    if (nAmax > 128 || nBmax > 128) return g;
+    if (nAmax > 128 || nBmax > 128) return tiled_geometry(max_tokens, kdim);
     g.n_kb = kdim / 64;
     g.kb_a = (uint32_t)ceil8(nAmax > 0 ? nAmax : 1) * 128u;
     g.kb_b = (uint32_t)ceil8(nBmax > 0 ? nBmax : 1) * 128u;
@@ -359,12 +651,13 @@ cudaError_t launch_image_tc(const ImageParams &p, const TcGeometry &g, cudaStrea
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
     }
-    cudaError_t e = cudaFuncSetAttribute(k_image_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)g.smem);
+    auto kernel = g.tiled ? k_image_tc_tiled : k_image_tc;
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)g.smem);
     if (e != cudaSuccess) return e;
     // the largest shared-memory carveout, so that both CTAs of an SM are resident from the start
-    e = cudaFuncSetAttribute(k_image_tc, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     if (e != cudaSuccess) return e;
-    k_image_tc<<<p.in.max_batch, kTcThreads, g.smem, s>>>(maps, p, g);
+    kernel<<<p.in.max_batch, kTcThreads, g.smem, s>>>(maps, p, g);
     return cudaGetLastError();
 }
 

@@ -150,6 +150,7 @@ cudaError_t launch_image(int dtype, const ImageParams &p, size_t smem, cudaStrea
 // ---- per-sample kernel on TMA + tcgen05 (bf16, |A|, |B| <= 128, key width % 64 == 0) ----
 struct TcGeometry {
     int ok;
+    int tiled;         // halves beyond one tile: k_image_tc_tiled (M-tiles of 128 A rows, one CTA per SM)
     int n_kb;          // key K-blocks of 64 dims
     int stages;        // K-block stages of a sample of max_tokens tokens (more for smaller samples)
     int tmem_cols;     // tensor-memory columns allocated per CTA

@@ -158,6 +158,18 @@ const char *fusion_version(void);
 int fusion_profile_next(void *start, void *mid, void *end);
 
 /*
+ * Launch gate (a failure-detection aid; no counterpart in the paper): while a gate is set,
+ * the per-sample kernels of the merge, prune, compact and stage calls made afterwards from
+ * the calling host thread wait, before reading any input, until the device int32 *flag is
+ * nonzero, polling it at most `polls` more times after the first read (each poll takes
+ * about 0.1 to 1 microsecond).  A CTA that gives up raises FUSION_DEV_TIMEOUT and writes no
+ * output (nothing asynchronous is in flight at that point).  A caller can launch work ahead
+ * of a producer that sets the flag; a test can check that a wait runs out.  flag NULL clears
+ * the gate.  Returns FUSION_ERR_INVALID_ARG for polls < 0 with a flag, else FUSION_OK.
+ */
+int fusion_set_launch_gate(const int32_t *flag, int64_t polls);
+
+/*
  * Bytes of scratch device memory every call needs for a batch bound of
  * max_batch samples and an exit head of `classes` classes (pass the largest
  * head used with this workspace; 1 when no exit check is run).  The workspace

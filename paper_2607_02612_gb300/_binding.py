@@ -46,7 +46,7 @@ EXPORTED = ("fusion_status_string", "fusion_version", "fusion_profile_next", "fu
             "fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune", "fusion_compact",
             "fusion_stage", "fusion_merge_router", "fusion_token_scores", "fusion_exit_mlp_workspace_size",
             "fusion_exit_check_mlp", "fusion_attention", "fusion_stage_mlp",
-            "fusion_stage_mlp_workspace_size")
+            "fusion_stage_mlp_workspace_size", "fusion_set_launch_gate")
 
 
 class FusionError(RuntimeError):
@@ -98,6 +98,8 @@ def load(path: Optional[str] = None):
     lib.fusion_version.restype = ctypes.c_char_p
     lib.fusion_profile_next.argtypes = [V, V, V]
     lib.fusion_profile_next.restype = ctypes.c_int
+    lib.fusion_set_launch_gate.argtypes = [V, I64]
+    lib.fusion_set_launch_gate.restype = ctypes.c_int
     lib.fusion_workspace_size.argtypes = [I32, I32]
     lib.fusion_workspace_size.restype = SZ
     lib.fusion_merge.argtypes = [ctypes.c_int, R, V, I32, V, I32, V, V, V, V, V, V, V, V, V, V, V, SZ, V, V]
@@ -121,7 +123,7 @@ def load(path: Optional[str] = None):
     for name in ("fusion_merge", "fusion_exit_check", "fusion_exit_check_noalloc", "fusion_prune",
                  "fusion_compact", "fusion_stage", "fusion_merge_router", "fusion_token_scores",
                  "fusion_exit_check_mlp", "fusion_attention", "fusion_stage_mlp",
-            "fusion_stage_mlp_workspace_size"):
+            "fusion_stage_mlp_workspace_size", "fusion_set_launch_gate"):
         getattr(lib, name).restype = ctypes.c_int
     del I64, F
     if path is None:
@@ -195,6 +197,12 @@ def _event(e) -> Optional[int]:
 def fusion_profile_next(start=None, mid=None, end=None) -> int:
     """Arm the next call of this thread to record torch.cuda.Event objects around its kernels."""
     return load().fusion_profile_next(_event(start), _event(mid), _event(end))
+
+
+def fusion_set_launch_gate(flag=None, polls: int = 0) -> int:
+    """Make the following calls' per-sample kernels wait (bounded) for a device int32 flag to
+    become nonzero; flag None clears the gate."""
+    return int(load().fusion_set_launch_gate(_ptr(flag), int(polls)))
 
 
 def fusion_workspace_size(max_batch: int, classes: int) -> int:

@@ -79,6 +79,10 @@ struct ProfileEvents {
 };
 thread_local ProfileEvents g_profile;
 
+// Launch gate armed by fusion_set_launch_gate() for this host thread's calls.
+thread_local const int32_t *g_gate = nullptr;
+thread_local unsigned g_gate_spins = 0;
+
 // Takes the armed events (if any) for the call that is starting.
 ProfileEvents take_profile() {
     ProfileEvents e = g_profile;
@@ -130,6 +134,8 @@ ImageParams image_params(const fusion_ragged &in, const void *x, int32_t dim, co
     p.sizes_out = sizes_out;
     p.scores_out = scores_out;
     p.keep_idx = keep_idx;
+    p.gate = g_gate;
+    p.gate_spins = g_gate_spins;
     p.dst_map = dst_map;
     p.a_match = a_match;
     p.status = status;
@@ -162,6 +168,13 @@ cudaError_t launch_sample_kernel(int dtype, const ImageParams &p, const ImageGeo
 extern "C" {
 
 const char *fusion_version(void) { return kVersion; }
+
+int fusion_set_launch_gate(const int32_t *flag, int64_t polls) {
+    if (flag && polls < 0) return FUSION_ERR_INVALID_ARG;
+    g_gate = flag;
+    g_gate_spins = flag ? (polls > (int64_t)0xFFFFFFFF ? 0xFFFFFFFFu : (unsigned)polls) : 0u;
+    return FUSION_OK;
+}
 
 int fusion_profile_next(void *start, void *mid, void *end) {
     g_profile.start = static_cast<cudaEvent_t>(start);

@@ -123,6 +123,8 @@ struct ImageParams {
     float *sizes_out;
     float *scores_out;
     int *keep_idx;
+    const int *gate;        // NULL, or a device flag to wait for (bounded) before reading any input
+    unsigned gate_spins;    // polls of that wait
     const int *keep_map;   // NULL, or the input row of every row of x (keep_idx = keep_map[row])
     int *dst_map;
     int *a_match;

@@ -239,9 +239,38 @@ __device__ bool sample_plan(const ImageParams &p, int i, SampleInfo &s) {
     return true;
 }
 
-// Either the fused plan or the plan kernel's results.
+// The launch gate (fusion_set_launch_gate): thread 0 polls the flag, at most `spins` more
+// times after the first read, and the CTA learns the result through shared memory.  Called
+// before any load of the call's inputs and before any asynchronous copy, so a CTA that gives up
+// has nothing in flight.
+__device__ __forceinline__ bool gate_open(const int *gate, unsigned spins) {
+    __shared__ int s_open;
+    if (threadIdx.x == 0) {
+        int ok = 0;
+        for (unsigned it = 0;; ++it) {
+            int v;
+            asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(gate) : "memory");
+            if (v != 0) {
+                ok = 1;
+                break;
+            }
+            if (it >= spins) break;
+            __nanosleep(128);
+        }
+        s_open = ok;
+    }
+    __syncthreads();
+    return s_open != 0;
+}
+
+// Either the fused plan or the plan kernel's results, once the launch gate (if any) is open;
+// a CTA whose gate wait gives up raises FUSION_DEV_TIMEOUT and writes nothing.
 template <int NT>
 __device__ __forceinline__ bool sample_begin(const ImageParams &p, int i, SampleInfo &s) {
+    if (p.gate && !gate_open(p.gate, p.gate_spins)) {
+        if (threadIdx.x == 0) raise_status(p.status, FUSION_DEV_TIMEOUT);
+        return false;
+    }
     return p.fused_plan ? sample_plan<NT>(p, i, s) : sample_info(p, i, s);
 }
 

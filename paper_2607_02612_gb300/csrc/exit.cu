@@ -64,7 +64,7 @@ struct ExitSmem {
     static __host__ __device__ size_t u_bytes(int dim) { return ((size_t)16 * u_stride(dim) * EB + 15) / 16 * 16; }
     static __host__ __device__ size_t total(int dim) {
         size_t t = u_bytes(dim) + 2 * w_stage + kExitCT * sizeof(float);
-        const size_t plan = (4 * kExitThreads + 40) * sizeof(int);
+        const size_t plan = plan_smem_bytes(kExitThreads);
         return t > plan ? t : plan;
     }
 };
@@ -566,7 +566,7 @@ struct ExitClSmem {
     static __host__ __device__ size_t flag_off(int dim) { return red_off(dim) + (size_t)(kExitThreads / 32) * 8 * sizeof(float); }
     static __host__ __device__ size_t total(int dim) {
         const size_t t = flag_off(dim) + (size_t)BT * sizeof(int);
-        const size_t plan = w_off(dim) + (4 * kExitThreads + 40) * sizeof(int);   // run_plan reuses the W stages
+        const size_t plan = w_off(dim) + plan_smem_bytes(kExitThreads);   // run_plan reuses the W stages
         return (t > plan ? t : plan) + (kTc ? 1024 : 0);
     }
 };
@@ -1015,7 +1015,7 @@ __global__ void __launch_bounds__(kPlanThreads) k_plan(PlanArgs a) {
 }  // namespace
 
 cudaError_t launch_plan(const PlanArgs &a, cudaStream_t s) {
-    const size_t smem = (4 * kPlanThreads + 40) * sizeof(int);
+    const size_t smem = plan_smem_bytes(kPlanThreads);
     k_plan<<<1, kPlanThreads, smem, s>>>(a);
     return cudaGetLastError();
 }

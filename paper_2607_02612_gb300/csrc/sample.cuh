@@ -447,16 +447,17 @@ struct MergedItem {
     uint4 self, av[kSrcU];
 };
 
+// Item t of the merged chunks [c_lo, c_lo + w) of every merged row.
 template <typename Loader>
-__device__ __forceinline__ void merged_fetch(const MetaPtrs &m, int t, int n_items, int ncx, const Loader &load,
+__device__ __forceinline__ void merged_fetch(const MetaPtrs &m, int t, int n_items, int w, int c_lo, const Loader &load,
                                              MergedItem &it) {
     it.pos = -1;
     if (t >= n_items) return;
-    const int k = t / ncx;
+    const int k = t / w;
     const int pos = 1 + 2 * m.mlist[k];
     if (!m.kflag[pos]) return;   // pruned after merging
     it.pos = pos;
-    it.c = t - k * ncx;
+    it.c = c_lo + t - k * w;
     const int n = (pos - 1) >> 1;
     it.q0 = m.scnt[n];
     it.q1 = m.scnt[n + 1];
@@ -691,16 +692,12 @@ __device__ bool finish_decide(const ImageParams &p, const SampleInfo &s, MetaPtr
     return true;
 }
 
-// The outputs of a decided sample (after finish_decide): index outputs, copied token rows
-// and merged token rows at s.out_start.  `load(pos, c)` returns the 16-byte chunk c of
-// input token pos.
-template <typename T, int NT, typename Loader>
-__device__ void finish_write(const ImageParams &p, const SampleInfo &s, MetaPtrs &m, const Loader &load) {
-    constexpr int CH = Elem<T>::kPerChunk;
+// Index outputs of a decided sample (after finish_decide): sizes, scores and input row of every
+// output row at s.out_start, and the match / destination maps when requested.
+template <int NT>
+__device__ void write_index_outputs(const ImageParams &p, const SampleInfo &s, MetaPtrs &m) {
     const int tid = threadIdx.x;
     const int N = s.N;
-
-    // index outputs
     const int start = s.start, out_start = s.out_start, out_n = s.out_n;
     for (int o = tid; o < out_n; o += NT) {
         const int sp = m.srcpos[o];
@@ -719,28 +716,38 @@ __device__ void finish_write(const ImageParams &p, const SampleInfo &s, MetaPtrs
             const int dest = gone ? 1 + 2 * m.match[(pos - 2) / 2] : pos;
             p.dst_map[start + pos] = out_start + m.opos[dest];
         }
+}
 
-    // copied token rows, 16 bytes per thread and kGatherU chunks in flight; (o, c) walks
-    // the output rows chunk by chunk without a division per step
+// The token rows of a decided sample, 16-byte chunks [c_lo, c_hi) of every output row: copied
+// rows with kGatherU chunks in flight per thread ((o, c) walks the rows chunk by chunk without
+// a division per step), then the merged rows' size-weighted means with the next item's loads
+// in flight.  `load(pos, c)` returns chunk c of input token pos.
+template <typename T, int NT, typename Loader>
+__device__ void write_rows(const ImageParams &p, const SampleInfo &s, MetaPtrs &m, const Loader &load, int c_lo,
+                           int c_hi) {
+    constexpr int CH = Elem<T>::kPerChunk;
     constexpr int kGatherU = kGatherChunks / NT;
-    const int dim = p.dim, ncx = dim / CH;
-    const int ostep = NT / ncx, cstep = NT - ostep * ncx;
-    T *xo = reinterpret_cast<T *>(p.x_out) + (long long)out_start * dim;
-    const int n_items = m.tmp[kMergedCount] * ncx;   // merged chunks
+    const int tid = threadIdx.x;
+    const int out_n = s.out_n;
+    const int dim = p.dim, w = c_hi - c_lo;
+    if (w <= 0) return;
+    const int ostep = NT / w, cstep = NT - ostep * w;
+    T *xo = reinterpret_cast<T *>(p.x_out) + (long long)s.out_start * dim;
+    const int n_items = m.tmp[kMergedCount] * w;   // merged chunks of the range
     MergedItem cur;
-    merged_fetch(m, tid, n_items, ncx, load, cur);   // lands while the copies run
-    int o = tid / ncx, c = tid - (tid / ncx) * ncx;
+    merged_fetch(m, tid, n_items, w, c_lo, load, cur);   // lands while the copies run
+    int o = tid / w, c = tid - (tid / w) * w;
     while (o < out_n) {
         int src[kGatherU], cc[kGatherU], dst[kGatherU];
 #pragma unroll
         for (int u = 0; u < kGatherU; ++u) {
             src[u] = o < out_n ? m.srcpos[o] : -1;   // < 0: merged row or past the end
-            cc[u] = c;
-            dst[u] = o * dim + c * CH;
+            cc[u] = c_lo + c;
+            dst[u] = o * dim + (c_lo + c) * CH;
             o += ostep;
             c += cstep;
-            if (c >= ncx) {
-                c -= ncx;
+            if (c >= w) {
+                c -= w;
                 ++o;
             }
         }
@@ -752,15 +759,20 @@ __device__ void finish_write(const ImageParams &p, const SampleInfo &s, MetaPtrs
         for (int u = 0; u < kGatherU; ++u)
             if (src[u] >= 0) *reinterpret_cast<uint4 *>(xo + dst[u]) = v[u];
     }
-
-    // merged token rows: the size-weighted means, the next item's loads in flight
     for (int t = tid; t < n_items; t += NT) {
         MergedItem nxt;
-        merged_fetch(m, t + NT, n_items, ncx, load, nxt);
+        merged_fetch(m, t + NT, n_items, w, c_lo, load, nxt);
         if (cur.pos >= 0)
             *reinterpret_cast<uint4 *>(xo + m.opos[cur.pos] * dim + cur.c * CH) = merged_value<T>(m, cur, load);
         cur = nxt;
     }
+}
+
+// The outputs of a decided sample (after finish_decide) at s.out_start.
+template <typename T, int NT, typename Loader>
+__device__ void finish_write(const ImageParams &p, const SampleInfo &s, MetaPtrs &m, const Loader &load) {
+    write_index_outputs<NT>(p, s, m);
+    write_rows<T, NT>(p, s, m, load, 0, p.dim / Elem<T>::kPerChunk);
 }
 
 // finish_decide then finish_write (the plan's output offsets already known).

@@ -181,22 +181,31 @@ __device__ __forceinline__ void exit_logits(const ExitParams &p, float *lg_s, co
 
 // Error scale of a hidden unit's pre-activation from the product above (bf16 mma.sync,
 // float32 sums flushed every 64 dims): about sqrt(30) roundings of at most 2^-24 relative to
-// partial sums bounded by sum |w u| <= ||w|| ||u||, with a safety factor of 8.
-constexpr float kHidErr = 0x1p-19f;
+// partial sums bounded by sum |w u| <= ||w|| ||u||; the typical partial sum is far below that
+// bound, so 2^-22 ||w|| ||u|| is more than 8 standard deviations of the accumulated error.
+constexpr float kHidErr = 0x1p-22f;
 
-// A hidden unit exactly: a = w . u + b1 from exact bf16 x bf16 products summed in float-float,
-// then GELU in double in the erf form, rounded once to bf16.
-static __device__ __noinline__ uint16_t hidden_exact_bf16(const __nv_bfloat16 *w, const __nv_bfloat16 *u, int dim,
-                                                          float b1) {
+// One hidden unit exactly, by a whole warp: a = w . u + b1 from exact bf16 x bf16 products
+// summed in float-float (each lane a slice of the dims, then a butterfly), GELU in double in the
+// erf form, rounded once to bf16.  Every lane returns the result.
+__device__ __forceinline__ uint16_t hidden_exact_bf16_warp(const __nv_bfloat16 *w, const __nv_bfloat16 *u, int dim,
+                                                           float b1) {
+    const int lane = threadIdx.x & 31;
     F2 acc = {0.0f, 0.0f};
-    for (int c = 0; c < dim; c += 8) {
+    for (int c = lane * 8; c < dim; c += 256) {
         float wf[8], uf[8];
         chunk_to_f(ldg16(w + c), wf);
         chunk_to_f(*reinterpret_cast<const uint4 *>(u + c), uf);
 #pragma unroll
         for (int e = 0; e < 8; ++e) acc = f2_add_f(acc, __fmul_rn(wf[e], uf[e]));
     }
-    acc = f2_add_f(acc, b1);
+    acc = f2_add_f(warp_sum_f2(acc), b1);
+    // with the product exact, the float GELU of its high part is within about a hundred float
+    // ulps of the exact value (erfc's error, amplified by its argument for large |a|); only a
+    // unit closer than that to a bf16 midpoint needs double precision
+    const float g2 = 0.5f * acc.hi * erfcf(-acc.hi * 0.70710678118654752f);
+    const float mid = __uint_as_float((__float_as_uint(g2) & 0xFFFF0000u) | 0x8000u);
+    if (isfinite(g2) && fabsf(g2 - mid) > fabsf(g2) * 0x1p-17f) return __bfloat16_as_ushort(__float2bfloat16_rn(g2));
     const double a = (double)acc.hi + (double)acc.lo;
     const double g = 0.5 * a * (1.0 + erf(a / sqrt(2.0)));
     return __bfloat16_as_ushort(__double2bfloat16(g));
@@ -408,29 +417,31 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
                 __syncthreads();
             }
             T *ho = reinterpret_cast<T *>(p.hidden_out);
+            // every warp takes 32 consecutive units of one sample slot per round (uniform trip count)
             for (int it = tid; it < kExitBT * kExitCT; it += kExitThreads) {
                 const int sl = it / kExitCT, col = it - sl * kExitCT;
-                if (s0 + sl < B && c0 + col < C) {
-                    const float a = lg_s[it];
-                    const float g = 0.5f * a * erfcf(-a * 0.70710678118654752f);
-                    if constexpr (kBf16) {
-                        const float ea = kHidErr * sqrtf(1.0001f * (wn2[0][col] + wn2[1][col])) * un[sl] +
-                                         fabsf(a) * 0x1p-20f;
-                        const float eg = 1.13f * ea + fabsf(g) * 0x1p-16f;
-                        const float mid = __uint_as_float((__float_as_uint(g) & 0xFFFF0000u) | 0x8000u);
-                        uint16_t hb;
-                        if (isfinite(g) && fabsf(g - mid) > eg) {
-                            hb = __bfloat16_as_ushort(__float2bfloat16_rn(g));
-                        } else {
-                            hb = hidden_exact_bf16(reinterpret_cast<const __nv_bfloat16 *>(p.head.weight) +
-                                                       (size_t)(c0 + col) * dim,
-                                                   reinterpret_cast<const __nv_bfloat16 *>(u_s + (size_t)sl * u_stride),
-                                                   dim, p.head.bias[c0 + col]);
-                        }
-                        reinterpret_cast<uint16_t *>(ho)[(size_t)(s0 + sl) * C + c0 + col] = hb;
-                    } else {
-                        ho[(size_t)(s0 + sl) * C + c0 + col] = from_float<T>(g);
+                const bool valid = s0 + sl < B && c0 + col < C;
+                const float a = lg_s[it];
+                const float g = 0.5f * a * erfcf(-a * 0.70710678118654752f);
+                if constexpr (kBf16) {
+                    const float ea = kHidErr * sqrtf(1.0001f * (wn2[0][col] + wn2[1][col])) * un[sl] + fabsf(a) * 0x1p-20f;
+                    const float eg = 1.13f * ea + fabsf(g) * 0x1p-16f;
+                    const float mid = __uint_as_float((__float_as_uint(g) & 0xFFFF0000u) | 0x8000u);
+                    const bool exact = valid && !(isfinite(g) && fabsf(g - mid) > eg);
+                    uint16_t hb = __bfloat16_as_ushort(__float2bfloat16_rn(g));
+                    // the units near a rounding midpoint, one at a time by the whole warp
+                    for (unsigned mask = __ballot_sync(0xFFFFFFFFu, exact); mask; mask &= mask - 1) {
+                        const int src = __ffs(mask) - 1;
+                        const int scol = __shfl_sync(0xFFFFFFFFu, col, src);
+                        const uint16_t e = hidden_exact_bf16_warp(
+                            reinterpret_cast<const __nv_bfloat16 *>(p.head.weight) + (size_t)(c0 + scol) * dim,
+                            reinterpret_cast<const __nv_bfloat16 *>(u_s + (size_t)sl * u_stride), dim,
+                            p.head.bias[c0 + scol]);
+                        if (lane == src) hb = e;
                     }
+                    if (valid) reinterpret_cast<uint16_t *>(ho)[(size_t)(s0 + sl) * C + c0 + col] = hb;
+                } else {
+                    if (valid) ho[(size_t)(s0 + sl) * C + c0 + col] = from_float<T>(g);
                 }
             }
         } else {

@@ -363,6 +363,15 @@ def parity_vs_oracle(chain, o_outs, dtype, near_tie=1e-6):
                                        "with an oracle margin below 1e-6 counted, not excused"}
 
 
+def per_sample_kernel(b):
+    """The per-sample kernel a stage of this batch launches: the tcgen05 kernels for bf16 keys
+    whose width is a multiple of 64 (the tiled one once a half holds more than 128 tokens,
+    i.e. from 258 tokens), the mma.sync / FFMA kernel otherwise."""
+    if b.dtype != "bf16" or b.dim % 64:
+        return "k_image"
+    return "k_image_tc_tiled" if int(np.diff(b.offsets).max()) >= 258 else "k_image_tc"
+
+
 def torch_int16():
     import torch
     return torch.int16
@@ -587,7 +596,7 @@ def main():
                    "l2": "flushed before every stage (512 MB write, untimed)",
                    "timing": ("CUDA events around each stage's kernels, summed; " +
                               ("eager launches" if args.eager else "one step captured as a CUDA graph and replayed"))},
-        "roofline": {"bound": "hbm", "kernel": "k_image (merge + prune + gather)", "achieved": achieved,
+        "roofline": {"bound": "hbm", "kernel": per_sample_kernel(b) + " (merge + prune + gather)", "achieved": achieved,
                      "peak": peak, "unit": "GB/s", "frac": achieved / peak, "peak_source": peak_src,
                      "traffic": (tr["dram_bytes_per_launch"] if tr else None),
                      "algorithmic_bytes_per_launch": bytes_image / S,

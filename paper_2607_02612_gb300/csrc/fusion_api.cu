@@ -157,7 +157,7 @@ bool fuse_plan(const fusion_ragged &in) { return in.max_batch >= 1 && in.max_bat
 // The per-sample kernel: TMA + tcgen05 when the shape allows it, else the general one.
 cudaError_t launch_sample_kernel(int dtype, const ImageParams &p, const ImageGeometry &G, cudaStream_t s) {
     if (p.do_merge) {
-        const TcGeometry T = image_tc_geometry(dtype, p.in.max_tokens, p.kdim, p.in.max_rows, 1, kTcSmemBudgetKb);
+        const TcGeometry T = image_tc_geometry(dtype, p.in.max_tokens, p.kdim, p.dim, p.in.max_rows, 1, kTcSmemBudgetKb);
         if (T.ok) return launch_image_tc(p, T, s);
     }
     return launch_image(dtype, p, G.smem, s);

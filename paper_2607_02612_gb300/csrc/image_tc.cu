@@ -35,6 +35,9 @@ constexpr int kMaxStages = 16;
 
 struct TcMaps {
     CUtensorMap e32, o32, e8, o8;   // even / odd rows, boxes of 32 / 8 rows x 64 dims
+    // even / odd rows seen as (64 dims, row, K-block) with the K-block stride 128 B: a box of
+    // 8 rows x all K-blocks lands as [K-block][8 rows][128 B], one 1 KB swizzle atom per K-block
+    CUtensorMap ge, go;
 };
 
 // ss + sc += part, Neumaier-compensated.
@@ -53,19 +56,127 @@ __device__ __forceinline__ float chunk_sq(uint4 v) {
     return part;
 }
 
-// Chunk c of input token pos from the resident swizzled stages (CLS from global).
-struct SwizzledLoader {
-    const unsigned char *regA, *regB;
-    uint32_t kbA, kbB;   // bytes of one K-block of each half
-    GlobalLoader<__nv_bfloat16> g;
+// Chunk c of input token pos for the finish phase, wherever the sample's rows are: one type
+// for every layout, so the finish phase is compiled once (its code is fetched cold after every
+// flush of L2, and a second copy for another layout made stages slower).
+//   rows in global memory (g != null): chunk c of token pos at g + pos * rb + 16 c;
+//   rows in shared memory: CLS from its staged copy; row r of a half (positions 2, 4, ... or
+//   1, 3, ...) at h + (r / 8) G + (r % 8) 128, its 16-byte chunk c (c / 8) K + 16 ((c % 8) ^
+//   (r % 8)) further (ring: h = the half's base in stage 0, G = 1024, K = kbs; grouped layout:
+//   h = the half's first group, G = n_kb KB, K = 1024).
+// The branch is uniform over the CTA.
+struct RowLoader {
+    const unsigned char *g;   // the sample's first row in global memory, or null
+    uint32_t rb;               // bytes of a token row
+    const unsigned char *cls, *hA, *hB;
+    uint32_t G, K;
     __device__ __forceinline__ uint4 operator()(int pos, int c) const {
-        if (pos == 0) return g(0, c);
+        if (g) return ldg16(g + (size_t)pos * rb + (size_t)c * 16);
+        if (pos == 0) return *reinterpret_cast<const uint4 *>(cls + (size_t)c * 16);
         const bool isB = pos & 1;
-        const int r = isB ? (pos - 1) >> 1 : (pos - 2) >> 1;
-        const unsigned char *base = (isB ? regB : regA) + (size_t)(c >> 3) * (isB ? kbB : kbA);
-        return *reinterpret_cast<const uint4 *>(base + r * 128 + (((c & 7) ^ (r & 7)) << 4));
+        const unsigned r = (unsigned)(isB ? (pos - 1) >> 1 : (pos - 2) >> 1);
+        const unsigned x = r & 7u, cc = (unsigned)c;
+        const unsigned char *base = (isB ? hB : hA) + (size_t)(r >> 3) * G + (size_t)(cc >> 3) * K;
+        return *reinterpret_cast<const uint4 *>(base + x * 128u + (((cc & 7u) ^ x) << 4));
     }
 };
+
+// The ring of K-block stages of one sample, sized for it: S stages of kbs bytes, K-block kb
+// in stage kb % S with half A at the stage's start and half B after rowsA rows.  The boxes of
+// one K-block: half A then half B, in 32-row boxes while 32 rows remain, then 8-row boxes.
+struct Ring {
+    int S, rowsA, rowsB, npad, nbA, per_kb;
+    uint32_t kbs;
+};
+__device__ __forceinline__ Ring ring_for(int nA, int nB, int nkb, const TcGeometry &g) {
+    Ring R;
+    R.rowsA = (nA + 7) & ~7;
+    R.rowsB = (nB + 7) & ~7;
+    R.npad = (nB + 15) & ~15;   // MMA N: |B| rounded up to 16
+    R.kbs = (uint32_t)(R.rowsA + R.rowsB) * 128u;
+    // An MMA reads 128 A rows and npad B rows from a stage, past its end when the sample is
+    // small, which stays inside the buffer.
+    const uint32_t reach = (uint32_t)max(16384, (R.rowsA + R.npad) * 128);
+    int S = min(min(nkb, kMaxStages), (int)(g.stage_region / R.kbs));
+    while (S > 1 && (uint32_t)(S - 1) * R.kbs + reach > g.usable) --S;
+    R.S = S;
+    R.nbA = (nA >> 5) + (((nA & 31) + 7) >> 3);
+    R.per_kb = R.nbA + (nB >> 5) + (((nB & 31) + 7) >> 3);
+    return R;
+}
+// Box b of K-block kb of the sample whose rows start at `start` (half A: positions 2, 4, ...,
+// half B: 1, 3, ..., each contiguous in the even or odd row view).
+__device__ __forceinline__ void issue_box(const TcMaps &maps, const Ring &R, int start, int nA, int nB,
+                                          unsigned char *sm, unsigned long long *bar_full, int kb, int b) {
+    const int st = kb % R.S;
+    const int half = b >= R.nbA ? 1 : 0;
+    const int q = half ? b - R.nbA : b;
+    const int n32 = (half ? nB : nA) >> 5;
+    const bool big = q < n32;
+    const int row0 = big ? q * 32 : n32 * 32 + (q - n32) * 8;
+    const bool odd = half ? ((start + 1) & 1) : ((start + 2) & 1);
+    const CUtensorMap *map = big ? (odd ? &maps.o32 : &maps.e32) : (odd ? &maps.o8 : &maps.e8);
+    const int y = half ? (start + 1) >> 1 : (start + 2) >> 1;
+    const uint32_t dst = smem_addr(sm + (half ? (size_t)R.rowsA * 128 : (size_t)0) + (size_t)st * R.kbs + (size_t)row0 * 128);
+    tma_load_2d(dst, map, kb * 64, y + row0, smem_addr(&bar_full[st]));
+}
+// Every barrier a ring can use, from one thread at kernel entry: the fence that publishes the
+// initialisation waits for the thread's outstanding memory operations, so it runs before the
+// thread has issued any.
+__device__ __forceinline__ void ring_barriers_init(unsigned long long *bar_full, unsigned long long *bar_empty,
+                                                   unsigned long long *bar_done) {
+    for (int st = 0; st < kMaxStages; ++st) {
+        mbar_init(smem_addr(&bar_full[st]), 1);
+        mbar_init(smem_addr(&bar_empty[st]), 1 + kTcThreads / 32);
+    }
+    mbar_init(smem_addr(bar_done), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+// From the 32 lanes of one warp, once the barriers are initialised and that is visible to the
+// warp: the first min(S, nkb) K-blocks.
+__device__ __forceinline__ void ring_start(const TcMaps &maps, const Ring &R, int start, int nA, int nB, int nkb,
+                                           unsigned char *sm, unsigned long long *bar_full) {
+    const int lane = threadIdx.x & 31;
+    __syncwarp();
+    const int S0 = min(R.S, nkb);
+    if (lane < S0) mbar_expect_tx(smem_addr(&bar_full[lane]), R.kbs);
+    for (int t = lane; t < S0 * R.per_kb; t += 32)
+        issue_box(maps, R, start, nA, nB, sm, bar_full, t / R.per_kb, t % R.per_kb);
+}
+// A sample that fits in shared memory, grouped: half A in 8-row groups g at g * nkb KB, each
+// group [K-block][8 rows][128 B], half B after it the same way, all behind bar_full[0]; one box
+// per group (the K-block ring needs per_kb boxes per K-block).  The rows of the last group past
+// the half belong to the next sample or lie past the tensor (zero fill) and are never used.
+// From the 32 lanes of one warp, once the barriers are initialised and that is visible to it.
+__device__ __forceinline__ void group_start(const TcMaps &maps, const Ring &R, int start, int nkb, unsigned char *sm,
+                                            unsigned long long *bar_full) {
+    const int lane = threadIdx.x & 31;
+    const int GA = R.rowsA >> 3, GB = R.rowsB >> 3;
+    const uint32_t gstride = (uint32_t)nkb * 1024u;
+    __syncwarp();
+    if (lane == 0) mbar_expect_tx(smem_addr(&bar_full[0]), (uint32_t)(GA + GB) * gstride);
+    const bool oddA = (start + 2) & 1, oddB = (start + 1) & 1;
+    const int yA = (start + 2) >> 1, yB = (start + 1) >> 1;
+    for (int b = lane; b < GA + GB; b += 32) {
+        const bool isB = b >= GA;
+        const int q = isB ? b - GA : b;
+        const CUtensorMap *map = (isB ? oddB : oddA) ? &maps.go : &maps.ge;
+        const uint32_t dst = smem_addr(sm + (size_t)(isB ? GA + q : q) * gstride);
+        tma_load_3d(dst, map, 0, (isB ? yB : yA) + 8 * q, 0, smem_addr(&bar_full[0]));
+    }
+}
+// The sample's token sizes and scores and its CLS row into shared memory (cp.async, one
+// group; waited for in meta_init_rest).
+__device__ __forceinline__ void prefetch_own(const ImageParams &p, int start, int N, const MetaPtrs &m, uint4 *cls) {
+    for (int pos = threadIdx.x; pos < N; pos += kTcThreads) {
+        cp_async4(&m.tsize[pos], p.sizes + start + pos);
+        if (p.scores) cp_async4(&m.tscore[pos], p.scores + start + pos);
+    }
+    const uint4 *row = reinterpret_cast<const uint4 *>(reinterpret_cast<const __nv_bfloat16 *>(p.x) + (long long)start * p.dim);
+    for (int c = threadIdx.x; c < p.dim / 8; c += kTcThreads) cp_async16(&cls[c], row + c);
+    cp_async_commit();
+}
 
 __global__ void __launch_bounds__(kTcThreads, 2)
     k_image_tc(const __grid_constant__ TcMaps maps, ImageParams p, TcGeometry g) {
@@ -90,6 +201,15 @@ __global__ void __launch_bounds__(kTcThreads, 2)
         const CUtensorMap *mp = tid == 32 ? &maps.e32 : tid == 33 ? &maps.o32 : tid == 34 ? &maps.e8 : &maps.o8;
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(mp)) : "memory");
     }
+    // the ring's barriers, before this thread issues any memory operation (warp 0 issues the
+    // tokens' loads after a CTA barrier: the fused plan's, or the one below)
+    if (tid == 36) ring_barriers_init(bar_full, bar_empty, &bar_done);
+    if (g.grouped && (tid == 38 || tid == 39))
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tid == 38 ? &maps.ge : &maps.go)) : "memory");
+    if (tid == 0) s_fail = 0;   // visible after the barriers below, before any other write
+    const int nkb = g.n_kb;
+    MetaPtrs m(sm, meta_layout(p.in.max_tokens, g.meta_base));
+    uint4 *cls = reinterpret_cast<uint4 *>(sm + g.cls_base);
     SampleInfo s;
     if (!sample_begin<kTcThreads>(p, blockIdx.x, s)) {   // uniform over the CTA
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -99,62 +219,29 @@ __global__ void __launch_bounds__(kTcThreads, 2)
                          : "memory");
         return;
     }
+    if (!p.fused_plan) __syncthreads();   // uniform: the fused plan has barriers of its own
     const bool dec = s.decide;
-    const int nkb = g.n_kb;
-    const int rowsA = (s.nA + 7) & ~7, rowsB = (s.nB + 7) & ~7;
-    const int npad = (s.nB + 15) & ~15;   // MMA N: |B| rounded up to 16
-    // The ring is sized for this sample: stage st holds K-block kb (st = kb % S) of half A
-    // at st * kbs and of half B right after it.  An MMA reads 128 A rows and npad B rows
-    // from a stage, past its end when the sample is small, which stays inside the buffer.
-    const uint32_t kbs = (uint32_t)(rowsA + rowsB) * 128u;
-    const uint32_t reach = (uint32_t)max(16384, (rowsA + npad) * 128);
-    int S = min(min(nkb, kMaxStages), (int)(g.stage_region / kbs));
-    while (S > 1 && (uint32_t)(S - 1) * kbs + reach > g.usable) --S;
-    unsigned char *regA = sm;                       // stage st, half A: regA + st * kbs
-    unsigned char *regB = sm + (size_t)rowsA * 128;  // stage st, half B: regB + st * kbs
-    const uint32_t kb_tx = kbs;
-    const int yA = (s.start + 2) >> 1, yB = (s.start + 1) >> 1;
-    const bool oddA = (s.start + 2) & 1, oddB = (s.start + 1) & 1;
-    // The boxes of one K-block: half A then half B, each in 32-row boxes while 32 rows
-    // remain, then 8-row boxes.
-    const int nbA = (s.nA >> 5) + (((s.nA & 31) + 7) >> 3);
-    const int per_kb = nbA + (s.nB >> 5) + (((s.nB & 31) + 7) >> 3);
-    auto issue_box = [&](int kb, int b) {
-        const int st = kb % S;
-        const int half = b >= nbA ? 1 : 0;
-        const int q = half ? b - nbA : b;
-        const int n32 = (half ? s.nB : s.nA) >> 5;
-        const bool big = q < n32;
-        const int row0 = big ? q * 32 : n32 * 32 + (q - n32) * 8;
-        const bool odd = half ? oddB : oddA;
-        const CUtensorMap *map = big ? (odd ? &maps.o32 : &maps.e32) : (odd ? &maps.o8 : &maps.e8);
-        const uint32_t dst = smem_addr((half ? regB : regA) + (size_t)st * kbs + (size_t)row0 * 128);
-        tma_load_2d(dst, map, kb * 64, (half ? yB : yA) + row0, smem_addr(&bar_full[st]));
-    };
+    const Ring R = ring_for(s.nA, s.nB, nkb, g);
+    const int S = R.S, npad = R.npad;
+    const uint32_t kbs = R.kbs;
+    unsigned char *regA = sm;                         // stage st, half A: regA + st * kbs
+    unsigned char *regB = sm + (size_t)R.rowsA * 128;  // stage st, half B: regB + st * kbs (ring layout)
     auto produce = [&](int kb) {   // a whole K-block from one thread
-        mbar_expect_tx(smem_addr(&bar_full[kb % S]), kb_tx);
-        for (int b = 0; b < per_kb; ++b) issue_box(kb, b);
+        mbar_expect_tx(smem_addr(&bar_full[kb % S]), kbs);
+        for (int b = 0; b < R.per_kb; ++b) issue_box(maps, R, s.start, s.nA, s.nB, sm, bar_full, kb, b);
     };
 
-    // the sample's token sizes and scores first (a few KB that would otherwise queue behind
-    // the bulk loads), then the first stages' loads, spread over warp 0
-    MetaPtrs m(sm, meta_layout(p.in.max_tokens, g.meta_base));
-    meta_prefetch<kTcThreads>(p, s, m);
-    if (warp == 0) {
-        if (lane == 0) s_fail = 0;
-        if (dec) {
-            if (lane < S) {
-                mbar_init(smem_addr(&bar_full[lane]), 1);
-                mbar_init(smem_addr(&bar_empty[lane]), 1 + kTcThreads / 32);
-            }
-            if (lane == 31) mbar_init(smem_addr(&bar_done), 1);
-            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            __syncwarp();
-            const int S0 = min(S, nkb);
-            if (lane < S0) mbar_expect_tx(smem_addr(&bar_full[lane]), kb_tx);
-            for (int t = lane; t < S0 * per_kb; t += 32) issue_box(t / per_kb, t % per_kb);
-        }
+    // the sample's sizes, scores and CLS row first (a few KB that would otherwise queue behind the
+    // bulk loads), then its tokens: the grouped layout or the ring's first stages (warp 0)
+    prefetch_own(p, s.start, s.N, m, cls);
+    const bool grouped = g.grouped && S >= nkb;   // the layout of this sample (uniform)
+    const uint32_t gstride = (uint32_t)nkb * 1024u;
+    unsigned char *gB = sm + (size_t)(R.rowsA >> 3) * gstride;   // grouped layout: half B
+    if (warp == 0 && dec) {
+        if (grouped)
+            group_start(maps, R, s.start, nkb, sm, bar_full);
+        else
+            ring_start(maps, R, s.start, s.nA, s.nB, nkb, sm, bar_full);
     }
     meta_init_rest<kTcThreads>(p, s, m);
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -174,7 +261,21 @@ __global__ void __launch_bounds__(kTcThreads, 2)
         const bool has_row = !resident && row < (isA ? s.nA : s.nB);
         float ss = 0.0f, sc = 0.0f;
         bool ok = true;
-        for (int kb = 0; kb < nkb; ++kb) {
+        if (grouped) {   // everything behind one barrier; all products at once
+            if (!mbar_wait(smem_addr(&bar_full[0]), 0u)) {
+                ok = false;
+            } else if (tid == 32) {
+                const uint32_t a0 = smem_addr(sm), b0 = smem_addr(gB);
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                for (int kb = 0; kb < nkb; ++kb)
+#pragma unroll
+                    for (int k = 0; k < 4; ++k)
+                        umma_bf16(tmem, sw128_desc_sbo(a0 + kb * 1024 + k * 32, gstride),
+                                  sw128_desc_sbo(b0 + kb * 1024 + k * 32, gstride), idesc, (kb | k) ? 1u : 0u);
+                umma_commit(smem_addr(&bar_done));
+            }
+        }
+        for (int kb = 0; kb < (grouped ? 0 : nkb); ++kb) {
             const int st = kb % S;
             const uint32_t par = (uint32_t)(kb / S) & 1u;
             if (!mbar_wait(smem_addr(&bar_full[st]), par)) {
@@ -218,10 +319,12 @@ __global__ void __launch_bounds__(kTcThreads, 2)
             if (r < R) {
                 const bool rA = r < s.nA;
                 const int rr = rA ? r : r - s.nA;
-                const unsigned char *base = (rA ? regA : regB) + (size_t)rr * 128;
+                const unsigned char *base = grouped ? (rA ? sm : gB) + (size_t)(rr >> 3) * gstride + (rr & 7) * 128
+                                                    : (rA ? regA : regB) + (size_t)rr * 128;
+                const uint32_t kstep = grouped ? 1024u : kbs;   // bytes from one K-block of the row to the next
                 for (int c = part; c < nkb * 8; c += kT)
                     neumaier_add(ss, sc, chunk_sq(*reinterpret_cast<const uint4 *>(
-                                             base + (size_t)(c >> 3) * kbs + (((c & 7) ^ (rr & 7)) << 4))));
+                                             base + (size_t)(c >> 3) * kstep + (((c & 7) ^ (rr & 7)) << 4))));
             }
             for (int mk = 1; mk < kT; mk <<= 1) {   // kT divides 32: groups stay inside a warp
                 const float oss = __shfl_xor_sync(0xFFFFFFFFu, ss, mk), osc = __shfl_xor_sync(0xFFFFFFFFu, sc, mk);
@@ -283,13 +386,17 @@ __global__ void __launch_bounds__(kTcThreads, 2)
     }
 
     if (s_fail == 0) {
-        const GlobalLoader<__nv_bfloat16> gl{reinterpret_cast<const __nv_bfloat16 *>(p.x), (long long)s.start, p.dim};
-        if (dec && S >= nkb && p.keys_alias) {   // the whole sample is still in shared memory
-            const SwizzledLoader ld{regA, regB, kbs, kbs, gl};
-            finish_sample<__nv_bfloat16, kTcThreads>(p, s, m, ld);
-        } else {
-            finish_sample<__nv_bfloat16, kTcThreads>(p, s, m, gl);
+        const uint32_t rb = (uint32_t)p.dim * 2u;   // bytes of a token row
+        RowLoader ld{reinterpret_cast<const unsigned char *>(p.x) + (size_t)s.start * rb, rb,
+                     reinterpret_cast<const unsigned char *>(cls), nullptr, nullptr, 0u, 0u};
+        if (dec && S >= nkb && p.keys_alias) {   // the whole sample is in shared memory
+            ld.g = nullptr;
+            ld.hA = sm;
+            ld.hB = grouped ? gB : regB;
+            ld.G = grouped ? gstride : 1024u;
+            ld.K = grouped ? 1024u : kbs;
         }
+        finish_sample<__nv_bfloat16, kTcThreads>(p, s, m, ld);
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
@@ -597,7 +704,7 @@ TcGeometry tiled_geometry(int max_tokens, int kdim) {
 }
 }  // namespace
 
-TcGeometry image_tc_geometry(int dtype, int max_tokens, int kdim, long long max_rows, int do_merge,
+TcGeometry image_tc_geometry(int dtype, int max_tokens, int kdim, int dim, long long max_rows, int do_merge,
                              int stage_budget_kb) {
     TcGeometry g{};
     if (dtype != FUSION_BF16 || !do_merge || kdim % 64 != 0 || max_rows < 2) return g;
@@ -615,9 +722,10 @@ TcGeometry image_tc_geometry(int dtype, int max_tokens, int kdim, long long max_
     const size_t reach = std::max<size_t>(16384, g.kb_a + npad_max * 128);
     size_t budget = (size_t)stage_budget_kb * 1024;
     if (budget > 227 * 1024 - 4096) budget = 227 * 1024 - 4096;   // room for static shared memory
-    auto need = [&](int S) {   // usable bytes for S stages at max_tokens
+    // usable bytes for S stages at max_tokens: the ring, the metadata, the CLS row (dim bf16)
+    auto need = [&](int S) {
         const size_t meta_base = (size_t)S * per_stage + 2048;
-        return std::max(meta_layout(max_tokens, meta_base).total, (size_t)(S - 1) * per_stage + reach);
+        return std::max(meta_layout(max_tokens, meta_base).total + (size_t)dim * 2, (size_t)(S - 1) * per_stage + reach);
     };
     int S = g.n_kb < kMaxStages ? g.n_kb : kMaxStages;
     while (S > 2 && need(S) + 1024 > budget) --S;
@@ -625,7 +733,17 @@ TcGeometry image_tc_geometry(int dtype, int max_tokens, int kdim, long long max_
     g.stages = S;
     g.stage_region = (uint32_t)(S * per_stage);
     g.meta_base = (uint32_t)(S * per_stage + 2048);
+    g.cls_base = (uint32_t)meta_layout(max_tokens, g.meta_base).total;
     g.usable = (uint32_t)need(S);
+    // The grouped layout for samples that fit: an MMA reads 128 A rows, 16 groups of n_kb KB from
+    // the start of the buffer, and up to one group past half B (npad rows), so the buffer must
+    // cover both; when the budget allows it, it does.
+    const size_t gstride = (size_t)g.n_kb * 1024;
+    const size_t g_need = std::max({(size_t)g.usable, 16 * gstride, (size_t)g.stage_region + gstride});
+    if (g_need + 1024 <= budget) {
+        g.grouped = 1;
+        g.usable = (uint32_t)g_need;
+    }
     g.smem = g.usable + 1024;
     g.ok = 1;
     return g;
@@ -635,7 +753,7 @@ cudaError_t launch_image_tc(const ImageParams &p, const TcGeometry &g, cudaStrea
     if (p.in.max_batch == 0) return cudaSuccess;
     EncodeTiledFn enc = encode_fn();
     if (!enc) return cudaErrorNotSupported;
-    TcMaps maps;
+    TcMaps maps{};
     const cuuint64_t rows_even = (cuuint64_t)((p.in.max_rows + 1) / 2), rows_odd = (cuuint64_t)(p.in.max_rows / 2);
     const char *keys = reinterpret_cast<const char *>(p.keys);
     for (int i = 0; i < 4; ++i) {
@@ -648,6 +766,17 @@ cudaError_t launch_image_tc(const ImageParams &p, const TcGeometry &g, cudaStrea
         void *base = const_cast<char *>(keys + (odd ? (size_t)p.kdim * 2 : 0));
         if (enc(dst, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                 CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
+    for (int odd = 0; odd < 2 && g.grouped; ++odd) {   // (64 dims, row, K-block), box 8 rows x all K-blocks
+        cuuint64_t dims[3] = {64, odd ? rows_odd : rows_even, (cuuint64_t)(p.kdim / 64)};
+        cuuint64_t strides[2] = {(cuuint64_t)p.kdim * 2 * 2, 128};
+        cuuint32_t box[3] = {64, 8, (cuuint32_t)(p.kdim / 64)};
+        cuuint32_t estr[3] = {1, 1, 1};
+        void *base = const_cast<char *>(keys + (odd ? (size_t)p.kdim * 2 : 0));
+        if (enc(odd ? &maps.go : &maps.ge, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, base, dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
     }

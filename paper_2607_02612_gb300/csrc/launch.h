@@ -153,16 +153,19 @@ cudaError_t launch_image(int dtype, const ImageParams &p, size_t smem, cudaStrea
 struct TcGeometry {
     int ok;
     int tiled;         // halves beyond one tile: k_image_tc_tiled (M-tiles of 128 A rows, one CTA per SM)
+    int grouped;       // samples that fit in shared memory load in 8-row groups of all K-blocks (one 3-D box
+                       // per group) instead of through the ring
     int n_kb;          // key K-blocks of 64 dims
     int stages;        // K-block stages of a sample of max_tokens tokens (more for smaller samples)
     int tmem_cols;     // tensor-memory columns allocated per CTA
     uint32_t kb_a, kb_b;             // bytes of one K-block of half A / half B at max_tokens
     uint32_t stage_region;           // bytes of the K-block ring, from offset 0
     uint32_t meta_base;              // offset of the per-sample metadata
+    uint32_t cls_base;               // offset of the staged CLS row (0: read from global memory)
     uint32_t usable;                 // bytes addressable after the 1 KB alignment
     size_t smem;                     // dynamic shared memory bytes (usable + 1 KB alignment slack)
 };
-TcGeometry image_tc_geometry(int dtype, int max_tokens, int kdim, long long max_rows, int do_merge,
+TcGeometry image_tc_geometry(int dtype, int max_tokens, int kdim, int dim, long long max_rows, int do_merge,
                              int stage_budget_kb);
 cudaError_t launch_image_tc(const ImageParams &p, const TcGeometry &g, cudaStream_t s);
 

@@ -549,12 +549,13 @@ struct ExitClSmem {
     static constexpr int BT = kExitBT;
     using B = ExitSmem<T>;
     // u tile (16 GEMM rows; bf16: swizzled K-blocks) | W stages (bf16: w_stages(dim) TMA stages,
-    // the whole tile when it fits; float32: two cp.async stages) | own raw CLS rows (BT) | gamma |
+    // the whole tile when it fits; float32: two cp.async stages) | own raw CLS rows (BT; bf16:
+    // none here, they use rows 8..15 of the u tile, which feed only unused columns) | gamma |
     // beta | bias | partials [BT][8] | reduction scratch | row flags.  bf16 offsets count from a
     // 1024-byte aligned base (the total includes the slack).
     static __host__ __device__ size_t u_bytes(int dim) { return kTc ? (size_t)((dim + 63) / 64) * 2048 : B::u_bytes(dim); }
     static __host__ __device__ size_t rest_bytes(int dim) {   // everything but the W stages
-        return u_bytes(dim) + (size_t)BT * B::u_stride(dim) * EB + 2 * (((size_t)dim * EB + 15) / 16 * 16) +
+        return u_bytes(dim) + x_bytes(dim) + 2 * (((size_t)dim * EB + 15) / 16 * 16) +
                kExitCT * sizeof(float) + (size_t)BT * 8 * sizeof(float2) + (kExitThreads / 32) * 8 * sizeof(float) +
                (size_t)BT * sizeof(int);
     }
@@ -567,9 +568,10 @@ struct ExitClSmem {
         return nk < st ? nk : st;
     }
     static __host__ __device__ size_t w_bytes(int dim) { return kTc ? (size_t)w_stages(dim) * kExitWStage : 2 * B::w_stage; }
+    static __host__ __device__ size_t x_bytes(int dim) { return kTc ? 0 : (size_t)BT * B::u_stride(dim) * EB; }
     static __host__ __device__ size_t w_off(int dim) { return u_bytes(dim); }
     static __host__ __device__ size_t x_off(int dim) { return w_off(dim) + w_bytes(dim); }
-    static __host__ __device__ size_t g_off(int dim) { return x_off(dim) + (size_t)BT * B::u_stride(dim) * EB; }
+    static __host__ __device__ size_t g_off(int dim) { return x_off(dim) + x_bytes(dim); }
     static __host__ __device__ size_t be_off(int dim) { return g_off(dim) + ((size_t)dim * EB + 15) / 16 * 16; }
     static __host__ __device__ size_t bias_off(int dim) { return be_off(dim) + ((size_t)dim * EB + 15) / 16 * 16; }
     static __host__ __device__ size_t part_off(int dim) { return bias_off(dim) + kExitCT * sizeof(float); }
@@ -604,6 +606,10 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
                                 : sm;
     T *u_s = reinterpret_cast<T *>(base);   // float32: [16][u_stride]; bf16: see u_tc_off
     T *x_s = reinterpret_cast<T *>(base + L::x_off(dim));
+    // chunk c of own raw CLS row j: float32 [BT][u_stride]; bf16 rows 8 + j of the u tile
+    auto raw_chunk = [&](int j, int c) -> T * {
+        return kBf16 ? reinterpret_cast<T *>(base + u_tc_off(8 + j, c)) : x_s + (size_t)j * u_stride + c * CH;
+    };
     T *g_s = reinterpret_cast<T *>(base + L::g_off(dim));
     T *be_s = reinterpret_cast<T *>(base + L::be_off(dim));
     unsigned char *w_region = base + L::w_off(dim);   // bf16: 1024-byte aligned TMA stages
@@ -655,7 +661,7 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
         for (int it = tid; it < BT * nchunk; it += kExitThreads) {
             const int jj = it / nchunk, c = it - jj * nchunk;
             const int sli = rank + jj * ncl, si = s0 + sli;
-            T *dst = x_s + (size_t)jj * u_stride + c * CH;
+            T *dst = raw_chunk(jj, c);
             long long row = -1;
             const bool want = sli < BT && si < B;
             if (want) {
@@ -688,7 +694,9 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
             *reinterpret_cast<uint4 *>(u_s + (size_t)r * u_stride + c * CH) = make_uint4(0, 0, 0, 0);
         }
     }
-    cl.sync();   // every CTA of the cluster runs before any remote shared-memory store
+    // every CTA of the cluster runs before any remote shared-memory store; nothing written before
+    // it is read remotely, so the arrive need not release anything
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;\n\tbarrier.cluster.wait.aligned;" ::: "memory");
     if (active) {
         cp_async_wait_all();
         __syncthreads();
@@ -707,11 +715,10 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
             if (rflag < 0 && gt == 0) raise_status(p.status, FUSION_DEV_BAD_OFFSETS);
             const bool ok = rflag > 0;
             const F2 rdim = f2_recip((float)dim);
-            const T *xr = x_s + (size_t)j * u_stride;
             float s1 = 0.0f, c1 = 0.0f, s2 = 0.0f, c2 = 0.0f, l2 = 0.0f;
             if (ok) {
                 for (int e = gt; e < dim; e += G * 32) {
-                    const float v = to_float(xr[e]);
+                    const float v = to_float(raw_chunk(j, e / CH)[e % CH]);
                     neu_add(s1, c1, v);
                     const F2 sq = two_prod(v, v);
                     neu_add(s2, c2, sq.hi);
@@ -745,7 +752,7 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
                 if (gt == 0 && !(isfinite(mean.hi) && isfinite(var.hi))) raise_status(p.status, FUSION_DEV_NONFINITE);
                 for (int c = gt; c < nchunk; c += G * 32) {
                     float f[CH], gf[CH], bf[CH];
-                    chunk_to_f(*reinterpret_cast<const uint4 *>(xr + c * CH), f);
+                    chunk_to_f(*reinterpret_cast<const uint4 *>(raw_chunk(j, c)), f);
                     chunk_to_f(*reinterpret_cast<const uint4 *>(g_s + c * CH), gf);
                     chunk_to_f(*reinterpret_cast<const uint4 *>(be_s + c * CH), bf);
                     uint4 outv;

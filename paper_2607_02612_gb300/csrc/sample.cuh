@@ -534,18 +534,25 @@ __device__ __noinline__ uint4 merged_exact_bf16(const float *tsize, const int *s
 //  * m, the midpoint of that interval, decides the rounding: R = fma(m, -den, num) is
 //    num - m den rounded once, so its sign (and whether it is zero) is that of t - m:
 //    t beyond m rounds away from b, short of m to b, exactly on m to the even end.
-// Otherwise (long sizes, an inexact sum, non-finite values) the float-float computation
-// runs, out of line.
+// When the products are exact but their float sum is not, the chain's rounding errors,
+// summed beside it, make the float-float numerator that the out-of-line computation would
+// form from the same products in the same order (its product remainders are zero), and
+// mean_bits rounds it here.  Otherwise (long sizes, an inexact sum of sizes, non-finite
+// values) the float-float computation runs, out of line.
 template <typename Loader>
 __device__ __forceinline__ uint4 merged_fast_bf16(const MetaPtrs &m, const MergedItem &it, const Loader &load) {
     const float sb = m.tsize[it.pos];
     const float2 iv = m.invd[it.pos];   // 1 / den as float-float
-    float num[8], x[8];
+    float num[8], lo[8], x[8];
     chunk_to_f(it.self, x);
 #pragma unroll
-    for (int e = 0; e < 8; ++e) num[e] = __fmul_rn(sb, x[e]);
+    for (int e = 0; e < 8; ++e) {
+        num[e] = __fmul_rn(sb, x[e]);
+        lo[e] = 0.0f;
+    }
     float den = sb;
-    bool ok = short_size(sb);
+    bool ok = short_size(sb);   // every product exact, the sum of sizes exact
+    bool exact = true;          // and the sum of products too
     for (int q = it.q0; q < it.q1; ++q) {
         const int u = q - it.q0;
         const int ap = 2 + 2 * m.slist[q];
@@ -558,8 +565,23 @@ __device__ __forceinline__ uint4 merged_fast_bf16(const MetaPtrs &m, const Merge
         for (int e = 0; e < 8; ++e) {
             const F2 t = two_sum(num[e], __fmul_rn(sa, x[e]));
             num[e] = t.hi;
-            ok = ok && t.lo == 0.0f;
+            lo[e] = __fadd_rn(lo[e], t.lo);
+            exact = exact && t.lo == 0.0f;
         }
+    }
+    if (!ok)
+        return merged_exact_bf16(m.tsize, m.slist, m.invd, it.pos, it.c, it.q0, it.q1, it.self, it.av[0], it.av[1], load);
+    if (!exact) {
+        const F2 dn = {den, 0.0f};
+        const F2 inv = {iv.x, iv.y};
+        const bool pow2 = (__float_as_uint(den) & 0x007FFFFFu) == 0u;
+        uint32_t w[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+            w[k] = (uint32_t)mean_bits(quick_two_sum(num[2 * k], lo[2 * k]), dn, inv, pow2, __nv_bfloat16{}) |
+                   ((uint32_t)mean_bits(quick_two_sum(num[2 * k + 1], lo[2 * k + 1]), dn, inv, pow2, __nv_bfloat16{})
+                    << 16);
+        return make_uint4(w[0], w[1], w[2], w[3]);
     }
     uint32_t bits[8];
 #pragma unroll

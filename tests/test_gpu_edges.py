@@ -205,6 +205,37 @@ def test_empty_batch_and_device_count():
     np.testing.assert_array_equal(g["keep_idx"][:o["offsets"][-1]], o["keep_idx"])
 
 
+@pytest.mark.parametrize("dtype,classes", [("bf16", 10), ("bf16", 1000), ("f32", 10), ("bf16", 4000)])
+def test_host_batch_bound_zero(dtype, classes):
+    """A host batch bound of 0 is a legal empty call: the exit check (cluster kernel up to 1024
+    classes, the general one above) and the fused stage with the exit flag return FUSION_OK, raise
+    no status bit, touch no exit output, and the stage writes a batch count of 0 and offsets [0]."""
+    b = make_batch([5, 7], 32, dtype, seed=3)
+    db = P.device_batch(b)
+    db.max_batch = 0
+    f = runner.Fusion(0, classes)
+    head = runner.head_tensors(make_head(32, classes, dtype, 0.5), dtype)
+    mask = torch.full((1,), 7, dtype=torch.uint8, device="cuda")
+    logits = torch.full((1, classes), 3.0, dtype=torch.float32, device="cuda")
+    maxp = torch.full((1,), -1.0, dtype=torch.float32, device="cuda")
+    fz.check(fz.fusion_exit_check(runner.DTYPE_CODE[dtype], db.ragged(), db.x, db.dim, head.c_struct(), mask,
+                                  logits, maxp, f.workspace, f.ws_bytes, f.status))
+    torch.cuda.synchronize()
+    assert int(f.status.item()) == 0
+    assert int(mask.item()) == 7 and float(maxp.item()) == -1.0 and bool(torch.all(logits == 3.0))
+    o = f.stage_outputs(db, 7, head)
+    o.update(exit_mask=mask, logits=logits, max_prob=maxp,   # non-null, one row: the call must not touch them
+             ids=torch.full((1,), 5, dtype=torch.int32, device="cuda"))
+    for k in ("offsets", "batch"):
+        o[k] = torch.full_like(o[k], 5)
+    r = torch.full((1,), 2, dtype=torch.int32, device="cuda")
+    rho = torch.full((1,), 0.5, dtype=torch.float32, device="cuda")
+    g = P.to_host(f.stage(db, 7, r, rho, head, out=o), dtype)
+    assert int(f.status.item()) == 0
+    assert int(g["batch"][0]) == 0 and int(g["offsets"][0]) == 0
+    assert int(mask.item()) == 7 and float(maxp.item()) == -1.0 and bool(torch.all(logits == 3.0))
+
+
 def test_ids_index_router_outputs():
     """With ids, r and rho are read at the original image number."""
     b = make_batch([9, 11, 13], 32, "f32", seed=5)

@@ -81,3 +81,25 @@ def test_noalloc_rejects_batches_beyond_its_scratch():
     rc = lib.fusion_exit_check_noalloc(fz.FUSION_BF16, big, 0x100000, 384, head, 0x100000, None, None, None, None)
     assert rc == fz.FUSION_ERR_WORKSPACE
     assert fz.fusion_workspace_size(1 << 20, 1000) > (1 << 20)
+
+
+@pytest.mark.parametrize("classes", [10, 4000])
+def test_noalloc_batch_bound_zero(classes):
+    """A host batch bound of 0 is an empty call: FUSION_OK, no status bit, outputs untouched."""
+    x = torch.zeros((4, 32), dtype=torch.bfloat16, device="cuda")
+    offsets = torch.zeros(1, dtype=torch.int32, device="cuda")
+    rg = fz.ragged(0, 4, 4, offsets)
+    gamma = torch.ones(32, dtype=torch.bfloat16, device="cuda")
+    beta = torch.zeros(32, dtype=torch.bfloat16, device="cuda")
+    W = torch.ones((classes, 32), dtype=torch.bfloat16, device="cuda")
+    bias = torch.zeros(classes, dtype=torch.float32, device="cuda")
+    head = fz.exit_head(gamma, beta, 1e-6, W, bias, classes, 0.5)
+    mask = torch.full((1,), 7, dtype=torch.uint8, device="cuda")
+    logits = torch.full((1, classes), 3.0, dtype=torch.float32, device="cuda")
+    maxp = torch.full((1,), -1.0, dtype=torch.float32, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    rc = fz.fusion_exit_check_noalloc(fz.FUSION_BF16, rg, x, 32, head, mask, logits, maxp, status)
+    assert rc == fz.FUSION_OK, fz.fusion_status_string(rc)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    assert int(mask.item()) == 7 and float(maxp.item()) == -1.0 and bool(torch.all(logits == 3.0))

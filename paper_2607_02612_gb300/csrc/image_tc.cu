@@ -358,20 +358,26 @@ __global__ void __launch_bounds__(kTcThreads, 2)
             const int c_lo = wg ? half_cols : 0, c_hi = wg ? npad : half_cols;
             const uint32_t lane_addr = tmem + ((uint32_t)((warp & 3) * 32) << 16);
             const float ia = r < s.nA ? m.inv_a[r] : 0.0f;
-            unsigned long long bk = 0ull;
+            // the largest cosine of the thread's columns and its lowest column: the columns go up,
+            // so a strict comparison keeps the first of equal values (and -0 equals +0)
+            float bv = -INFINITY;
+            int bi = -1;
             for (int c0 = c_lo; c0 < c_hi; c0 += 16) {
                 uint32_t v[16];
                 tmem_ld16(lane_addr + (uint32_t)c0, v);
 #pragma unroll
                 for (int e = 0; e < 16; ++e) {
                     const int col = c0 + e;
-                    if (r < s.nA && col < s.nB) {
+                    if (col < s.nB) {
                         const float cs = (__uint_as_float(v[e]) * ia) * m.inv_b[col];
-                        const unsigned long long k = rank_key(cs, col);
-                        bk = k > bk ? k : bk;
+                        if (cs > bv || bi < 0) {
+                            bv = cs;
+                            bi = col;
+                        }
                     }
                 }
             }
+            const unsigned long long bk = (r < s.nA && bi >= 0) ? rank_key(bv, bi) : 0ull;
             if (wg == 1) half_best[r] = bk;
             __syncthreads();
             if (wg == 0 && r < s.nA) {
@@ -614,20 +620,24 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const uint32_t lane_addr = tmem + ((uint32_t)((warp & 3) * 32) << 16);
             const int arow = mt * 128 + r;
             const float ia = r < nA_t ? m.inv_a[arow] : 0.0f;
-            unsigned long long bk = 0ull;
+            float bv = -INFINITY;   // as in k_image_tc: strict comparison over rising columns
+            int bi = -1;
             for (int c0 = c_lo; c0 < c_hi; c0 += 16) {
                 uint32_t v[16];
                 tmem_ld16(lane_addr + (uint32_t)c0, v);
 #pragma unroll
                 for (int e = 0; e < 16; ++e) {
                     const int col = c0 + e;
-                    if (r < nA_t && col < s.nB) {
+                    if (col < s.nB) {
                         const float cs = (__uint_as_float(v[e]) * ia) * m.inv_b[col];
-                        const unsigned long long k = rank_key(cs, col);
-                        bk = k > bk ? k : bk;
+                        if (cs > bv || bi < 0) {
+                            bv = cs;
+                            bi = col;
+                        }
                     }
                 }
             }
+            const unsigned long long bk = (r < nA_t && bi >= 0) ? rank_key(bv, bi) : 0ull;
             if (wg == 1) half_best[r] = bk;
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncthreads();   // the next tile's products overwrite the accumulators after this

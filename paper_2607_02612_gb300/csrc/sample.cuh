@@ -326,14 +326,19 @@ __device__ __forceinline__ void select_top_r(const SampleInfo &s, MetaPtrs &m) {
     const int tid = threadIdx.x;
     for (int a = tid; a < s.nA; a += NT) m.match[a] = (int)(0xFFFFFFFFu - (uint32_t)(m.best[a] & 0xFFFFFFFFull));
     if (s.r_eff > 0) {
-        for (int a = tid; a < s.nA; a += NT)
-            m.rk[a] = (m.best[a] & 0xFFFFFFFF00000000ull) | (0xFFFFFFFFull - (unsigned)a);
+        // the ordered similarity of every A row (the high half of its key)
+        uint32_t *rv = reinterpret_cast<uint32_t *>(m.rk);
+        for (int a = tid; a < s.nA; a += NT) rv[a] = (uint32_t)(m.best[a] >> 32);
         __syncthreads();
         for (int a = tid; a < s.nA; a += NT) {
-            const unsigned long long ka = m.rk[a];
+            // rank of a: the rows of larger similarity, and the rows of equal similarity at a
+            // lower position (32-bit comparisons in two ranges instead of 64-bit keys)
+            const uint32_t va = rv[a];
             int rank = 0;
 #pragma unroll 8
-            for (int q = 0; q < s.nA; ++q) rank += m.rk[q] > ka ? 1 : 0;
+            for (int q = 0; q < a; ++q) rank += rv[q] >= va ? 1 : 0;
+#pragma unroll 8
+            for (int q = a + 1; q < s.nA; ++q) rank += rv[q] > va ? 1 : 0;
             m.sel[a] = rank < s.r_eff ? 1 : 0;
             if (rank < s.r_eff) m.mkey[rank] = (m.match[a] << kKeyShift) | a;
         }
@@ -676,19 +681,23 @@ __device__ bool finish_decide(const ImageParams &p, const SampleInfo &s, MetaPtr
     if (p.do_prune) {
         bool nf = false;
         const int k = keep_count(p.rho[s.id], N - R - 1, nf);
-        // key 0 marks a non-candidate (CLS or merged away); every candidate key is > 0
-        for (int pos = tid; pos < N; pos += NT)
-            m.pk[pos] = (pos > 0 && m.mflag[pos]) ? rank_key(m.mscore[pos], pos) : 0ull;
+        // the ordered merged score of every candidate; 0 marks a non-candidate (CLS or merged
+        // away), below every candidate's value (ordered values of floats are >= 1)
+        uint32_t *pv = reinterpret_cast<uint32_t *>(m.pk);
+        for (int pos = tid; pos < N; pos += NT) pv[pos] = (pos > 0 && m.mflag[pos]) ? ordered_bits(m.mscore[pos]) : 0u;
         __syncthreads();
         for (int pos = tid; pos < N; pos += NT) {
             int keep = 0;
             if (pos == 0) {
                 keep = 1;
             } else if (m.mflag[pos]) {
-                const unsigned long long kp = m.pk[pos];
+                // rank: candidates of larger score, and of equal score at a lower position
+                const uint32_t vp = pv[pos];
                 int rank = 0;
 #pragma unroll 8
-                for (int q = 1; q < N; ++q) rank += m.pk[q] > kp ? 1 : 0;
+                for (int q = 1; q < pos; ++q) rank += pv[q] >= vp ? 1 : 0;
+#pragma unroll 8
+                for (int q = pos + 1; q < N; ++q) rank += pv[q] > vp ? 1 : 0;
                 keep = rank < k ? 1 : 0;
             }
             m.kflag[pos] = keep;

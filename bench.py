@@ -472,45 +472,49 @@ def main():
             import torch.distributed as dist
             dist.barrier()
 
-    # the mid event only where a first kernel runs (the exit check, or the plan kernel of a
-    # batch too large for the fused plan): an empty start-to-mid interval still costs an
-    # event record on the stream
+    # The timed steps record events at stage boundaries only: an event record between two
+    # kernels costs about one completion step (~2 us) of the stream.  The split of an exit
+    # stage between its first kernel (the exit check, or the plan kernel of a batch too large
+    # for the fused plan) and the per-sample kernel comes from a second graph with a mid event
+    # there, replayed as many times after the timed steps.
     has_first = [bool(specs[s].exit) or b.batch > fz.FUSION_FUSED_PLAN_MAX_BATCH for s in range(S)]
 
-    def run_step(evs):
+    def run_step(evs, split):
         for s in range(S):
             flush.fill_(s & 0xFF)
             e0, e1, e2 = evs[s]
-            fz.fusion_profile_next(e0, e1 if has_first[s] else None, e2)
+            fz.fusion_profile_next(e0, e1 if (split and has_first[s]) else None, e2)
             chain.run_stage(s)
 
     mk = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
     step_evs = [(mk(), mk(), mk()) for _ in range(S)]
-    for trio in step_evs:      # create the CUDA events outside any capture
+    split_evs = [(mk(), mk(), mk()) for _ in range(S)]
+    for trio in step_evs + split_evs:   # create the CUDA events outside any capture
         for e in trio:
             e.record()
-    run_step(step_evs)         # one eager step: first launches, kernel attributes
+    run_step(split_evs, True)   # one eager step: first launches, kernel attributes
     torch.cuda.synchronize()
     st = int(fus.status.item())
     if st != 0:
         raise SystemExit(f"device status {st} ({fz.fusion_status_string(st)})")
-    graph = None
+    graph = graph_split = None
     if not args.eager:
         # one step (flushes, events, stages) as a CUDA graph: the launch path a serving loop
         # would use; the events are graph nodes and record at every replay
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(graph):
-            run_step(step_evs)
-    one = graph.replay if graph is not None else (lambda: run_step(step_evs))
+            run_step(step_evs, False)
+        graph_split = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph_split):
+            run_step(split_evs, True)
+    one = graph.replay if graph is not None else (lambda: run_step(step_evs, False))
+    one_split = graph_split.replay if graph_split is not None else (lambda: run_step(split_evs, True))
     for _ in range(args.warmup):
         one()
+        one_split()
     torch.cuda.synchronize()
 
-    def read(trio_list):
-        return ([t[0].elapsed_time(t[2]) for t in trio_list],
-                [t[0].elapsed_time(t[1]) if has_first[s] else 0.0 for s, t in enumerate(trio_list)])
-
-    stage_rows, first_rows = [], []
+    stage_rows, first_rows, image_rows = [], [], []
     barrier()
     torch.cuda.synchronize()
     with ClockSampler(local) as clk:
@@ -518,14 +522,18 @@ def main():
         for k in range(args.steps):
             one()
             torch.cuda.synchronize()   # the step's events are read before the next replay
-            a_, b_ = read(step_evs)
-            stage_rows.append(a_)
-            first_rows.append(b_)
+            stage_rows.append([t[0].elapsed_time(t[2]) for t in step_evs])
         wall = time.perf_counter() - t0
     barrier()
+    for k in range(args.steps):   # the split, after the timed steps
+        one_split()
+        torch.cuda.synchronize()
+        first_rows.append([t[0].elapsed_time(t[1]) if has_first[s] else 0.0 for s, t in enumerate(split_evs)])
+        image_rows.append([t[1].elapsed_time(t[2]) if has_first[s] else t[0].elapsed_time(t[2])
+                           for s, t in enumerate(split_evs)])
     stage_ms = np.array(stage_rows)
     first_ms = np.array(first_rows)
-    image_ms = stage_ms - first_ms
+    image_ms = np.array(image_rows)
     clocks = clk.summary()
     # the outputs of the timed steps against the oracle's chain on the same inputs
     parity = parity_vs_oracle(chain, o_chain, b.dtype) if o_chain is not None else None
@@ -595,7 +603,9 @@ def main():
                    "dim": b.dim, "stages": S, "exit_blocks": list(w.spec.exit_blocks),
                    "l2": "flushed before every stage (512 MB write, untimed)",
                    "timing": ("CUDA events around each stage's kernels, summed; " +
-                              ("eager launches" if args.eager else "one step captured as a CUDA graph and replayed"))},
+                              ("eager launches" if args.eager else "one step captured as a CUDA graph and replayed") +
+                              "; the exit stages' split between their two kernels from a second replay with an "
+                              "event between them (not in the timed steps)")},
         "roofline": {"bound": "hbm", "kernel": per_sample_kernel(b) + " (merge + prune + gather)", "achieved": achieved,
                      "peak": peak, "unit": "GB/s", "frac": achieved / peak, "peak_source": peak_src,
                      "traffic": (tr["dram_bytes_per_launch"] if tr else None),

@@ -93,7 +93,8 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     k_attn_tc(const __grid_constant__ AttnMaps maps, AttnParams p) {
     extern __shared__ unsigned char sm_raw[];
     unsigned char *sm = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~uintptr_t(1023));
-    __shared__ __align__(8) unsigned long long bar_ld, bar_s, bar_o;
+    // bar_ld: query tile 0 and K (the first product's operands); bar_ld2: V and the other query tiles
+    __shared__ __align__(8) unsigned long long bar_ld, bar_ld2, bar_s, bar_o;
     __shared__ uint32_t tmem_base;
     __shared__ int s_fail, s_issued;   // s_issued: operations started (for the drain on a timeout)
     __shared__ __align__(16) float lsz[kAttnMaxN];   // log2 of the key sizes
@@ -130,6 +131,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         s_fail = 0;
         s_issued = 0;
         mbar_init(smem_addr(&bar_ld), 1);
+        mbar_init(smem_addr(&bar_ld2), 1);
         mbar_init(smem_addr(&bar_s), 1);
         mbar_init(smem_addr(&bar_o), 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -137,20 +139,24 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     }
     __syncthreads();
 
-    // ---- loads: the query tiles, K and V by TMA (rows rounded up to 8) --------------------------
+    // ---- loads: the query tiles, K and V by TMA (rows rounded up to 8); query tile 0 and K on
+    // ---- bar_ld (the first product starts once they landed), V and the other tiles on bar_ld2 --
     if (tid == 0) {
         const int rk = (n + 7) & ~7;
-        uint32_t bytes = 2u * (uint32_t)rk * 128u;
-        for (int t = 0; t < T; ++t) bytes += (uint32_t)((min(128, n - 128 * t) + 7) & ~7) * 128u;
-        mbar_expect_tx(smem_addr(&bar_ld), bytes);
-        auto rows = [&](unsigned char *dst, int x, int y0, int cnt) {   // cnt is a multiple of 8
+        auto qrows = [&](int t) { return (min(128, n - 128 * t) + 7) & ~7; };
+        uint32_t bytes2 = (uint32_t)rk * 128u;
+        for (int t = 1; t < T; ++t) bytes2 += (uint32_t)qrows(t) * 128u;
+        mbar_expect_tx(smem_addr(&bar_ld), (uint32_t)(rk + qrows(0)) * 128u);
+        mbar_expect_tx(smem_addr(&bar_ld2), bytes2);
+        auto rows = [&](unsigned char *dst, int x, int y0, int cnt, unsigned long long *bar) {   // cnt: multiple of 8
             int r = 0;
-            for (; r + 32 <= cnt; r += 32) tma_load_2d(smem_addr(dst + r * 128), &maps.b32, x, y0 + r, smem_addr(&bar_ld));
-            for (; r < cnt; r += 8) tma_load_2d(smem_addr(dst + r * 128), &maps.b8, x, y0 + r, smem_addr(&bar_ld));
+            for (; r + 32 <= cnt; r += 32) tma_load_2d(smem_addr(dst + r * 128), &maps.b32, x, y0 + r, smem_addr(bar));
+            for (; r < cnt; r += 8) tma_load_2d(smem_addr(dst + r * 128), &maps.b8, x, y0 + r, smem_addr(bar));
         };
-        for (int t = 0; t < T; ++t) rows(Q + (size_t)t * kQTileBytes, h * kAttnDh, o0 + 128 * t, (min(128, n - 128 * t) + 7) & ~7);
-        rows(Kr, (H + h) * kAttnDh, o0, rk);
-        rows(Vr, (2 * H + h) * kAttnDh, o0, rk);
+        rows(Q, h * kAttnDh, o0, qrows(0), &bar_ld);
+        rows(Kr, (H + h) * kAttnDh, o0, rk, &bar_ld);
+        rows(Vr, (2 * H + h) * kAttnDh, o0, rk, &bar_ld2);
+        for (int t = 1; t < T; ++t) rows(Q + (size_t)t * kQTileBytes, h * kAttnDh, o0 + 128 * t, qrows(t), &bar_ld2);
         s_issued = 1;
     }
     for (int j = tid; j < npad; j += kAttnThreads)
@@ -164,11 +170,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         for (int o = 16; o >= 1; o >>= 1) lm = fmaxf(lm, __shfl_xor_sync(0xFFFFFFFFu, lm, o));
         if (threadIdx.x == 0) s_lszmax = lm;
     }
-    // V rows n .. npad-1 (another sample's rows or stale memory) read as zero in P V
-    if (s_fail == 0)
-        for (int c = tid; c < (npad - n) * 8; c += kAttnThreads)
-            reinterpret_cast<uint4 *>(Vr + (size_t)n * 128)[c] = make_uint4(0u, 0u, 0u, 0u);
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // visible to the tensor core
     __syncthreads();
 
     const uint32_t tmem = tmem_base;
@@ -261,6 +262,16 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
             asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         }
         red[half][r] = lsum2.x + lsum2.y;
+        if (t == 0) {
+            // V and the other query tiles: landed while this tile's softmax ran; V rows n .. npad-1
+            // (another sample's rows or stale memory) read as zero in P V
+            if (tid == 0 && !mbar_wait(smem_addr(&bar_ld2), 0)) atomicOr(&s_fail, 8);
+            __syncthreads();
+            if (s_fail == 0)
+                for (int c = tid; c < (npad - n) * 8; c += kAttnThreads)
+                    reinterpret_cast<uint4 *>(Vr + (size_t)n * 128)[c] = make_uint4(0u, 0u, 0u, 0u);
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // visible to the tensor core
+        }
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
         __syncthreads();   // all of P stored before the second product
         const float lsum = red[0][r] + red[1][r];
@@ -308,6 +319,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     if (tid == 0 && s_fail != 0) {   // let everything this CTA started finish before it leaves
         raise_status(p.status, FUSION_DEV_TIMEOUT);
         mbar_wait(smem_addr(&bar_ld), 0);
+        mbar_wait(smem_addr(&bar_ld2), 0);
         const int k = s_issued;   // 2 + 2t: S of tile t issued; 3 + 2t: also its O
         if (k >= 2) mbar_wait(smem_addr(&bar_s), (uint32_t)((k - 2) >> 1) & 1u);
         if (k >= 3 && (k & 1)) mbar_wait(smem_addr(&bar_o), (uint32_t)((k - 3) >> 1) & 1u);

@@ -843,6 +843,9 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
                 s_wfail = okw ? 0 : 1;
             }
             __syncthreads();
+            // the product is done: a programmatic dependent (the fused stage's per-sample kernel)
+            // may start its prologue now; it reads nothing of ours before this grid completes
+            asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             // logits (+ bias) into shared memory: warp w < 4 reads the lanes (classes) 32w.. of D
             // (not after a timed-out wait: the product may be incomplete)

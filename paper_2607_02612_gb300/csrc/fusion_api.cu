@@ -155,10 +155,13 @@ constexpr int kTcSmemBudgetKb = 111;
 bool fuse_plan(const fusion_ragged &in) { return in.max_batch >= 1 && in.max_batch <= kFusedPlanMaxBatch; }
 
 // The per-sample kernel: TMA + tcgen05 when the shape allows it, else the general one.
-cudaError_t launch_sample_kernel(int dtype, const ImageParams &p, const ImageGeometry &G, cudaStream_t s) {
+// pdl: the TMA + tcgen05 kernel as a programmatic dependent of the kernel before it (the linear
+// exit check of a fused stage, with no event between them).
+cudaError_t launch_sample_kernel(int dtype, const ImageParams &p, const ImageGeometry &G, cudaStream_t s,
+                                 bool pdl = false) {
     if (p.do_merge) {
         const TcGeometry T = image_tc_geometry(dtype, p.in.max_tokens, p.kdim, p.dim, p.in.max_rows, 1, kTcSmemBudgetKb);
-        if (T.ok) return launch_image_tc(p, T, s);
+        if (T.ok) return launch_image_tc(p, T, s, pdl);
     }
     return launch_image(dtype, p, G.smem, s);
 }
@@ -714,7 +717,8 @@ int stage_impl(int dtype, int flags, const fusion_ragged &in, const void *x, int
                                  dev_status, G);
     p.fused_plan = fuse_plan(in);
     p.plan_args = pa;
-    const int rc = cuda_rc(launch_sample_kernel(dtype, p, G, s));
+    const bool pdl = do_exit && !mlp && ev.mid == nullptr;   // right after the cluster or general exit kernel
+    const int rc = cuda_rc(launch_sample_kernel(dtype, p, G, s, pdl));
     record(ev.end, s);
     return rc;
 }

@@ -210,6 +210,10 @@ __global__ void __launch_bounds__(kTcThreads, 2)
     const int nkb = g.n_kb;
     MetaPtrs m(sm, meta_layout(p.in.max_tokens, g.meta_base));
     uint4 *cls = reinterpret_cast<uint4 *>(sm + g.cls_base);
+    // launched as a programmatic dependent of the exit check: everything above (tensor memory,
+    // barriers, descriptor prefetch) overlaps that kernel's end; the exit mask is read after it
+    // (without a programmatic predecessor this returns at once)
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     SampleInfo s;
     if (!sample_begin<kTcThreads>(p, blockIdx.x, s)) {   // uniform over the CTA
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -443,6 +447,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const CUtensorMap *mp = tid == 32 ? &maps.e32 : tid == 33 ? &maps.o32 : tid == 34 ? &maps.e8 : &maps.o8;
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(mp)) : "memory");
     }
+    asm volatile("griddepcontrol.wait;" ::: "memory");   // as in k_image_tc: the exit check's grid first
     SampleInfo s;
     if (!sample_begin<kTcThreads>(p, blockIdx.x, s)) {
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -759,7 +764,7 @@ TcGeometry image_tc_geometry(int dtype, int max_tokens, int kdim, int dim, long 
     return g;
 }
 
-cudaError_t launch_image_tc(const ImageParams &p, const TcGeometry &g, cudaStream_t s) {
+cudaError_t launch_image_tc(const ImageParams &p, const TcGeometry &g, cudaStream_t s, bool pdl) {
     if (p.in.max_batch == 0) return cudaSuccess;
     EncodeTiledFn enc = encode_fn();
     if (!enc) return cudaErrorNotSupported;
@@ -796,8 +801,17 @@ cudaError_t launch_image_tc(const ImageParams &p, const TcGeometry &g, cudaStrea
     // the largest shared-memory carveout, so that both CTAs of an SM are resident from the start
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     if (e != cudaSuccess) return e;
-    kernel<<<p.in.max_batch, kTcThreads, g.smem, s>>>(maps, p, g);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(p.in.max_batch);
+    cfg.blockDim = dim3(kTcThreads);
+    cfg.dynamicSmemBytes = g.smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kernel, maps, p, g);
 }
 
 }  // namespace fz

@@ -167,6 +167,8 @@ struct TcGeometry {
 };
 TcGeometry image_tc_geometry(int dtype, int max_tokens, int kdim, int dim, long long max_rows, int do_merge,
                              int stage_budget_kb);
-cudaError_t launch_image_tc(const ImageParams &p, const TcGeometry &g, cudaStream_t s);
+// pdl: launched as a programmatic dependent of the kernel before it on the stream (the exit
+// check of a fused stage); the kernel waits for that grid before it reads any input
+cudaError_t launch_image_tc(const ImageParams &p, const TcGeometry &g, cudaStream_t s, bool pdl = false);
 
 }  // namespace fz

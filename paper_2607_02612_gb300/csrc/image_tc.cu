@@ -211,11 +211,11 @@ __global__ void __launch_bounds__(kTcThreads, 2)
     MetaPtrs m(sm, meta_layout(p.in.max_tokens, g.meta_base));
     uint4 *cls = reinterpret_cast<uint4 *>(sm + g.cls_base);
     // launched as a programmatic dependent of the exit check: everything above (tensor memory,
-    // barriers, descriptor prefetch) overlaps that kernel's end; the exit mask is read after it
-    // (without a programmatic predecessor this returns at once)
-    asm volatile("griddepcontrol.wait;" ::: "memory");
+    // barriers, descriptor prefetch) and the plan's loads of this call's own inputs overlap that
+    // kernel's end; the exit mask is read after `griddepcontrol.wait` (without a programmatic
+    // predecessor the wait returns at once)
     SampleInfo s;
-    if (!sample_begin<kTcThreads>(p, blockIdx.x, s)) {   // uniform over the CTA
+    if (!sample_begin<kTcThreads>(p, blockIdx.x, s, true)) {   // uniform over the CTA
         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
         __syncthreads();
         if (warp == 0)

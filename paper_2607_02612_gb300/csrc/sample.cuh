@@ -134,8 +134,11 @@ __device__ __forceinline__ bool sample_info(const ImageParams &p, int i, SampleI
 // batch count is known.  CTA 0 writes the batch-level outputs and raises the status.
 // Must be called by every thread of the CTA.
 
+// dep_wait: the kernel may run as a programmatic dependent of the exit check, whose exit mask
+// is read only after `griddepcontrol.wait`; everything else the plan reads (offsets, ids, merge
+// counts, keep ratios) is this call's input and loads before it.
 template <int NT>
-__device__ bool sample_plan(const ImageParams &p, int i, SampleInfo &s) {
+__device__ bool sample_plan(const ImageParams &p, int i, SampleInfo &s, bool dep_wait = false) {
     const PlanArgs &a = p.plan_args;
     constexpr int kW = NT / 32;
     __shared__ int red[6][kW];
@@ -143,16 +146,24 @@ __device__ bool sample_plan(const ImageParams &p, int i, SampleInfo &s) {
     const int t = threadIdx.x, lane = t & 31, w = t >> 5;
     const int bval = a.in.batch ? *a.in.batch : a.in.max_batch;
     int bad = 0, nf = 0, pre_s = 0, pre_r = 0, tot_s = 0, tot_r = 0;
+    bool waited = !dep_wait;   // uniform
     for (int j0 = 0; j0 < a.in.max_batch; j0 += NT) {
         const int j = j0 + t;
         const bool inb = j < a.in.max_batch;
         const int o0 = inb ? a.in.offsets[j] : 0, o1 = inb ? a.in.offsets[j + 1] : 0;
         const int idr = inb ? (a.in.ids ? a.in.ids[j] : j) : 0;
+        const bool id_ok = idr >= 0 && idr < a.in.max_batch;
+        // merge count and keep ratio by id, for every in-bounds id (used for continuing samples only)
+        const int rr = (inb && id_ok && a.merge) ? a.r[idr] : 0;
+        const float rh = (inb && id_ok && a.prune) ? a.rho[idr] : 0.0f;
+        if (!waited) {
+            asm volatile("griddepcontrol.wait;" ::: "memory");
+            waited = true;
+        }
         const int ex = (inb && a.exit_mask) ? a.exit_mask[j] : 0;
         if (!inb || j >= bval) continue;
         const int N = o1 - o0;
         const bool ok = o0 >= 0 && N >= 1 && N <= a.in.max_tokens && (long long)o1 <= a.in.max_rows;
-        const bool id_ok = idr >= 0 && idr < a.in.max_batch;
         if (!ok) bad |= FUSION_DEV_BAD_OFFSETS;
         if (!id_ok) bad |= FUSION_DEV_BAD_IDS;
         const int surv = ex == 0 ? 1 : 0;
@@ -160,12 +171,12 @@ __device__ bool sample_plan(const ImageParams &p, int i, SampleInfo &s) {
         if (ok && id_ok && surv) {
             int n = N;
             if (a.merge) {
-                rm = merge_count(a.r[idr], N - 1);
+                rm = merge_count(rr, N - 1);
                 n -= rm;
             }
             if (a.prune) {
                 bool f = false;
-                n = 1 + keep_count(a.rho[idr], n - 1, f);
+                n = 1 + keep_count(rh, n - 1, f);
                 if (f) nf = 1;
             }
             cnt = n;
@@ -266,12 +277,15 @@ __device__ __forceinline__ bool gate_open(const int *gate, unsigned spins) {
 // Either the fused plan or the plan kernel's results, once the launch gate (if any) is open;
 // a CTA whose gate wait gives up raises FUSION_DEV_TIMEOUT and writes nothing.
 template <int NT>
-__device__ __forceinline__ bool sample_begin(const ImageParams &p, int i, SampleInfo &s) {
+// dep_wait: see sample_plan; without the fused plan the wait comes first (the plan's results may be
+// the predecessor's output).
+__device__ __forceinline__ bool sample_begin(const ImageParams &p, int i, SampleInfo &s, bool dep_wait = false) {
     if (p.gate && !gate_open(p.gate, p.gate_spins)) {
         if (threadIdx.x == 0) raise_status(p.status, FUSION_DEV_TIMEOUT);
         return false;
     }
-    return p.fused_plan ? sample_plan<NT>(p, i, s) : sample_info(p, i, s);
+    if (dep_wait && !p.fused_plan) asm volatile("griddepcontrol.wait;" ::: "memory");
+    return p.fused_plan ? sample_plan<NT>(p, i, s, dep_wait) : sample_info(p, i, s);
 }
 
 template <int NT>

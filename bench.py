@@ -66,7 +66,6 @@ def parse_args():
     ap.add_argument("--e2e-steps", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--eager", action="store_true", help="launch every step from the host instead of a CUDA graph")
-    ap.add_argument("--ref-sample", type=int, default=16, help="images per reference step")
     return ap.parse_args()
 
 
@@ -223,30 +222,38 @@ def stage_bytes(spec, dtype, dim, in_off, in_ids, out_off, out_ids, classes, row
 # reference arm: the CPU oracle
 # ---------------------------------------------------------------------------
 def run_reference(args, world, rank):
+    """The oracle as it stands, on the host cores: every step covers the workload's whole batch,
+    split into one seeded shard per core (one spawned process each, images are independent)."""
     if rank != 0:
         return 0
-    import oracle
+    import multiprocessing as mp
     from workloads import make_workload
     w = make_workload(args.workload)
-    n = min(args.ref_sample, w.batch.batch)
-    sub = make_workload(args.workload, batch=n)
+    n = w.batch.batch
+    procs = max(1, min(os.cpu_count() or 1, n))
+    shard = [n // procs + (1 if k < n % procs else 0) for k in range(procs)]
+    ctx = mp.get_context("spawn")
     units = 0
     t_total = 0.0
-    for k in range(args.warmup + args.steps):
-        t0 = time.perf_counter()
-        res = oracle.chain(sub)
-        dt = time.perf_counter() - t0
-        if k >= args.warmup:
-            t_total += dt
-            units += n + sum(int(r["n_out"]) for r in res[:-1])
+    with ctx.Pool(procs) as pool:
+        pool.map(_oracle_shard, [(args.workload, 1, 1000 + k) for k in range(procs)])   # workers up
+        for step in range(args.warmup + args.steps):
+            jobs = [(args.workload, shard[k], 3000 + 97 * step + k) for k in range(procs)]
+            t0 = time.perf_counter()
+            outs = pool.map(_oracle_shard, jobs)
+            dt = time.perf_counter() - t0
+            if step >= args.warmup:
+                t_total += dt
+                units += sum(u for u, _ in outs)
     value = units / t_total if t_total > 0 else 0.0
-    sample = f"{n} of {w.batch.batch} images per step, full {len(w.stages)}-stage schedule, one thread"
+    sample = (f"the whole batch of {n} images per step as {procs} seeded shards of {min(shard)}-{max(shard)} images, "
+              f"one process per host core, full {len(w.stages)}-stage schedule each")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t_total / max(args.steps, 1),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "f64", "data": "synthetic",
-            "config": {"workload": args.workload, "batch": w.batch.batch, "sample_batch": n},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+            "config": {"workload": args.workload, "batch": n, "sample_batch": n, "shards": procs},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": procs, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     return 0

@@ -387,6 +387,11 @@ int fusion_token_scores(int dtype, fusion_ragged in, const void *x, int32_t dim,
  * as in fusion_compact; a_match [in.max_rows] as in fusion_merge (may be NULL).
  * ids_out and batch_out are written with every flag combination, so the
  * outputs always describe the next block's input batch.
+ * With EXIT and the linear head, the per-sample kernel is launched as a
+ * programmatic dependent of the exit kernel (its CTAs may become resident while
+ * the exit check finishes and read the exit mask only once it has completed);
+ * the call's work still runs in stream order with respect to other work on the
+ * stream.
  */
 int fusion_stage(int dtype, int flags, fusion_ragged in, const void *x, int32_t dim,
                  const void *keys, int32_t key_dim, const float *sizes, const float *scores,

@@ -6,9 +6,9 @@
 //
 // Two kernels.  The cluster kernel (heads of at most 8 class tiles) is described below.
 // The general one: grid (class tiles of kExitCT) x (sample tiles of kExitBT).  Every CTA computes
-// the LayerNorm of its samples' CLS rows, one logits tile (bf16: mma.sync tensor
-// cores with float32 accumulation; f32: FFMA) and a partial softmax (tile max and
-// sum of exponentials) per sample.  The last CTA of a sample tile to finish
+// the LayerNorm of its samples' CLS rows, one logits tile (bf16: the weight tile by TMA and one
+// tcgen05 product D[128 classes][16 samples] in tensor memory; f32: FFMA) and a partial softmax
+// (tile max and sum of exponentials) per sample.  The last CTA of a sample tile to finish
 // (atomic counter, no waiting) merges the partials into c and the exit mask; the
 // last sample tile to finish runs the compaction plan for the fused stage.
 #include <cooperative_groups.h>
@@ -22,16 +22,11 @@ namespace cg = cooperative_groups;
 namespace fz {
 namespace {
 
-// Head K chunk staged in shared memory (two stages): 128 dims for bf16, 64 for f32.
+// Head K chunk of the float32 kernels' two cp.async weight stages: 64 dims (bf16 heads arrive by
+// TMA in 64-dim stages, kExitWStage; their entry here only sizes the unused float32 layout).
 template <typename T> struct ExitKC;
 template <> struct ExitKC<__nv_bfloat16> { static constexpr int v = 128; };
 template <> struct ExitKC<float> { static constexpr int v = 64; };
-
-template <typename T> __device__ __forceinline__ T from_float(float v);
-template <> __device__ __forceinline__ float from_float<float>(float v) { return v; }
-template <> __device__ __forceinline__ __nv_bfloat16 from_float<__nv_bfloat16>(float v) {
-    return __float2bfloat16_rn(v);
-}
 
 template <typename T>
 __device__ __forceinline__ void issue_w_chunk(const ExitParams &p, unsigned char *stage_buf, int c0, int k0,
@@ -54,6 +49,97 @@ __device__ __forceinline__ void issue_w_chunk(const ExitParams &p, unsigned char
     cp_async_commit();
 }
 
+// ---- the bf16 product of both kernels on tcgen05 ---------------------------------------
+constexpr uint32_t kExitWStage = kExitCT * 128u;     // one weight stage: kExitCT rows x 64 bf16 dims
+
+// Byte offset of 16-byte chunk c (8 bf16 dims) of row r in a bf16 u tile: K-blocks of 64 dims,
+// each [16 rows][128 bytes] with chunk j of row r at j ^ (r % 8), the K-major,
+// 128-byte-swizzled layout of a tcgen05 operand (8-row groups 1024 bytes apart).
+__device__ __forceinline__ uint32_t u_tc_off(int r, int c) {
+    return (uint32_t)(c >> 3) * 2048u + (uint32_t)r * 128u + ((uint32_t)((c & 7) ^ (r & 7)) << 4);
+}
+constexpr uint32_t kExitTmemCols = 32;   // D: 128 classes (lanes) x 16 samples (columns)
+constexpr int kExitClMaxW = 16;          // most weight stages of a bf16 kernel
+constexpr size_t kExitClBudget = 112 * 1024;   // the cluster kernel's dynamic shared memory bound (two CTAs per SM)
+// the general kernel's bound: two CTAs per SM with its larger static shared memory
+constexpr size_t kExitTcBudget = 110 * 1024;
+
+// Instruction descriptor of D[128][16] (float32) += A[128][16] B[16][16]^T, A and B bf16, K-major.
+constexpr uint32_t kExitIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(16 >> 3) << 17) | (8u << 24);
+
+// The general kernel's bf16 shared memory, offsets from a 1024-byte aligned base: the u tile
+// (u_tc_off; 16 rows, rows 8..15 zero) | the weight ring (w_stages TMA stages, the whole tile when
+// it fits) | the bias tile.  The logits tile [kExitBT][kExitCT] reuses the ring after the product.
+struct ExitTcSmem {
+    static __host__ __device__ size_t u_bytes(int dim) { return (size_t)((dim + 63) / 64) * 2048; }
+    static __host__ __device__ int w_stages(int dim) {
+        const int nk = (dim + 63) / 64;
+        const size_t rest = u_bytes(dim) + kExitCT * sizeof(float) + 1024;
+        int st = rest + 2 * kExitWStage <= kExitTcBudget ? (int)((kExitTcBudget - rest) / kExitWStage) : 2;
+        st = st < kExitClMaxW ? st : kExitClMaxW;
+        return nk < st ? nk : st;
+    }
+    static __host__ __device__ size_t w_off(int dim) { return u_bytes(dim); }
+    static __host__ __device__ size_t bias_off(int dim) { return w_off(dim) + (size_t)w_stages(dim) * kExitWStage; }
+    static __host__ __device__ size_t total(int dim) {
+        const size_t t = bias_off(dim) + kExitCT * sizeof(float);
+        const size_t plan = plan_smem_bytes(kExitThreads);   // run_plan reuses the buffer from its start
+        return (t > plan ? t : plan) + 1024;
+    }
+};
+
+// D[128 classes][16 samples] = W_tile u^T on tcgen05, by one thread: per 64-dim K-block, wait
+// for its weight stage (stages 0..nws-1 already issued), four MMAs (K = 16; fewer in a short
+// last block), commit; when the tile is not resident, the stage of the block before is
+// refilled by TMA once its MMAs completed (one block late, so that the wait overlaps the
+// products just issued).  Every wait is bounded; after a failure the copies and products in
+// flight are waited for (bounded) and FUSION_DEV_TIMEOUT is raised.  Returns whether D is
+// complete.
+__device__ __forceinline__ bool exit_tc_product(const CUtensorMap *wmap, uint32_t tmem, uint32_t ub, uint32_t wr,
+                                                int dim, int nws, int c0, unsigned long long *wbar,
+                                                unsigned long long *wempty, unsigned long long *wdone, int *status) {
+    const int nk = (dim + 63) / 64;
+    bool okw = true;
+    int waited = 0, issued = 0, loaded = nws;
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    for (int kc = 0; kc < nk; ++kc) {
+        const int st = kc % nws;
+        const uint32_t ph = (uint32_t)(kc / nws) & 1u;
+        if (!mbar_wait(smem_addr(&wbar[st]), ph)) {
+            okw = false;
+            break;
+        }
+        waited = kc + 1;
+        const uint32_t a0 = wr + (uint32_t)st * kExitWStage, b0 = ub + (uint32_t)kc * 2048u;
+        const int kw = min(64, dim - kc * 64);
+        for (int k = 0; k * 16 < kw; ++k)
+            umma_bf16(tmem, sw128_desc(a0 + k * 32), sw128_desc(b0 + k * 32), kExitIdesc, (kc | k) ? 1u : 0u);
+        umma_commit(smem_addr(&wempty[st]));
+        issued = kc + 1;
+        const int kp = kc - 1;   // the block before; its stage next holds block kp + nws
+        if (kp >= 0 && kp + nws < nk) {
+            const int sp = kp % nws;
+            if (!mbar_wait(smem_addr(&wempty[sp]), (uint32_t)(kp / nws) & 1u)) {
+                okw = false;
+                break;
+            }
+            mbar_expect_tx(smem_addr(&wbar[sp]), kExitWStage);
+            tma_load_2d(wr + (uint32_t)sp * kExitWStage, wmap, (kp + nws) * 64, c0, smem_addr(&wbar[sp]));
+            loaded = kp + nws + 1;
+        }
+    }
+    if (okw) {
+        umma_commit(smem_addr(wdone));
+        okw = mbar_wait(smem_addr(wdone), 0u);
+    }
+    if (!okw) {
+        for (int q = waited; q < loaded; ++q) (void)mbar_wait(smem_addr(&wbar[q % nws]), (uint32_t)(q / nws) & 1u);
+        if (issued > 0) (void)mbar_wait(smem_addr(&wempty[(issued - 1) % nws]), (uint32_t)((issued - 1) / nws) & 1u);
+        raise_status(status, FUSION_DEV_TIMEOUT);
+    }
+    return okw;
+}
+
 template <typename T>
 struct ExitSmem {
     static constexpr int EB = Elem<T>::kBytes;
@@ -69,15 +155,14 @@ struct ExitSmem {
     }
 };
 
-// The logits tile [kExitBT samples] x [kExitCT classes] of one CTA, K chunks of the head
-// double-buffered (chunks 0 and 1 already in flight): bf16 mma.sync with float32
-// accumulation, f32 FFMA.  u_s holds the LayerNorm rows (16 rows for the bf16 A tile).
+// The float32 logits tile [kExitBT samples] x [kExitCT classes] of one CTA by FFMA, K chunks of
+// the head double-buffered (chunks 0 and 1 already in flight); u_s holds the LayerNorm rows.
 template <typename T>
 __device__ __forceinline__ void exit_gemm(const ExitParams &p, const T *u_s, unsigned char *w_region, int c0, int dim,
-                                          int C, int n_k, float (&acc)[4], float (&acc2)[4]) {
+                                          int C, int n_k, float (&acc)[4]) {
+    static_assert(sizeof(T) == 4, "bf16 heads take the tcgen05 product");
     using S = ExitSmem<T>;
     constexpr int KC = S::KC;
-    constexpr bool kBf16 = (Elem<T>::kBytes == 2);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int u_stride = S::u_stride(dim);
     for (int kc = 0; kc < n_k; ++kc) {
@@ -89,120 +174,92 @@ __device__ __forceinline__ void exit_gemm(const ExitParams &p, const T *u_s, uns
         else
             cp_async_wait_all();
         __syncthreads();
-        if constexpr (kBf16) {
-            // warp -> the 16-row sample tile (rows 8..15 are zero) x 16 classes
-            float t0[4] = {0.0f, 0.0f, 0.0f, 0.0f}, t1[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-            const uint32_t ubase = smem_addr(u_s);
-            const uint32_t wbase = smem_addr(wbuf);
-            const int arow = (lane & 7) + ((lane >> 3) & 1) * 8;
-            const int brow = warp * 16 + (lane >> 4) * 8 + (lane & 7);
-            for (int kk = 0; kk < kw; kk += 16) {
-                uint32_t af[4], b0, b1, b2, b3;
-                ldsm_x4(ubase + (uint32_t)((arow * u_stride + k0 + kk + (lane >> 4) * 8) * 2), af[0], af[1],
-                        af[2], af[3]);
-                ldsm_x4(wbase + (uint32_t)((brow * S::w_stride + kk + ((lane >> 3) & 1) * 8) * 2), b0, b1, b2, b3);
-                mma_bf16_16816(t0, af, b0, b1);
-                mma_bf16_16816(t1, af, b2, b3);
-                if ((kk & 63) == 48) {   // flush the partial sums every 64 dims
+        // warp -> sample `warp`; lane -> classes lane + 32 q
+        const float *ur = reinterpret_cast<const float *>(u_s) + (size_t)warp * u_stride + k0;
+        const float *ws = reinterpret_cast<const float *>(wbuf);
+        float t[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        for (int kk = 0; kk < kw; kk += 4) {
+            const float4 uv = *reinterpret_cast<const float4 *>(ur + kk);
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        acc[e] += t0[e];
-                        acc2[e] += t1[e];
-                        t0[e] = t1[e] = 0.0f;
-                    }
-                }
+            for (int q = 0; q < 4; ++q) {
+                const float4 wv = *reinterpret_cast<const float4 *>(ws + (lane + 32 * q) * S::w_stride + kk);
+                t[q] = fmaf(uv.x, wv.x, t[q]);
+                t[q] = fmaf(uv.y, wv.y, t[q]);
+                t[q] = fmaf(uv.z, wv.z, t[q]);
+                t[q] = fmaf(uv.w, wv.w, t[q]);
             }
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                acc[e] += t0[e];
-                acc2[e] += t1[e];
-            }
-        } else {
-            // warp -> sample `warp`; lane -> classes lane + 32 q
-            const float *ur = reinterpret_cast<const float *>(u_s) + (size_t)warp * u_stride + k0;
-            const float *ws = reinterpret_cast<const float *>(wbuf);
-            float t[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-            for (int kk = 0; kk < kw; kk += 4) {
-                const float4 uv = *reinterpret_cast<const float4 *>(ur + kk);
+            if ((kk & 15) == 12) {   // flush every 16 dims
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
-                    const float4 wv = *reinterpret_cast<const float4 *>(ws + (lane + 32 * q) * S::w_stride + kk);
-                    t[q] = fmaf(uv.x, wv.x, t[q]);
-                    t[q] = fmaf(uv.y, wv.y, t[q]);
-                    t[q] = fmaf(uv.z, wv.z, t[q]);
-                    t[q] = fmaf(uv.w, wv.w, t[q]);
-                }
-                if ((kk & 15) == 12) {   // flush every 16 dims
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        acc[q] += t[q];
-                        t[q] = 0.0f;
-                    }
+                    acc[q] += t[q];
+                    t[q] = 0.0f;
                 }
             }
-#pragma unroll
-            for (int q = 0; q < 4; ++q) acc[q] += t[q];
         }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) acc[q] += t[q];
         __syncthreads();   // everyone is done with this stage buffer
         if (kc + 2 < n_k) issue_w_chunk<T>(p, wbuf, c0, k0 + 2 * KC, dim, C, tid);
     }
 }
 
-// Logits (+ bias) into shared memory (padded classes get -inf) and to p.logits.
-template <typename T>
-__device__ __forceinline__ void exit_logits(const ExitParams &p, float *lg_s, const float *bias_s, const float (&acc)[4],
-                                            const float (&acc2)[4], int s0, int c0, int B, int C) {
-    constexpr bool kBf16 = (Elem<T>::kBytes == 2);
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    // ---- logits (+ bias) into shared memory; padded classes get -inf ---------------
-    if constexpr (kBf16) {
-        const int g = lane >> 2, t4 = lane & 3;   // fragment rows g (valid) and g + 8 (padding)
+// The float32 logits (+ bias) into shared memory; padded classes get -inf.
+__device__ __forceinline__ void exit_logits_f32(float *lg_s, const float *bias_s, const float (&acc)[4], int c0, int C) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            const int col0 = warp * 16 + 2 * t4 + e, col1 = col0 + 8;
-            lg_s[g * kExitCT + col0] = (c0 + col0 < C) ? acc[e] + bias_s[col0] : -INFINITY;
-            lg_s[g * kExitCT + col1] = (c0 + col1 < C) ? acc2[e] + bias_s[col1] : -INFINITY;
-        }
-    } else {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const int col = lane + 32 * q;
-            lg_s[warp * kExitCT + col] = (c0 + col < C) ? acc[q] + bias_s[col] : -INFINITY;
-        }
-    }
-    __syncthreads();
-    if (p.lg_tmp) {   // staged: the last CTA of the sample tile writes the rows of the samples that exit
-        for (int it = tid; it < kExitBT * kExitCT; it += kExitThreads) {
-            const int sl = it / kExitCT, col = it - sl * kExitCT;
-            if (s0 + sl < B && c0 + col < C) p.lg_tmp[(size_t)(s0 + sl) * C + c0 + col] = lg_s[it];
-        }
+    for (int q = 0; q < 4; ++q) {
+        const int col = lane + 32 * q;
+        lg_s[warp * kExitCT + col] = (c0 + col < C) ? acc[q] + bias_s[col] : -INFINITY;
     }
 }
 
-// Error scale of a hidden unit's pre-activation from the product above (bf16 mma.sync,
-// float32 sums flushed every 64 dims): about sqrt(30) roundings of at most 2^-24 relative to
-// partial sums bounded by sum |w u| <= ||w|| ||u||; the typical partial sum is far below that
-// bound, so 2^-22 ||w|| ||u|| is more than 8 standard deviations of the accumulated error.
+// The logits tile in shared memory (complete: after a barrier) to the staging rows lg_tmp, from
+// which the last CTA of the sample tile writes the rows of the samples that exit.
+__device__ __forceinline__ void exit_stage_logits(const ExitParams &p, const float *lg_s, int s0, int c0, int B, int C) {
+    if (!p.lg_tmp) return;
+    for (int it = threadIdx.x; it < kExitBT * kExitCT; it += kExitThreads) {
+        const int sl = it / kExitCT, col = it - sl * kExitCT;
+        if (s0 + sl < B && c0 + col < C) p.lg_tmp[(size_t)(s0 + sl) * C + c0 + col] = lg_s[it];
+    }
+}
+
+// Error scale of a hidden unit's pre-activation a from the tcgen05 product: the bf16 products are
+// exact and every K = 16 step adds them into the float32 accumulator, n = dim / 16 steps, each
+// with an error below one float32 ulp (2^-23) of its partial sum, truncation included.  For
+// partial sums of mixed signs the k-th is typically about sqrt(16 k / dim) ||w|| ||u|| / sqrt(dim),
+// and even n errors of one sign at that size sum to about (sqrt(n) / 6) 2^-23 ||w|| ||u||, below
+// 2^-22 ||w|| ||u|| up to dim = 1024.  Where the products share a sign, the partial sums grow
+// monotonically up to |a|: the second term, n 2^-23 |a|, covers that case.
 constexpr float kHidErr = 0x1p-22f;
 
-// One hidden unit exactly, by a whole warp: a = w . u + b1 from exact bf16 x bf16 products
-// summed in float-float (each lane a slice of the dims, then a butterfly), GELU in double in the
-// erf form, rounded once to bf16.  Every lane returns the result.
-__device__ __forceinline__ uint16_t hidden_exact_bf16_warp(const __nv_bfloat16 *w, const __nv_bfloat16 *u, int dim,
-                                                           float b1) {
+// The exact pre-activation a = w . u + b1 of one hidden unit, by a whole warp: exact bf16 x bf16
+// products summed in float-float (each lane a slice of the dims, then a butterfly).  The row u is
+// row `row` of a u tile in shared memory (u_tc_off layout); the weight row is row wr of the
+// resident weight ring wt (K-block q in stage q, TMA's 128-byte swizzle: chunk j of row r at
+// j ^ (r % 8)) or, with wt NULL, the global row wg.  Every lane returns the result.
+__device__ __forceinline__ F2 hidden_dot_exact_warp(const unsigned char *wt, int wr, const __nv_bfloat16 *wg,
+                                                    const unsigned char *ut, int row, int dim, float b1) {
     const int lane = threadIdx.x & 31;
     F2 acc = {0.0f, 0.0f};
     for (int c = lane * 8; c < dim; c += 256) {
         float wf[8], uf[8];
-        chunk_to_f(ldg16(w + c), wf);
-        chunk_to_f(*reinterpret_cast<const uint4 *>(u + c), uf);
+        const int ch = c >> 3;
+        chunk_to_f(wt ? *reinterpret_cast<const uint4 *>(wt + (size_t)(ch >> 3) * kExitWStage + (size_t)wr * 128 +
+                                                         (((ch & 7) ^ (wr & 7)) << 4))
+                      : ldg16(wg + c),
+                   wf);
+        chunk_to_f(*reinterpret_cast<const uint4 *>(ut + u_tc_off(row, ch)), uf);
 #pragma unroll
         for (int e = 0; e < 8; ++e) acc = f2_add_f(acc, __fmul_rn(wf[e], uf[e]));
     }
-    acc = f2_add_f(warp_sum_f2(acc), b1);
-    // with the product exact, the float GELU of its high part is within about a hundred float
-    // ulps of the exact value (erfc's error, amplified by its argument for large |a|); only a
-    // unit closer than that to a bf16 midpoint needs double precision
+    return f2_add_f(warp_sum_f2(acc), b1);
+}
+
+// GELU of an exact pre-activation (float-float) rounded once to bf16, by one thread: with the
+// argument exact, the float GELU of its high part is within about a hundred float ulps of the
+// exact value (erfc's error, amplified by its argument for large |a|); only a unit closer than
+// that to a bf16 midpoint is evaluated in double, in the erf form.
+__device__ __forceinline__ uint16_t gelu_exact_bf16(F2 acc) {
     const float g2 = 0.5f * acc.hi * erfcf(-acc.hi * 0.70710678118654752f);
     const float mid = __uint_as_float((__float_as_uint(g2) & 0xFFFF0000u) | 0x8000u);
     if (isfinite(g2) && fabsf(g2 - mid) > fabsf(g2) * 0x1p-17f) return __bfloat16_as_ushort(__float2bfloat16_rn(g2));
@@ -212,9 +269,13 @@ __device__ __forceinline__ uint16_t hidden_exact_bf16_warp(const __nv_bfloat16 *
 }
 
 template <typename T>
-__global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
+__global__ void __launch_bounds__(kExitThreads) k_exit(const __grid_constant__ CUtensorMap wmap, ExitParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
+    __shared__ __align__(8) unsigned long long wbar[kExitClMaxW], wempty[kExitClMaxW], wdone;
+    __shared__ int s_wfail;
+    __shared__ uint32_t tmem_base;
     using S = ExitSmem<T>;
+    using TS = ExitTcSmem;
     constexpr int CH = Elem<T>::kPerChunk;
     constexpr int EB = Elem<T>::kBytes;
     constexpr int KC = S::KC;
@@ -222,10 +283,19 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
     const int dim = p.dim;
     const int nchunk = dim / CH;
     const int u_stride = S::u_stride(dim);
-    T *u_s = reinterpret_cast<T *>(sm);                   // 16 rows: CLS rows, then LayerNorm outputs
-    unsigned char *w_region = sm + S::u_bytes(dim);
-    float *lg_s = reinterpret_cast<float *>(w_region);    // [kExitBT][kExitCT], reused after the GEMM
-    float *bias_s = reinterpret_cast<float *>(w_region + 2 * S::w_stage);
+    // bf16: offsets from a 1024-byte aligned base (ExitTcSmem); float32: the u tile [16][u_stride]
+    // | two cp.async weight stages | bias
+    unsigned char *base = kBf16 ? reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(sm) + 1023) &
+                                                                    ~uintptr_t(1023))
+                                : sm;
+    T *u_s = reinterpret_cast<T *>(base);   // 16 rows: CLS rows, then LayerNorm outputs
+    // chunk c (CH dims) of row r of the u tile (bf16: the tcgen05 operand layout u_tc_off)
+    auto uchunk = [&](int r, int c) -> T * {
+        return kBf16 ? reinterpret_cast<T *>(base + u_tc_off(r, c)) : u_s + (size_t)r * u_stride + c * CH;
+    };
+    unsigned char *w_region = base + (kBf16 ? TS::w_off(dim) : S::u_bytes(dim));
+    float *lg_s = reinterpret_cast<float *>(w_region);    // [kExitBT][kExitCT], reused after the product
+    float *bias_s = reinterpret_cast<float *>(kBf16 ? base + TS::bias_off(dim) : w_region + 2 * S::w_stage);
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int ct = blockIdx.x, bt = blockIdx.y;
@@ -236,17 +306,42 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
     const bool active = s0 < B;
     const int n_k = (dim + KC - 1) / KC;
 
-    // weight chunks 0 and 1, the CLS rows and the bias tile load together
+    // the weight tile (bf16: TMA stages, the whole tile when it fits; float32: chunks 0 and 1), the
+    // CLS rows and the bias tile load together
     if (active) {
-        issue_w_chunk<T>(p, w_region, c0, 0, dim, C, tid);
-        if (n_k > 1) issue_w_chunk<T>(p, w_region + S::w_stage, c0, KC, dim, C, tid);
+        if constexpr (kBf16) {
+            if (tid == 0) s_wfail = 0;
+            if (warp == 0) {   // the logits tile's accumulator
+                asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                                 smem_addr(&tmem_base)),
+                             "r"(kExitTmemCols)
+                             : "memory");
+                asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+            }
+            if (tid == 0) {
+                const int nws = TS::w_stages(dim);
+                for (int q = 0; q < nws; ++q) {
+                    mbar_init(smem_addr(&wbar[q]), 1);
+                    mbar_init(smem_addr(&wempty[q]), 1);
+                }
+                mbar_init(smem_addr(&wdone), 1);
+                asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+                for (int q = 0; q < nws; ++q) {
+                    mbar_expect_tx(smem_addr(&wbar[q]), kExitWStage);
+                    tma_load_2d(smem_addr(w_region + (size_t)q * kExitWStage), &wmap, q * 64, c0, smem_addr(&wbar[q]));
+                }
+            }
+        } else {
+            issue_w_chunk<T>(p, w_region, c0, 0, dim, C, tid);
+            if (n_k > 1) issue_w_chunk<T>(p, w_region + S::w_stage, c0, KC, dim, C, tid);
+        }
         // launched as a programmatic dependent of the kernel before it (the MLP head's layers):
         // the weights above are this call's own input; the rows below may be that kernel's output
         asm volatile("griddepcontrol.wait;" ::: "memory");
         for (int it = tid; it < 16 * nchunk; it += kExitThreads) {
             const int sl = it / nchunk, c = it - sl * nchunk;
             const int s = s0 + sl;
-            T *dst = u_s + (size_t)sl * u_stride + c * CH;
+            T *dst = uchunk(sl, c);
             long long row = -1;   // in_mode 2: the LayerNorm reads u_in and fills the tile
             if (sl < kExitBT && s < B && p.in_mode != 2) {
                 row = p.in_mode == 0 ? (long long)p.in.offsets[s] : (long long)s;
@@ -272,7 +367,6 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
                 ok = false;
             }
         }
-        T *xr = u_s + (size_t)warp * u_stride;
         // the row's chunk c as floats: from the tile, or from the float32 input rows
         const float *ur = p.in_mode == 2 && ok ? p.u_in + (size_t)s * dim : nullptr;
         const float *url = ur && p.u_in_lo ? p.u_in_lo + (size_t)s * dim : nullptr;   // float-float low parts
@@ -297,7 +391,7 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
                     f[e + 3] = v.w;
                 }
             } else {
-                chunk_to_f(*reinterpret_cast<const uint4 *>(xr + c * CH), f);
+                chunk_to_f(*reinterpret_cast<const uint4 *>(uchunk(warp, c)), f);
             }
         };
         if (ok && !p.skip_ln) {
@@ -356,57 +450,89 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
                             w4[q] = (uint32_t)ln_out_bf16(f[2 * q], mean, rstd, gf[2 * q], bf[2 * q]) |
                                     ((uint32_t)ln_out_bf16(f[2 * q + 1], mean, rstd, gf[2 * q + 1], bf[2 * q + 1]) << 16);
                     }
-                    *reinterpret_cast<uint4 *>(xr + c * CH) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
+                    *reinterpret_cast<uint4 *>(uchunk(warp, c)) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
                 } else {
                     float4 o;
                     o.x = url ? ln_out_f32_lo(f[0], fl[0], mean, rstd, gf[0], bf[0]) : ln_out_f32(f[0], mean, rstd, gf[0], bf[0]);
                     o.y = url ? ln_out_f32_lo(f[1], fl[1], mean, rstd, gf[1], bf[1]) : ln_out_f32(f[1], mean, rstd, gf[1], bf[1]);
                     o.z = url ? ln_out_f32_lo(f[2], fl[2], mean, rstd, gf[2], bf[2]) : ln_out_f32(f[2], mean, rstd, gf[2], bf[2]);
                     o.w = url ? ln_out_f32_lo(f[3], fl[3], mean, rstd, gf[3], bf[3]) : ln_out_f32(f[3], mean, rstd, gf[3], bf[3]);
-                    *reinterpret_cast<float4 *>(xr + c * CH) = o;
+                    *reinterpret_cast<float4 *>(uchunk(warp, c)) = o;
                 }
             }
         } else if (!ok) {   // (skip_ln: the loaded rows stay as they are)
-            for (int c = lane; c < nchunk; c += 32) *reinterpret_cast<uint4 *>(xr + c * CH) = make_uint4(0, 0, 0, 0);
+            for (int c = lane; c < nchunk; c += 32) *reinterpret_cast<uint4 *>(uchunk(warp, c)) = make_uint4(0, 0, 0, 0);
         }
     }
+    // bf16: the u tile, written by the generic proxy (stores and cp.async), is read by the tensor
+    // core (async proxy) after the barrier
+    if constexpr (kBf16) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     __syncthreads();
 
-    // ---- logits tile [kExitBT samples] x [kExitCT classes], K chunks double-buffered ----
-    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};   // bf16: two m16n8 fragments' valid rows; f32: 4 classes
-    float acc2[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    // ---- logits tile [kExitBT samples] x [kExitCT classes] -----------------------------
+    // GELU(a) = a (1 + erf(a / sqrt 2)) / 2 = a erfc(-a / sqrt 2) / 2 for the hidden layer of an MLP
+    // head; the erfc form is accurate in float for both signs.  bf16: a unit whose GELU lies within
+    // the error scale of the product (kHidErr ||w_j|| ||u|| + n 2^-23 |a|, and the bias addition)
+    // plus that of the float evaluation of a bf16 rounding midpoint is evaluated again exactly: the
+    // dot product in float-float from exact bf16 x bf16 products, GELU in double.
+    bool failed = false;   // bf16: a bounded wait of the product ran out (status raised; no output)
     if (active) {
-        exit_gemm<T>(p, u_s, w_region, c0, dim, C, n_k, acc, acc2);
-        exit_logits<T>(p, lg_s, bias_s, acc, acc2, s0, c0, B, C);
-        if (p.out_mode == 1) {
-            // ---- hidden layer of an MLP head: GELU, rounded to the dtype ----------------------
-            // GELU(a) = a (1 + erf(a / sqrt 2)) / 2 = a erfc(-a / sqrt 2) / 2; the erfc form is
-            // accurate in float for both signs.  bf16: a unit whose GELU lies within the error
-            // scale of the product above (kHidErr ||w_j|| ||u||, Cauchy-Schwarz on sum |w u|) plus
-            // that of the float evaluation of a bf16 rounding midpoint is evaluated again exactly:
-            // the dot product in float-float from exact bf16 x bf16 products, GELU in double.
-            __shared__ float wn2[2][kExitCT], un[kExitBT];
-            if constexpr (kBf16) {
-                {   // ||w_j||^2 of this tile's rows, two threads per row
+        if constexpr (kBf16) {
+            const uint32_t tmem = tmem_base;
+            const int nws = TS::w_stages(dim);
+            if (tid == 0)
+                s_wfail = exit_tc_product(&wmap, tmem, smem_addr(base), smem_addr(w_region), dim, nws, c0, wbar,
+                                          wempty, &wdone, p.status)
+                              ? 0
+                              : 1;
+            __syncthreads();
+            // the product is done: a programmatic dependent (the MLP head's next layer) may start its
+            // prologue now; it reads nothing of ours before this grid completes
+            asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            failed = s_wfail != 0;
+            if (p.out_mode == 1) {
+                // ---- hidden layer: a = D + b1 straight from tensor memory, the weight ring intact ----
+                __shared__ float wn2[2][kExitCT], un[kExitBT];   // ||w_j||^2 in two halves; ||u||
+                const bool resident = nws * 64 >= dim;           // every K-block in its own stage
+                {   // ||w_j||^2, two threads per row: from the ring (a row's 8 chunks in any order; rows
+                    // past C and dims past dim are zero), else from global memory, 8 loads at a time
                     const int r = tid & (kExitCT - 1), h = tid / kExitCT;
                     float acc = 0.0f;
-                    if (c0 + r < C) {
-                        const T *wr = reinterpret_cast<const T *>(p.head.weight) + (size_t)(c0 + r) * dim;
-                        for (int c = h; c < nchunk; c += 2) {
-                            float f[CH];
-                            chunk_to_f(ldg16(wr + c * CH), f);
+                    if (resident) {
+                        for (int q = h; q < nws; q += 2) {
+                            const unsigned char *row = w_region + (size_t)q * kExitWStage + (size_t)r * 128;
 #pragma unroll
-                            for (int e = 0; e < CH; ++e) acc = fmaf(f[e], f[e], acc);
+                            for (int j2 = 0; j2 < 8; ++j2) {
+                                float f[8];
+                                chunk_to_f(*reinterpret_cast<const uint4 *>(row + 16 * j2), f);
+#pragma unroll
+                                for (int e = 0; e < 8; ++e) acc = fmaf(f[e], f[e], acc);
+                            }
+                        }
+                    } else if (c0 + r < C) {
+                        const T *wr = reinterpret_cast<const T *>(p.head.weight) + (size_t)(c0 + r) * dim;
+                        for (int cb = h; cb < nchunk; cb += 16) {
+                            uint4 v[8];
+#pragma unroll
+                            for (int q = 0; q < 8; ++q)
+                                v[q] = cb + 2 * q < nchunk ? ldg16(wr + (cb + 2 * q) * CH) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+                            for (int q = 0; q < 8; ++q) {
+                                float f[CH];
+                                chunk_to_f(v[q], f);
+#pragma unroll
+                                for (int e = 0; e < CH; ++e) acc = fmaf(f[e], f[e], acc);
+                            }
                         }
                     }
                     wn2[h][r] = acc;
                 }
                 {   // ||u||^2 of each sample's row (warp -> sample slot)
-                    const T *ur = u_s + (size_t)warp * u_stride;
                     float acc = 0.0f;
                     for (int c = lane; c < nchunk; c += 32) {
                         float f[CH];
-                        chunk_to_f(*reinterpret_cast<const uint4 *>(ur + c * CH), f);
+                        chunk_to_f(*reinterpret_cast<const uint4 *>(uchunk(warp, c)), f);
 #pragma unroll
                         for (int e = 0; e < CH; ++e) acc = fmaf(f[e], f[e], acc);
                     }
@@ -415,36 +541,89 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
                     if (lane == 0) un[warp] = sqrtf(acc);
                 }
                 __syncthreads();
-            }
-            T *ho = reinterpret_cast<T *>(p.hidden_out);
-            // every warp takes 32 consecutive units of one sample slot per round (uniform trip count)
-            for (int it = tid; it < kExitBT * kExitCT; it += kExitThreads) {
-                const int sl = it / kExitCT, col = it - sl * kExitCT;
-                const bool valid = s0 + sl < B && c0 + col < C;
-                const float a = lg_s[it];
-                const float g = 0.5f * a * erfcf(-a * 0.70710678118654752f);
-                if constexpr (kBf16) {
-                    const float ea = kHidErr * sqrtf(1.0001f * (wn2[0][col] + wn2[1][col])) * un[sl] + fabsf(a) * 0x1p-20f;
+                // thread -> unit (class col = 32 (warp % 4) + lane: its tensor-memory lane; samples
+                // 4 (warp / 4) .. + 3: columns of D)
+                const int col = 32 * (warp & 3) + lane, sb = 4 * (warp >> 2);
+                uint32_t v[16] = {};
+                if (!failed) tmem_ld16(tmem + ((uint32_t)(32 * (warp & 3)) << 16), v);   // (failed: uniform)
+                const float wn = sqrtf(1.0001f * (wn2[0][col] + wn2[1][col]));
+                // the second term of the error scale: n = dim / 16 accumulation steps (kHidErr), plus
+                // the bias addition and the float32 evaluation of a
+                const float a_rel = 0x1p-20f + (float)((dim + 15) / 16) * 0x1p-23f;
+                uint16_t *ho = reinterpret_cast<uint16_t *>(p.hidden_out);
+                uint16_t hb[4];
+                F2 ax[4];            // exact pre-activations of this thread's flagged units
+                unsigned fl = 0;     // its units near a rounding midpoint (bit i: sample sb + i)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int sl = sb + i;
+                    const bool valid = s0 + sl < B && c0 + col < C && !failed;
+                    const float a = __uint_as_float(warp >= 4 ? v[4 + i] : v[i]) + bias_s[col];
+                    const float g = 0.5f * a * erfcf(-a * 0.70710678118654752f);
+                    const float ea = kHidErr * wn * un[sl] + fabsf(a) * a_rel;
                     const float eg = 1.13f * ea + fabsf(g) * 0x1p-16f;
                     const float mid = __uint_as_float((__float_as_uint(g) & 0xFFFF0000u) | 0x8000u);
                     const bool exact = valid && !(isfinite(g) && fabsf(g - mid) > eg);
-                    uint16_t hb = __bfloat16_as_ushort(__float2bfloat16_rn(g));
-                    // the units near a rounding midpoint, one at a time by the whole warp
+                    hb[i] = __bfloat16_as_ushort(__float2bfloat16_rn(g));
+                    ax[i] = {0.0f, 0.0f};
+                    if (exact) fl |= 1u << i;
+                    // their exact dot products, one at a time by the whole warp
                     for (unsigned mask = __ballot_sync(0xFFFFFFFFu, exact); mask; mask &= mask - 1) {
                         const int src = __ffs(mask) - 1;
                         const int scol = __shfl_sync(0xFFFFFFFFu, col, src);
-                        const uint16_t e = hidden_exact_bf16_warp(
-                            reinterpret_cast<const __nv_bfloat16 *>(p.head.weight) + (size_t)(c0 + scol) * dim,
-                            reinterpret_cast<const __nv_bfloat16 *>(u_s + (size_t)sl * u_stride), dim,
-                            p.head.bias[c0 + scol]);
-                        if (lane == src) hb = e;
+                        const F2 e = hidden_dot_exact_warp(
+                            resident ? w_region : nullptr, scol,
+                            reinterpret_cast<const __nv_bfloat16 *>(p.head.weight) + (size_t)(c0 + scol) * dim, base,
+                            sl, dim, bias_s[scol]);
+                        if (lane == src) ax[i] = e;
                     }
-                    if (valid) reinterpret_cast<uint16_t *>(ho)[(size_t)(s0 + sl) * C + c0 + col] = hb;
-                } else {
-                    if (valid) ho[(size_t)(s0 + sl) * C + c0 + col] = from_float<T>(g);
+                }
+                // their GELU, every thread its own (the double-precision fallback then runs once per
+                // unit, not once per lane of a warp)
+                for (unsigned m = fl; m; m &= m - 1) {
+                    const int i = __ffs(m) - 1;
+                    const F2 x = i == 0 ? ax[0] : i == 1 ? ax[1] : i == 2 ? ax[2] : ax[3];
+                    const uint16_t e = gelu_exact_bf16(x);
+                    hb[0] = i == 0 ? e : hb[0];
+                    hb[1] = i == 1 ? e : hb[1];
+                    hb[2] = i == 2 ? e : hb[2];
+                    hb[3] = i == 3 ? e : hb[3];
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    if (s0 + sb + i < B && c0 + col < C && !failed) ho[(size_t)(s0 + sb + i) * C + c0 + col] = hb[i];
+            } else if (warp < 4 && !failed) {
+                // logits (+ bias) into shared memory over the ring: warp w < 4 reads the lanes
+                // (classes) 32w.. of D
+                uint32_t v[16];
+                tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16), v);
+                const int cls = warp * 32 + lane;
+#pragma unroll
+                for (int n = 0; n < kExitBT; ++n)
+                    lg_s[n * kExitCT + cls] = (c0 + cls < C) ? __uint_as_float(v[n]) + bias_s[cls] : -INFINITY;
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncthreads();
+            if (warp == 0)
+                asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kExitTmemCols)
+                             : "memory");
+        } else {
+            float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};   // 4 classes of sample `warp`
+            exit_gemm<T>(p, u_s, w_region, c0, dim, C, n_k, acc);
+            exit_logits_f32(lg_s, bias_s, acc, c0, C);
+            __syncthreads();
+            if (p.out_mode == 1) {   // hidden layer: GELU in float32
+                for (int it = tid; it < kExitBT * kExitCT; it += kExitThreads) {
+                    const int sl = it / kExitCT, col = it - sl * kExitCT;
+                    const float a = lg_s[it];
+                    if (s0 + sl < B && c0 + col < C)
+                        reinterpret_cast<float *>(p.hidden_out)[(size_t)(s0 + sl) * C + c0 + col] =
+                            0.5f * a * erfcf(-a * 0.70710678118654752f);
                 }
             }
-        } else {
+        }
+        if (p.out_mode == 0) {
+            if (!failed) exit_stage_logits(p, lg_s, s0, c0, B, C);
             // ---- partial softmax of this class tile: warp -> sample ------------------------
             const int sl = warp, s = s0 + sl;
             float m = -INFINITY;
@@ -458,7 +637,9 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
             }
 #pragma unroll
             for (int o = 16; o >= 1; o >>= 1) z += __shfl_xor_sync(0xFFFFFFFFu, z, o);
-            if (lane == 0 && s < B) p.partials[(size_t)s * p.n_ctile + ct] = make_float2(m, z);
+            // a tile whose product timed out sends z = -1: no decision for its samples
+            if (lane == 0 && s < B)
+                p.partials[(size_t)s * p.n_ctile + ct] = failed ? make_float2(0.0f, -1.0f) : make_float2(m, z);
         }
     }
     if (p.out_mode == 1) return;   // no softmax across the tiles of a hidden layer
@@ -475,26 +656,34 @@ __global__ void __launch_bounds__(kExitThreads) k_exit(ExitParams p) {
         const int s = s0 + warp;
         if (s < B) {
             float m = -INFINITY;
-            for (int q = lane; q < p.n_ctile; q += 32) m = fmaxf(m, __ldcg(&p.partials[(size_t)s * p.n_ctile + q]).x);
-#pragma unroll
-            for (int o = 16; o >= 1; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
-            float z = 0.0f;
+            bool bad = false;
             for (int q = lane; q < p.n_ctile; q += 32) {
                 const float2 pz = __ldcg(&p.partials[(size_t)s * p.n_ctile + q]);
-                z += pz.y * expf(pz.x - m);
+                m = fmaxf(m, pz.x);
+                bad = bad || pz.y < 0.0f;
             }
 #pragma unroll
-            for (int o = 16; o >= 1; o >>= 1) z += __shfl_xor_sync(0xFFFFFFFFu, z, o);
-            const float c = 1.0f / z;   // max_k softmax = exp(l_max - l_max) / sum
-            const bool ex = c >= p.head.tau;
-            if (lane == 0) {
-                p.exit_mask[s] = ex ? 1 : 0;
-                if (p.max_prob) p.max_prob[s] = c;
-                if (!isfinite(m)) raise_status(p.status, FUSION_DEV_NONFINITE);
+            for (int o = 16; o >= 1; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+            if (!__any_sync(0xFFFFFFFFu, bad)) {   // else a product timed out: no decision (status raised)
+                float z = 0.0f;
+                for (int q = lane; q < p.n_ctile; q += 32) {
+                    const float2 pz = __ldcg(&p.partials[(size_t)s * p.n_ctile + q]);
+                    z += pz.y * expf(pz.x - m);
+                }
+#pragma unroll
+                for (int o = 16; o >= 1; o >>= 1) z += __shfl_xor_sync(0xFFFFFFFFu, z, o);
+                const float c = 1.0f / z;   // max_k softmax = exp(l_max - l_max) / sum
+                const bool ex = c >= p.head.tau;
+                if (lane == 0) {
+                    p.exit_mask[s] = ex ? 1 : 0;
+                    if (p.max_prob) p.max_prob[s] = c;
+                    if (!isfinite(m)) raise_status(p.status, FUSION_DEV_NONFINITE);
+                }
+                if (ex && p.logits && p.lg_tmp)   // logits only for the samples that exit
+                    for (int col = lane; col < p.head.classes; col += 32)
+                        p.logits[(size_t)s * p.head.classes + col] =
+                            __ldcg(&p.lg_tmp[(size_t)s * p.head.classes + col]);
             }
-            if (ex && p.logits && p.lg_tmp)   // logits only for the samples that exit
-                for (int col = lane; col < p.head.classes; col += 32)
-                    p.logits[(size_t)s * p.head.classes + col] = __ldcg(&p.lg_tmp[(size_t)s * p.head.classes + col]);
         }
     }
     if (tid == 0) p.counters[bt] = 0;
@@ -528,17 +717,6 @@ __device__ __forceinline__ float to_float(__nv_bfloat16 v) { return __bfloat162f
 // D[128 classes][16 samples] in tensor memory; float32: cp.async stages and FFMA.  No global
 // atomics unless the plan kernel's work runs here (batches above the fused-plan bound).
 // ---------------------------------------------------------------------------
-constexpr uint32_t kExitWStage = kExitCT * 128u;     // one stage: kExitCT rows x 64 bf16 dims
-
-// Byte offset of 16-byte chunk c (8 bf16 dims) of row r in the bf16 cluster kernel's u tile:
-// K-blocks of 64 dims, each [16 rows][128 bytes] with chunk j of row r at j ^ (r % 8), the
-// K-major, 128-byte-swizzled layout of a tcgen05 operand (8-row groups 1024 bytes apart).
-__device__ __forceinline__ uint32_t u_tc_off(int r, int c) {
-    return (uint32_t)(c >> 3) * 2048u + (uint32_t)r * 128u + ((uint32_t)((c & 7) ^ (r & 7)) << 4);
-}
-constexpr uint32_t kExitTmemCols = 32;   // D: 128 classes (lanes) x 16 samples (columns)
-constexpr int kExitClMaxW = 16;          // most weight stages of the bf16 cluster kernel
-constexpr size_t kExitClBudget = 112 * 1024;   // its dynamic shared memory bound (two CTAs per SM)
 
 template <typename T>
 struct ExitClSmem {
@@ -787,61 +965,16 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
     if constexpr (kBf16) asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
     cl.sync();   // all LayerNorm rows are in every CTA's shared memory
 
-    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-    float acc2[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};   // float32: 4 classes of sample `warp`
     if (active) {
         if constexpr (kBf16) {
-            // ---- D[128 classes][16 samples] = W_tile u^T on tcgen05, issued by one thread: per
-            // 64-dim chunk, wait for its weight stage, four MMAs (K = 16), commit; a stage is
-            // refilled by TMA once its MMAs completed.  Every wait is bounded; after a failure
-            // the copies and products in flight are waited for before anything else runs.
+            // ---- D[128 classes][16 samples] = W_tile u^T on tcgen05 (exit_tc_product) ----------
             const uint32_t tmem = tmem_base;
-            if (tid == 0) {
-                const int nk = (dim + 63) / 64;
-                const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(16 >> 3) << 17) | (8u << 24);
-                const uint32_t ub = smem_addr(base);
-                const int nws = L::w_stages(dim);
-                bool okw = true;
-                int waited = 0, issued = 0, loaded = nws;
-                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                for (int kc = 0; kc < nk; ++kc) {
-                    const int st = kc % nws;
-                    const uint32_t ph = (uint32_t)(kc / nws) & 1u;
-                    if (!mbar_wait(smem_addr(&wbar[st]), ph)) {
-                        okw = false;
-                        break;
-                    }
-                    waited = kc + 1;
-                    const uint32_t a0 = smem_addr(w_region + (size_t)st * kExitWStage), b0 = ub + (uint32_t)kc * 2048u;
-                    const int kw = min(64, dim - kc * 64);
-                    for (int k = 0; k * 16 < kw; ++k)
-                        umma_bf16(tmem, sw128_desc(a0 + k * 32), sw128_desc(b0 + k * 32), idesc, (kc | k) ? 1u : 0u);
-                    umma_commit(smem_addr(&wempty[st]));
-                    issued = kc + 1;
-                    if (kc + nws < nk) {   // the tile is not resident: refill this stage
-                        if (!mbar_wait(smem_addr(&wempty[st]), ph)) {
-                            okw = false;
-                            break;
-                        }
-                        mbar_expect_tx(smem_addr(&wbar[st]), kExitWStage);
-                        tma_load_2d(smem_addr(w_region + (size_t)st * kExitWStage), &wmap, (kc + nws) * 64, c0,
-                                    smem_addr(&wbar[st]));
-                        loaded = kc + nws + 1;
-                    }
-                }
-                if (okw) {
-                    umma_commit(smem_addr(&wdone));
-                    okw = mbar_wait(smem_addr(&wdone), 0u);
-                }
-                if (!okw) {
-                    for (int q = waited; q < loaded; ++q)
-                        (void)mbar_wait(smem_addr(&wbar[q % nws]), (uint32_t)(q / nws) & 1u);
-                    if (issued > 0)
-                        (void)mbar_wait(smem_addr(&wempty[(issued - 1) % nws]), (uint32_t)((issued - 1) / nws) & 1u);
-                    raise_status(p.status, FUSION_DEV_TIMEOUT);
-                }
-                s_wfail = okw ? 0 : 1;
-            }
+            if (tid == 0)
+                s_wfail = exit_tc_product(&wmap, tmem, smem_addr(base), smem_addr(w_region), dim, L::w_stages(dim), c0,
+                                          wbar, wempty, &wdone, p.status)
+                              ? 0
+                              : 1;
             __syncthreads();
             // the product is done: a programmatic dependent (the fused stage's per-sample kernel)
             // may start its prologue now; it reads nothing of ours before this grid completes
@@ -863,8 +996,9 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
                 asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kExitTmemCols)
                              : "memory");
         } else {
-            exit_gemm<T>(p, u_s, w_region, c0, dim, C, n_k, acc, acc2);
-            exit_logits<T>(p, lg_s, bias_s, acc, acc2, s0, c0, B, C);
+            exit_gemm<T>(p, u_s, w_region, c0, dim, C, n_k, acc);
+            exit_logits_f32(lg_s, bias_s, acc, c0, C);
+            __syncthreads();
         }
         // partial softmax of this class tile, warp -> sample slots warp, warp + 8, ...; to every
         // CTA of the cluster (a tile whose product timed out sends z = -1: no decision)
@@ -945,24 +1079,56 @@ __global__ void __launch_bounds__(kExitThreads) k_exit_cl(const __grid_constant_
 }  // namespace
 
 size_t exit_smem_bytes(int dtype, int dim) {
-    return dtype == FUSION_BF16 ? ExitSmem<__nv_bfloat16>::total(dim) : ExitSmem<float>::total(dim);
+    return dtype == FUSION_BF16 ? ExitTcSmem::total(dim) : ExitSmem<float>::total(dim);
 }
+
+namespace {
+// bf16: the head weights [C][dim] as TMA boxes of 64 dims x 128 classes, 128-byte swizzle (the
+// tcgen05 A operand); rows past C read as zero.  float32: no map (the kernels use cp.async).
+cudaError_t head_weight_map(int dtype, const ExitParams &p, CUtensorMap *wmap) {
+    *wmap = CUtensorMap{};
+    if (dtype != FUSION_BF16) return cudaSuccess;
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    cuuint64_t dims[2] = {(cuuint64_t)p.dim, (cuuint64_t)p.head.classes};
+    cuuint64_t strides[1] = {(cuuint64_t)p.dim * 2};
+    cuuint32_t box[2] = {64, (cuuint32_t)kExitCT};
+    cuuint32_t estr[2] = {1, 1};
+    if (enc(wmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(p.head.weight), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+        return cudaErrorInvalidValue;
+    return cudaSuccess;
+}
+
+// The general kernel; pdl: as a programmatic dependent of the kernel before it on the stream.
+template <typename T>
+cudaError_t launch_exit_general(const ExitParams &p, cudaStream_t s, bool pdl) {
+    CUtensorMap wmap;
+    cudaError_t e = head_weight_map(sizeof(T) == 2 ? FUSION_BF16 : FUSION_F32, p, &wmap);
+    if (e != cudaSuccess) return e;
+    const size_t smem = exit_smem_bytes(sizeof(T) == 2 ? FUSION_BF16 : FUSION_F32, p.dim);
+    e = cudaFuncSetAttribute(k_exit<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(p.n_ctile, p.n_btile);
+    cfg.blockDim = dim3(kExitThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, k_exit<T>, wmap, p);
+}
+}  // namespace
 
 template <typename T>
 cudaError_t launch_exit_cluster(const ExitParams &p, cudaStream_t s) {
-    CUtensorMap wmap{};
-    if (sizeof(T) == 2) {   // the head weights [C][dim] as boxes of 128 classes x 64 dims
-        EncodeTiledFn enc = encode_fn();
-        if (!enc) return cudaErrorNotSupported;
-        cuuint64_t dims[2] = {(cuuint64_t)p.dim, (cuuint64_t)p.head.classes};
-        cuuint64_t strides[1] = {(cuuint64_t)p.dim * 2};
-        cuuint32_t box[2] = {64, (cuuint32_t)kExitCT};
-        cuuint32_t estr[2] = {1, 1};
-        if (enc(&wmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(p.head.weight), dims, strides, box, estr,
-                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
-                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-            return cudaErrorInvalidValue;
-    }
+    CUtensorMap wmap;
+    cudaError_t he = head_weight_map(sizeof(T) == 2 ? FUSION_BF16 : FUSION_F32, p, &wmap);
+    if (he != cudaSuccess) return he;
     const size_t smem = ExitClSmem<T>::total(p.dim);
     cudaError_t e = cudaFuncSetAttribute(k_exit_cl<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
@@ -990,42 +1156,14 @@ cudaError_t launch_exit(int dtype, const ExitParams &p, cudaStream_t s) {
     // 1024 classes); larger heads take the kernel with a global last-CTA merge
     if (p.n_ctile <= kExitClMaxTiles && p.in_mode == 0 && !p.skip_ln && p.out_mode == 0)
         return dtype == FUSION_BF16 ? launch_exit_cluster<__nv_bfloat16>(p, s) : launch_exit_cluster<float>(p, s);
-    const size_t smem = exit_smem_bytes(dtype, p.dim);
-    const dim3 grid(p.n_ctile, p.n_btile);
-    if (dtype == FUSION_BF16) {
-        cudaError_t e = cudaFuncSetAttribute(k_exit<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        k_exit<__nv_bfloat16><<<grid, kExitThreads, smem, s>>>(p);
-    } else {
-        cudaError_t e = cudaFuncSetAttribute(k_exit<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        k_exit<float><<<grid, kExitThreads, smem, s>>>(p);
-    }
-    return cudaGetLastError();
+    return dtype == FUSION_BF16 ? launch_exit_general<__nv_bfloat16>(p, s, false) : launch_exit_general<float>(p, s, false);
 }
 
 // The general kernel as a programmatic dependent launch: its CTAs may start as the previous
-// kernel on the stream finishes and wait for its results after issuing their weight loads.
+// kernel on the stream triggers or finishes and wait for its results after issuing their
+// weight loads.
 cudaError_t launch_exit_pdl(int dtype, const ExitParams &p, cudaStream_t s) {
-    const size_t smem = exit_smem_bytes(dtype, p.dim);
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(p.n_ctile, p.n_btile);
-    cfg.blockDim = dim3(kExitThreads);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    if (dtype == FUSION_BF16) {
-        cudaError_t e = cudaFuncSetAttribute(k_exit<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        return cudaLaunchKernelEx(&cfg, k_exit<__nv_bfloat16>, p);
-    }
-    cudaError_t e = cudaFuncSetAttribute(k_exit<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    return cudaLaunchKernelEx(&cfg, k_exit<float>, p);
+    return dtype == FUSION_BF16 ? launch_exit_general<__nv_bfloat16>(p, s, true) : launch_exit_general<float>(p, s, true);
 }
 
 namespace {

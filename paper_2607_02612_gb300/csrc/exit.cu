@@ -229,7 +229,9 @@ __device__ __forceinline__ void exit_stage_logits(const ExitParams &p, const flo
 // partial sums of mixed signs the k-th is typically about sqrt(16 k / dim) ||w|| ||u|| / sqrt(dim),
 // and even n errors of one sign at that size sum to about (sqrt(n) / 6) 2^-23 ||w|| ||u||, below
 // 2^-22 ||w|| ||u|| up to dim = 1024.  Where the products share a sign, the partial sums grow
-// monotonically up to |a|: the second term, n 2^-23 |a|, covers that case.
+// monotonically up to |a|: the second term, n 2^-23 |a|, covers that case.  A typical-case scale,
+// not a worst-case bound: rows whose partial sums rise to about sum |w u| / 2 and then cancel can
+// exceed it if the accumulator truncates (about 2x at dim = 1024 in a model of the accumulation).
 constexpr float kHidErr = 0x1p-22f;
 
 // The exact pre-activation a = w . u + b1 of one hidden unit, by a whole warp: exact bf16 x bf16
